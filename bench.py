@@ -1,0 +1,367 @@
+"""Benchmark of the PRCR revisit path (rebind + inject) on GB300.
+
+One step = one call of the whole path over one batch: the plan kernel
+(positions, slots) and the fused gather / M-RoPE rebind / inject kernel, for
+every selected token x layer x KV head of every sequence in the batch.
+
+Default workload: the largest one (16-frame 16x32x32 video per sequence,
+4096 revisited tokens per sequence in 3 revisits, batch 32, 36 layers, 8 KV
+heads, head_dim 128, paged cache with block 16): 38.65 GB moved per step,
+far larger than L2, so no flush is needed between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the CPU oracle on bounded samples
+
+Prints one JSON line (rank 0). Under torchrun (N > 1) every rank runs its own
+full batch on its own GPU (weak scaling, no collective on the data path);
+the step time is the maximum over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import dataclasses
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "rebind+inject GB/s (read+write)"
+UNIT = "GB/s"
+SPEC_HBM_GBS = 8000.0
+
+# DRAM traffic (read + write bytes) of one rebind launch on the default
+# workload, from an ncu capture; valid only for the kernel source it was
+# measured on (its sha256 prefix), reported as null otherwise.
+TRAFFIC = {}
+
+
+def _sha(path):
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["prcr", "reference"], default="prcr")
+    ap.add_argument("--workload", default="stress")
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-check", action="store_true", help="skip the pre-timing parity check")
+    return ap.parse_args()
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    """Maximum of a per-rank float over all ranks (identity at world 1)."""
+    if world == 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ----------------------------------------------------------------------------
+# clocks during the timed region
+# ----------------------------------------------------------------------------
+class Clocks:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-f", self.path], stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        pw = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows), "power_w_max": max(pw) if pw else None}
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+# ----------------------------------------------------------------------------
+# the CPU oracle on a bounded sample
+# ----------------------------------------------------------------------------
+def sample_batch(wl, n_layers: int, n_tokens=None, device="cpu"):
+    """A bounded sample of the workload: its first sequence (same grids,
+    selection recipe and value distribution) with n_layers layers, optionally
+    cut to the first n_tokens selected tokens (one revisit), on the host."""
+    from workloads import make_batch
+    import torch
+    b = make_batch(dataclasses.replace(wl, n_seqs=1, n_layers=n_layers), device=device)
+    if device != "cpu":
+        b = dataclasses.replace(b, **{f: getattr(b, f).cpu() for f in (
+            "store_k", "store_v", "coords", "seq_rev_off", "rev_tok_off", "idx", "p_txt",
+            "cache_len_in")})
+    if n_tokens is not None and n_tokens < b.total_k:
+        b = dataclasses.replace(b, idx=b.idx[:n_tokens].clone(),
+                                rev_tok_off=torch.tensor([0, n_tokens], dtype=torch.int32),
+                                seq_rev_off=torch.tensor([0, 1], dtype=torch.int32))
+    return b
+
+
+def oracle_step(batch):
+    """Time the oracle's whole call on the batch (positions, gather, rebind,
+    value copy) on the host; returns seconds."""
+    import numpy as np
+    import torch
+    from oracle import prcr_oracle as O
+    wl = batch.wl
+    kb = batch.store_k.view(torch.int16).numpy()
+    vb = batch.store_v.view(torch.int16).numpy()
+    t0 = time.perf_counter()
+    out = O.rebind_inject(kb, vb, batch.coords.numpy(), batch.seq_rev_off.numpy(),
+                          batch.rev_tok_off.numpy(), batch.idx.numpy(), batch.p_txt.numpy(),
+                          batch.cache_len_in.numpy(), wl.head_dim, wl.sections, wl.theta, wl.L)
+    dt = time.perf_counter() - t0
+    assert np.isfinite(out["k_hat"]).all()
+    return dt
+
+
+def describe_sample(wl, batch):
+    return (f"sequence 0 of '{wl.name}': {batch.total_k} selected tokens in {batch.n_revisits} "
+            f"revisit(s) x {batch.wl.n_layers} of {wl.n_layers} layers x {wl.n_kv_heads} KV heads "
+            f"({batch.algorithmic_bytes() / 1e6:.1f} MB algorithmic); numpy float64, one thread")
+
+
+def cpu_baseline(wl, n_layers: int, device="cpu"):
+    batch = sample_batch(wl, n_layers, device=device)
+    t = oracle_step(batch)
+    nbytes = batch.algorithmic_bytes()
+    return dict(value=nbytes / t / 1e9, unit=UNIT, cores=1, kind="oracle",
+                sample=describe_sample(wl, batch), seconds=t)
+
+
+# ----------------------------------------------------------------------------
+# reference arm: the oracle as it stands, timed on the host cores
+# ----------------------------------------------------------------------------
+REF_TOKENS = 512  # tokens of one revisit, one layer, per reference step
+
+
+def run_reference(args):
+    world, rank, local = dist_env()
+    if rank != 0:
+        return
+    from workloads import get
+    wl = get(args.workload)
+    batch = sample_batch(wl, 1, n_tokens=REF_TOKENS)
+    for _ in range(args.warmup):
+        oracle_step(batch)
+    times = [oracle_step(batch) for _ in range(args.steps)]
+    t = sum(times)
+    nbytes = batch.algorithmic_bytes() * args.steps
+    value = nbytes / t / 1e9
+    line = dict(metric=METRIC, value=value, unit=UNIT, n_gpus=args.gpus, steps=args.steps,
+                warmup=args.warmup, ms_per_step=1e3 * t / args.steps, higher_is_better=True,
+                scaling="weak", vs_baseline=None, dtype="f64", data="synthetic",
+                config=dict(workload=wl.name, sample_per_step=describe_sample(wl, batch)),
+                impl="reference",
+                cpu_baseline=dict(kind="oracle", cores=1, value=value, unit=UNIT,
+                                  sample=describe_sample(wl, batch)),
+                e2e=dict(value=value, unit=UNIT, h2d_bytes_per_step=0, d2h_bytes_per_step=0),
+                gpu_launches=0)
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------
+# GPU arm
+# ----------------------------------------------------------------------------
+def run_gpu(args):
+    import torch
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+
+    from paper_2606_26631_gb300 import _build
+    if not _build.up_to_date():
+        if rank == 0:
+            _build.build()
+        barrier(world)
+    sys.path.insert(0, os.path.join(ROOT, "tests"))
+    import parity_util as pu
+    from workloads import get, make_batch
+
+    wl = get(args.workload)
+    batch = make_batch(wl, device=dev, seed=rank)
+    rv = pu.make_revisit(batch)
+    nbytes = batch.algorithmic_bytes()
+
+    # correctness gate before timing: positions/slots everywhere, rows on samples
+    rv.run()
+    torch.cuda.synchronize()
+    if rv.status_value() != 0:
+        raise RuntimeError(f"device status {rv.status_value():#x}")
+    check = None
+    if not args.no_check:
+        pl = pu.oracle_plan(batch)
+        pu.check_plan(rv, pl)
+        import numpy as np
+        seqs = sorted({0, wl.n_seqs // 2, wl.n_seqs - 1})
+        toks = np.nonzero(np.isin(pl["seq"], np.asarray(seqs)))[0]
+        layers = sorted({0, wl.n_layers // 2, wl.n_layers - 1})
+        e = pu.check_rows(batch, rv, pl, toks, layers)
+        check = dict(k_max_err=e["max_err"], k_max_rel=e["max_rel"], rows_checked=e["n"],
+                     positions_slots_bit_exact=True, v_bit_exact=True)
+
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        rv.run_plan()
+        rv.run_apply()
+    torch.cuda.synchronize()
+
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    barrier(world)
+    torch.cuda.synchronize()
+    with Clocks(local) as clk:
+        for e0, e1, e2 in ev:
+            e0.record(stream)
+            rv.run_plan()
+            e1.record(stream)
+            rv.run_apply()
+            e2.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    step_ms = [e0.elapsed_time(e2) for e0, _, e2 in ev]
+    apply_ms = [e1.elapsed_time(e2) for _, e1, e2 in ev]
+    plan_ms = [e0.elapsed_time(e1) for e0, e1, _ in ev]
+    total_s = sum(step_ms) / 1e3
+    total_s = max_over_ranks(total_s, world, dev)
+    value = nbytes * world * K / total_s / 1e9
+    ms_per_step = 1e3 * total_s / K
+
+    # end to end through the public call, host buffers, copies inside the timed region
+    for _ in range(2):
+        rv.run_from_host()
+    barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(args.e2e_steps):
+        st = rv.run_from_host()
+        if st != 0:
+            raise RuntimeError(f"device status {st:#x}")
+    e2e_s = max_over_ranks(time.perf_counter() - t0, world, dev)
+    e2e_value = nbytes * world * args.e2e_steps / e2e_s / 1e9
+
+    peak, peak_kind = measured_peaks()
+    apply_avg_s = statistics.mean(apply_ms) / 1e3
+    achieved = nbytes / apply_avg_s / 1e9
+    src_sha = _sha(os.path.join(ROOT, "paper_2606_26631_gb300", "csrc", "prcr_rebind.cu"))
+    traffic = TRAFFIC.get((wl.name, src_sha))
+    roof = dict(bound="hbm", achieved=achieved, peak=peak, unit="GB/s", frac=achieved / peak,
+                traffic=traffic, kernel="rebind_kernel", peak_kind=f"{peak_kind} copy (hbm_gbs)",
+                bytes_per_launch=nbytes, avg_launch_us=1e6 * apply_avg_s)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(wl, 8, device=dev)
+
+    if rank == 0:
+        R = batch.n_revisits
+        line = dict(
+            metric=METRIC, value=value, unit=UNIT, n_gpus=world, steps=K, warmup=args.warmup,
+            ms_per_step=ms_per_step, higher_is_better=True, scaling="weak", vs_baseline=None,
+            dtype="f32", io_dtype="bf16", data="synthetic",
+            config=dict(workload=wl.name, n_layers=wl.n_layers, n_kv_heads=wl.n_kv_heads,
+                        head_dim=wl.head_dim, sections=list(wl.sections), batch=wl.n_seqs,
+                        tokens=batch.total_k, revisits=R, cache=f"{wl.cache}/{wl.block_size}",
+                        L=wl.L, bytes_per_step=nbytes,
+                        l2="inputs larger than L2 (no flush): each step moves %.2f GB" % (nbytes / 1e9)),
+            pct_of_hbm_measured=100.0 * value / peak, pct_of_hbm_spec_8tbs=100.0 * value / SPEC_HBM_GBS,
+            us_per_revisit=1e3 * ms_per_step / R,
+            token_layers_per_s=batch.total_k * wl.n_layers * world * K / total_s,
+            plan_us_avg=1e3 * statistics.mean(plan_ms),
+            roofline=roof, cpu_baseline=cpu,
+            e2e=dict(value=e2e_value, unit=UNIT, h2d_bytes_per_step=rv.h2d_bytes(),
+                     d2h_bytes_per_step=rv.d2h_bytes(), steps=args.e2e_steps),
+            gpu_launches=2 * K, clocks=clk.summary(), parity=check)
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

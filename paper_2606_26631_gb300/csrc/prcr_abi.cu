@@ -1,0 +1,335 @@
+// extern "C" entry points of libprcr.so: argument checks, launch planning
+// and the two-kernel revisit path (plan, then rebind + inject).
+#include <cmath>
+#include <cstdint>
+#include <map>
+#include <mutex>
+#include <tuple>
+
+#include "prcr_internal.h"
+
+namespace prcr {
+namespace {
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline bool aligned4(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; }
+inline bool aligned8(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 7u) == 0; }
+inline bool mult8(int64_t s) { return s >= 0 && (s & 7) == 0; }
+
+int check_cfg(const prcr_rope_cfg* c) {
+    if (!c) return PRCR_EINVAL;
+    const int D = c->head_dim;
+    if (c->n_layers < 1 || c->n_kv_heads < 1 || D < 16 || D > PRCR_MAX_HEAD_DIM || (D & 15))
+        return PRCR_EINVAL;
+    if (int64_t(c->n_kv_heads) * D > PRCR_MAX_ROW_ELEMS) return PRCR_EINVAL;
+    if (c->sections[0] < 0 || c->sections[1] < 0 || c->sections[2] < 0 ||
+        c->sections[0] + c->sections[1] + c->sections[2] != D / 2)
+        return PRCR_EINVAL;
+    if (c->layout != PRCR_LAYOUT_SECTIONED && c->layout != PRCR_LAYOUT_INTERLEAVED)
+        return PRCR_EINVAL;
+    if (c->reserved != 0) return PRCR_EINVAL;
+    if (!(c->theta > 1.0) || !std::isfinite(c->theta)) return PRCR_EINVAL;
+    return PRCR_OK;
+}
+
+int check_store(const prcr_rope_cfg* c, const prcr_store_desc* s) {
+    if (!s || !s->k || !s->v || !s->coords) return PRCR_EINVAL;
+    const int64_t row = int64_t(c->n_kv_heads) * c->head_dim;
+    if (s->n_seqs < 1 || s->n_tokens < 1) return PRCR_EINVAL;
+    if (s->token_stride < row || s->layer_stride < 0 || s->seq_stride < 0) return PRCR_EINVAL;
+    if (s->coord_seq_stride < 3 * int64_t(s->n_tokens) && s->n_seqs > 1) return PRCR_EINVAL;
+    if (!aligned16(s->k) || !aligned16(s->v) || !aligned4(s->coords)) return PRCR_EALIGN;
+    if (!mult8(s->seq_stride) || !mult8(s->layer_stride) || !mult8(s->token_stride))
+        return PRCR_EALIGN;
+    return PRCR_OK;
+}
+
+int check_cache(const prcr_rope_cfg* c, const prcr_cache_desc* k) {
+    if (!k || !k->k || !k->v) return PRCR_EINVAL;
+    const int64_t row = int64_t(c->n_kv_heads) * c->head_dim;
+    if (k->slot_stride < row || k->layer_stride < 0 || k->n_seqs < 1) return PRCR_EINVAL;
+    if (!aligned16(k->k) || !aligned16(k->v)) return PRCR_EALIGN;
+    if (!mult8(k->layer_stride) || !mult8(k->slot_stride)) return PRCR_EALIGN;
+    if (k->kind == PRCR_CACHE_CONTIGUOUS) {
+        if (k->max_slots < 0 || k->seq_stride < 0) return PRCR_EINVAL;
+        if (!mult8(k->seq_stride)) return PRCR_EALIGN;
+    } else if (k->kind == PRCR_CACHE_PAGED) {
+        if (!k->block_table || k->block_size < 1 || k->bt_stride < 0 || k->n_blocks < 0 ||
+            k->block_stride < 0)
+            return PRCR_EINVAL;
+        if (!aligned4(k->block_table)) return PRCR_EALIGN;
+        if (!mult8(k->block_stride)) return PRCR_EALIGN;
+    } else {
+        return PRCR_EINVAL;
+    }
+    return PRCR_OK;
+}
+
+int check_call(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+               const prcr_cache_desc* cache, const prcr_revisit_batch* b,
+               const prcr_outputs* o, int32_t mode, int32_t L, int32_t flags, void* ws,
+               size_t ws_bytes) {
+    int rc = check_cfg(cfg);
+    if (rc) return rc;
+    if ((rc = check_store(cfg, store))) return rc;
+    if ((rc = check_cache(cfg, cache))) return rc;
+    if (!b || !o) return PRCR_EINVAL;
+    if (mode < PRCR_MODE_PCR || mode > PRCR_MODE_LPA) return PRCR_EINVAL;
+    if (L < 0 || (flags & ~PRCR_FLAG_DEGENERATE_CENTER)) return PRCR_EINVAL;
+    if (b->n_seqs < 0 || b->n_revisits < 0 || b->total_k < 0 || b->total_k > INT32_MAX)
+        return PRCR_EINVAL;
+    if (b->n_seqs == 0) return (b->n_revisits == 0 && b->total_k == 0) ? PRCR_OK : PRCR_EINVAL;
+    if (b->n_seqs > store->n_seqs || b->n_seqs > cache->n_seqs) return PRCR_EINVAL;
+    if (!b->seq_rev_off || !b->rev_tok_off || !b->p_txt || !b->cache_len_in) return PRCR_EINVAL;
+    if (b->total_k > 0 && !b->idx) return PRCR_EINVAL;
+    if (!o->cache_len_out || !o->next_pos_out || !o->status) return PRCR_EINVAL;
+    if (static_cast<const void*>(o->cache_len_out) == static_cast<const void*>(b->cache_len_in))
+        return PRCR_EINVAL;
+    if (!aligned4(b->seq_rev_off) || !aligned4(b->rev_tok_off) || !aligned4(b->cache_len_in) ||
+        !aligned8(b->p_txt) || (b->idx && !aligned4(b->idx)) || !aligned4(o->cache_len_out) ||
+        !aligned8(o->next_pos_out) || !aligned4(o->status) ||
+        (o->pos_out && !aligned8(o->pos_out)) || (o->slot_out && !aligned4(o->slot_out)))
+        return PRCR_EALIGN;
+    if (b->total_k > 0) {
+        if (!ws || ws_bytes < workspace_bytes(b->total_k)) return PRCR_EWORKSPACE;
+        if (!aligned16(ws)) return PRCR_EALIGN;
+    }
+    return PRCR_OK;
+}
+
+PlanArgs make_plan_args(const prcr_store_desc* store, const prcr_cache_desc* cache,
+                        const prcr_revisit_batch* b, const prcr_outputs* o, int32_t mode,
+                        int32_t L, int32_t flags, void* ws) {
+    PlanArgs a = {};
+    a.coords = store->coords;
+    a.coord_seq_stride = store->coord_seq_stride;
+    a.store_seq_stride = store->seq_stride;
+    a.store_token_stride = store->token_stride;
+    a.n_tokens = store->n_tokens;
+    a.cache_kind = cache->kind;
+    a.block_size = cache->kind == PRCR_CACHE_PAGED ? cache->block_size : 1;
+    a.bt_stride = cache->bt_stride;
+    a.n_blocks = cache->n_blocks;
+    a.max_slots = cache->max_slots;
+    a.cache_seq_stride = cache->seq_stride;
+    a.block_stride = cache->block_stride;
+    a.slot_stride = cache->slot_stride;
+    a.block_table = cache->block_table;
+    a.seq_rev_off = b->seq_rev_off;
+    a.rev_tok_off = b->rev_tok_off;
+    a.idx = b->idx;
+    a.p_txt = b->p_txt;
+    a.cache_len_in = b->cache_len_in;
+    a.n_seqs = b->n_seqs;
+    a.n_revisits = b->n_revisits;
+    a.total_k = b->total_k;
+    a.cache_len_out = o->cache_len_out;
+    a.next_pos_out = o->next_pos_out;
+    a.pos_out = o->pos_out;
+    a.slot_out = o->slot_out;
+    a.status = o->status;
+    a.plan = plan_view(ws, b->total_k);
+    a.mode = mode;
+    a.L = L;
+    a.flags = flags;
+    return a;
+}
+
+// Occupancy of the rebind kernel per (device, block, smem), cached.
+int blocks_per_sm(int dev, int block, size_t smem) {
+    static std::mutex mu;
+    static std::map<std::tuple<int, int, size_t>, int> cache;
+    const auto key = std::make_tuple(dev, block, smem);
+    {
+        std::lock_guard<std::mutex> g(mu);
+        auto it = cache.find(key);
+        if (it != cache.end()) return it->second;
+    }
+    int n = 0;
+    if (rebind_blocks_per_sm(block, smem, &n) != cudaSuccess || n < 1) n = 1;
+    std::lock_guard<std::mutex> g(mu);
+    cache[key] = n;
+    return n;
+}
+
+int sm_count(int dev) {
+    static std::mutex mu;
+    static std::map<int, int> cache;
+    {
+        std::lock_guard<std::mutex> g(mu);
+        auto it = cache.find(dev);
+        if (it != cache.end()) return it->second;
+    }
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
+        n = 1;
+    std::lock_guard<std::mutex> g(mu);
+    cache[dev] = n;
+    return n;
+}
+
+int do_rebind(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+              const prcr_cache_desc* cache, const prcr_revisit_batch* b, const prcr_outputs* o,
+              void* ws, cudaStream_t stream) {
+    if (b->total_k == 0) return PRCR_OK;
+    RebindArgs a = {};
+    a.store_k = static_cast<const uint16_t*>(store->k);
+    a.store_v = static_cast<const uint16_t*>(store->v);
+    a.cache_k = static_cast<uint16_t*>(cache->k);
+    a.cache_v = static_cast<uint16_t*>(cache->v);
+    a.store_layer_stride = store->layer_stride;
+    a.cache_layer_stride = cache->layer_stride;
+    const PlanView pv = plan_view(ws, b->total_k);
+    a.plan_src = pv.src;
+    a.plan_dst = pv.dst;
+    a.plan_pos = pv.pos;
+    a.status = o->status;
+    a.total_k = b->total_k;
+    a.n_layers = cfg->n_layers;
+    a.head_dim = cfg->head_dim;
+    a.layout = cfg->layout;
+    a.sec_t = cfg->sections[0];
+    a.sec_h = cfg->sections[1];
+    a.sec_w = cfg->sections[2];
+    const int P = cfg->head_dim / 2;
+    for (int i = 0; i < P; ++i)
+        a.inv_freq[i] = std::pow(cfg->theta, -2.0 * double(i) / double(cfg->head_dim));
+
+    // One thread per (token, head, 16-byte vector of the first half row).
+    const int lanes = cfg->n_kv_heads * (cfg->head_dim / 16);
+    int T = kRebindTargetThreads / lanes;
+    if (T < 1) T = 1;
+    const int block = T * lanes;
+    const size_t smem = size_t(2) * T * P * sizeof(float);
+    a.lanes = lanes;
+    a.tok_per_cta = T;
+
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return PRCR_ECUDA;
+    const int64_t tiles = (b->total_k + T - 1) / T;
+    const int64_t target = int64_t(sm_count(dev)) * blocks_per_sm(dev, block, smem) * 4;
+    int64_t groups = 1;
+    if (tiles < target) groups = (target + tiles - 1) / tiles;
+    if (groups > cfg->n_layers) groups = cfg->n_layers;
+    if (groups > 65535) groups = 65535;
+    const int G = int((cfg->n_layers + groups - 1) / groups);
+    groups = (cfg->n_layers + G - 1) / G;
+    a.layers_per_cta = G;
+    if (tiles > INT32_MAX) return PRCR_EINVAL;
+    const dim3 grid(unsigned(tiles), unsigned(groups), 1);
+    return launch_rebind(a, grid, block, smem, stream) == cudaSuccess ? PRCR_OK : PRCR_ECUDA;
+}
+
+int do_plan(const prcr_store_desc* store, const prcr_cache_desc* cache,
+            const prcr_revisit_batch* b, const prcr_outputs* o, int32_t mode, int32_t L,
+            int32_t flags, void* ws, cudaStream_t stream) {
+    const PlanArgs a = make_plan_args(store, cache, b, o, mode, L, flags, ws);
+    return launch_plan(a, stream) == cudaSuccess ? PRCR_OK : PRCR_ECUDA;
+}
+
+}  // namespace
+}  // namespace prcr
+
+using namespace prcr;
+
+extern "C" {
+
+size_t prcr_workspace_size(int64_t total_k) { return workspace_bytes(total_k); }
+
+int prcr_plan(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+              const prcr_cache_desc* cache, const prcr_revisit_batch* batch,
+              const prcr_outputs* out, int32_t mode, int32_t L, int32_t flags, void* workspace,
+              size_t workspace_bytes, void* stream) {
+    int rc = check_call(cfg, store, cache, batch, out, mode, L, flags, workspace, workspace_bytes);
+    if (rc || batch->n_seqs == 0) return rc;
+    return do_plan(store, cache, batch, out, mode, L, flags, workspace,
+                   static_cast<cudaStream_t>(stream));
+}
+
+int prcr_rebind_apply(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+                      const prcr_cache_desc* cache, const prcr_revisit_batch* batch,
+                      const prcr_outputs* out, int32_t mode, int32_t L, int32_t flags,
+                      void* workspace, size_t workspace_bytes, void* stream) {
+    int rc = check_call(cfg, store, cache, batch, out, mode, L, flags, workspace, workspace_bytes);
+    if (rc || batch->n_seqs == 0) return rc;
+    return do_rebind(cfg, store, cache, batch, out, workspace, static_cast<cudaStream_t>(stream));
+}
+
+int prcr_rebind_inject(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+                       const prcr_cache_desc* cache, const prcr_revisit_batch* batch,
+                       const prcr_outputs* out, int32_t mode, int32_t L, int32_t flags,
+                       void* workspace, size_t workspace_bytes, void* stream) {
+    int rc = check_call(cfg, store, cache, batch, out, mode, L, flags, workspace, workspace_bytes);
+    if (rc || batch->n_seqs == 0) return rc;
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    rc = do_plan(store, cache, batch, out, mode, L, flags, workspace, s);
+    if (rc) return rc;
+    return do_rebind(cfg, store, cache, batch, out, workspace, s);
+}
+
+int prcr_store_raw(const prcr_rope_cfg* cfg, const prcr_store_desc* store, int32_t seq,
+                   int32_t layer_begin, int32_t n_layers, int32_t m_begin, int32_t m_count,
+                   const void* k_src, const void* v_src, int64_t src_layer_stride,
+                   int64_t src_token_stride, const int32_t* coords_src, void* stream) {
+    int rc = check_cfg(cfg);
+    if (rc) return rc;
+    if ((rc = check_store(cfg, store))) return rc;
+    if (seq < 0 || seq >= store->n_seqs || layer_begin < 0 || n_layers < 0 ||
+        layer_begin + int64_t(n_layers) > cfg->n_layers || m_begin < 0 || m_count < 0 ||
+        m_begin + int64_t(m_count) > store->n_tokens)
+        return PRCR_EINVAL;
+    if (n_layers == 0 || m_count == 0) return PRCR_OK;
+    const int64_t row = int64_t(cfg->n_kv_heads) * cfg->head_dim;
+    if (!k_src || !v_src || src_token_stride < row || src_layer_stride < 0) return PRCR_EINVAL;
+    if (!aligned16(k_src) || !aligned16(v_src) || !mult8(src_layer_stride) ||
+        !mult8(src_token_stride) || (coords_src && !aligned4(coords_src)))
+        return PRCR_EALIGN;
+    StoreArgs a = {};
+    const int64_t base = int64_t(seq) * store->seq_stride + int64_t(layer_begin) * store->layer_stride +
+                         int64_t(m_begin) * store->token_stride;
+    a.dst_k = static_cast<uint16_t*>(store->k) + base;
+    a.dst_v = static_cast<uint16_t*>(store->v) + base;
+    a.src_k = static_cast<const uint16_t*>(k_src);
+    a.src_v = static_cast<const uint16_t*>(v_src);
+    a.dst_layer_stride = store->layer_stride;
+    a.dst_token_stride = store->token_stride;
+    a.src_layer_stride = src_layer_stride;
+    a.src_token_stride = src_token_stride;
+    a.n_layers = n_layers;
+    a.m_count = m_count;
+    a.row_vecs = int32_t(row / 8);
+    a.dst_coords = coords_src ? store->coords + int64_t(seq) * store->coord_seq_stride +
+                                    3 * int64_t(m_begin)
+                              : nullptr;
+    a.src_coords = coords_src;
+    return launch_store(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? PRCR_OK
+                                                                             : PRCR_ECUDA;
+}
+
+int64_t prcr_next_text_pos(int64_t p_txt, int64_t k_seq, int32_t mode) {
+    switch (mode) {
+        case PRCR_MODE_PCR:
+        case PRCR_MODE_ORIGINAL:
+        case PRCR_MODE_UIR:
+            return p_txt + 1;
+        case PRCR_MODE_LPA:
+            return p_txt + k_seq + 1;
+        default:
+            return INT64_MIN;
+    }
+}
+
+const char* prcr_error_string(int code) {
+    switch (code) {
+        case PRCR_OK: return "ok";
+        case PRCR_EINVAL: return "invalid argument";
+        case PRCR_EALIGN: return "pointer or stride not 16-byte aligned";
+        case PRCR_EWORKSPACE: return "workspace missing or too small";
+        case PRCR_ECUDA: return "CUDA launch failed";
+        default: return "unknown error";
+    }
+}
+
+int prcr_version(void) { return PRCR_VERSION; }
+
+}  // extern "C"

@@ -1,0 +1,127 @@
+// Internal interfaces between the C-ABI layer (prcr_abi.cu) and the kernels.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+#include "prcr.h"
+
+namespace prcr {
+
+constexpr int kPlanThreads = 256;
+constexpr int kMaxPairs = PRCR_MAX_HEAD_DIM / 2;
+constexpr int kRebindTargetThreads = 256;
+
+// Per-token plan left in the workspace by the plan kernel for the rebind
+// kernel (structure of arrays, each array 256-byte aligned).
+struct PlanView {
+    int64_t* src;  // element offset of the token's store row, layer term excluded
+    int64_t* dst;  // element offset of the token's cache row, layer term excluded; -1 = skip
+    double*  pos;  // reassigned (t, h, w)
+};
+
+inline size_t align256(size_t n) { return (n + 255) & ~size_t(255); }
+
+inline size_t workspace_bytes(int64_t total_k) {
+    if (total_k <= 0) return 0;
+    const size_t n = size_t(total_k);
+    return 2 * align256(8 * n) + align256(24 * n);
+}
+
+inline PlanView plan_view(void* ws, int64_t total_k) {
+    char* p = static_cast<char*>(ws);
+    const size_t n = size_t(total_k > 0 ? total_k : 0);
+    PlanView v;
+    v.src = reinterpret_cast<int64_t*>(p);
+    v.dst = reinterpret_cast<int64_t*>(p + align256(8 * n));
+    v.pos = reinterpret_cast<double*>(p + 2 * align256(8 * n));
+    return v;
+}
+
+struct PlanArgs {
+    // store
+    const int32_t* coords;
+    int64_t coord_seq_stride;
+    int64_t store_seq_stride;
+    int64_t store_token_stride;
+    int32_t n_tokens;
+    // cache
+    int32_t cache_kind;
+    int32_t block_size;
+    int32_t bt_stride;
+    int32_t n_blocks;
+    int32_t max_slots;
+    int64_t cache_seq_stride;
+    int64_t block_stride;
+    int64_t slot_stride;
+    const int32_t* block_table;
+    // batch
+    const int32_t* seq_rev_off;
+    const int32_t* rev_tok_off;
+    const int32_t* idx;
+    const int64_t* p_txt;
+    const int32_t* cache_len_in;
+    int32_t n_seqs;
+    int32_t n_revisits;
+    int64_t total_k;
+    // outputs
+    int32_t* cache_len_out;
+    int64_t* next_pos_out;
+    double* pos_out;
+    int32_t* slot_out;
+    uint32_t* status;
+    PlanView plan;
+    int32_t mode;
+    int32_t L;
+    int32_t flags;
+};
+
+struct RebindArgs {
+    const uint16_t* store_k;
+    const uint16_t* store_v;
+    uint16_t* cache_k;
+    uint16_t* cache_v;
+    int64_t store_layer_stride;
+    int64_t cache_layer_stride;
+    const int64_t* plan_src;
+    const int64_t* plan_dst;
+    const double* plan_pos;
+    const uint32_t* status;
+    int64_t total_k;
+    int32_t n_layers;
+    int32_t head_dim;
+    int32_t lanes;           // threads per token: n_kv_heads * head_dim / 16
+    int32_t tok_per_cta;     // T
+    int32_t layers_per_cta;  // G
+    int32_t layout;
+    int32_t sec_t;
+    int32_t sec_h;
+    int32_t sec_w;
+    double inv_freq[kMaxPairs];
+};
+
+struct StoreArgs {
+    uint16_t* dst_k;        // store row of (seq, layer_begin, m_begin)
+    uint16_t* dst_v;
+    const uint16_t* src_k;
+    const uint16_t* src_v;
+    int64_t dst_layer_stride;
+    int64_t dst_token_stride;
+    int64_t src_layer_stride;
+    int64_t src_token_stride;
+    int32_t n_layers;
+    int32_t m_count;
+    int32_t row_vecs;       // 16-byte vectors per row: H * D / 8
+    int32_t* dst_coords;    // store coordinates of (seq, m_begin), or null
+    const int32_t* src_coords;
+};
+
+cudaError_t launch_plan(const PlanArgs& a, cudaStream_t stream);
+cudaError_t launch_rebind(const RebindArgs& a, dim3 grid, int block, size_t smem,
+                          cudaStream_t stream);
+cudaError_t rebind_blocks_per_sm(int block, size_t smem, int* out);
+cudaError_t launch_store(const StoreArgs& a, cudaStream_t stream);
+
+}  // namespace prcr

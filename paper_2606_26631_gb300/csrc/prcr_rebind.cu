@@ -1,0 +1,207 @@
+// Rebind + inject kernel (Sec. 3.3, Eq. "cache_reconstruction" and
+// "active_cache"; Algorithm 1, the loop over layers).
+//
+// For every selected token, every layer and every KV head, the raw key row
+// is gathered from the store, rotated with M-RoPE at the token's reassigned
+// (t, h, w) position, rounded to bf16 and written to the token's cache slot;
+// the raw value row is copied unchanged next to it.
+//
+// Work layout. A CTA owns T tokens x G layers. Its threads first build the
+// float32 cos/sin of every (token, rotation pair) of the tile in shared
+// memory, once for all G layers and all heads: the angle is formed in float64
+// (position x inverse frequency), reduced modulo 2*pi in float64 (Cody-Waite
+// with a two-term 2*pi), and only then handed to float32 sincosf, so a
+// position near 3e4 keeps a ~1e-7 rad angle error instead of ~2e-3.
+// Then each thread owns one (token, head, 16-byte vector v) slot of the row:
+// it loads the 8 bf16 of the first half at v and the 8 bf16 of the second
+// half at v + D/2 (the rotate-half partners), for K and V, and walks the G
+// layers. Consecutive threads cover consecutive 16-byte vectors of a row, so
+// every warp-wide load and store is a set of whole 128-byte lines.
+//
+// The kernel is launched with programmatic dependent launch behind the plan
+// kernel and waits on it (griddepcontrol.wait) before touching the plan.
+#include <cmath>
+
+#include <cuda_bf16.h>
+
+#include "prcr_internal.h"
+
+namespace prcr {
+namespace {
+
+// 2*pi split into a float64 head and the float64 nearest to the remainder.
+constexpr double kTwoPiHi = 6.283185307179586;
+constexpr double kTwoPiLo = 2.4492935982947064e-16;
+constexpr double kInvTwoPi = 0.15915494309189535;
+
+__device__ __forceinline__ uint4 ld_stream(const uint16_t* p) {
+    uint4 r;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+                 : "l"(p));
+    return r;
+}
+
+__device__ __forceinline__ void st_row(uint16_t* p, const uint4& v) {
+    asm volatile("st.global.v4.u32 [%0], {%1, %2, %3, %4};"
+                 :
+                 : "l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+
+__device__ __forceinline__ float lo_f32(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float hi_f32(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+// Rotate four bf16 pairs held as (first-half word x, second-half word y):
+// x' = x cos - y sin, y' = y cos + x sin, float32, bf16 round-to-nearest-even.
+__device__ __forceinline__ void rotate_word(uint32_t x, uint32_t y, float c0, float s0, float c1,
+                                           float s1, uint32_t& xo, uint32_t& yo) {
+    const float x0 = lo_f32(x), x1 = hi_f32(x);
+    const float y0 = lo_f32(y), y1 = hi_f32(y);
+    const float a0 = fmaf(x0, c0, -y0 * s0);
+    const float a1 = fmaf(x1, c1, -y1 * s1);
+    const float b0 = fmaf(y0, c0, x0 * s0);
+    const float b1 = fmaf(y1, c1, x1 * s1);
+    xo = pack_bf16x2(a0, a1);
+    yo = pack_bf16x2(b0, b1);
+}
+
+__device__ __forceinline__ void rotate_vec(const uint4& x, const uint4& y, const float (&c)[8],
+                                           const float (&s)[8], uint4& xo, uint4& yo) {
+    rotate_word(x.x, y.x, c[0], s[0], c[1], s[1], xo.x, yo.x);
+    rotate_word(x.y, y.y, c[2], s[2], c[3], s[3], xo.y, yo.y);
+    rotate_word(x.z, y.z, c[4], s[4], c[5], s[5], xo.z, yo.z);
+    rotate_word(x.w, y.w, c[6], s[6], c[7], s[7], xo.w, yo.w);
+}
+
+__device__ __forceinline__ int pair_axis(int i, int layout, int st, int sh, int sw) {
+    if (layout == PRCR_LAYOUT_SECTIONED) return i < st ? 0 : (i < st + sh ? 1 : 2);
+    const int r = i % 3;
+    if (r == 1 && i < 3 * sh) return 1;
+    if (r == 2 && i < 3 * sw) return 2;
+    return 0;
+}
+
+__global__ void __launch_bounds__(512) rebind_kernel(const __grid_constant__ RebindArgs a) {
+    extern __shared__ float smem[];
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (*reinterpret_cast<const volatile uint32_t*>(a.status) & PRCR_ST_CSR) return;
+
+    const int D = a.head_dim;
+    const int P = D >> 1;
+    const int T = a.tok_per_cta;
+    float* cos_s = smem;
+    float* sin_s = smem + T * P;
+    const int64_t tok0 = int64_t(blockIdx.x) * T;
+
+    for (int q = threadIdx.x; q < T * P; q += blockDim.x) {
+        const int t = q / P;
+        const int i = q - t * P;
+        const int64_t tok = tok0 + t;
+        float c = 1.0f, s = 0.0f;
+        if (tok < a.total_k) {
+            const int ax = pair_axis(i, a.layout, a.sec_t, a.sec_h, a.sec_w);
+            const double ang = a.plan_pos[3 * tok + ax] * a.inv_freq[i];
+            const double k = rint(ang * kInvTwoPi);
+            double r = fma(-k, kTwoPiHi, ang);
+            r = fma(-k, kTwoPiLo, r);
+            sincosf(float(r), &s, &c);
+        }
+        cos_s[q] = c;
+        sin_s[q] = s;
+    }
+    __syncthreads();
+
+    const int lanes = a.lanes;
+    const int t = threadIdx.x / lanes;
+    const int lane = threadIdx.x - t * lanes;
+    const int64_t tok = tok0 + t;
+    if (t >= T || tok >= a.total_k) return;
+    const int64_t dst = a.plan_dst[tok];
+    if (dst < 0) return;
+    const int64_t src = a.plan_src[tok];
+
+    const int vph = D >> 4;  // 16-byte vectors per half row of one head
+    const int h = lane / vph;
+    const int v = lane - h * vph;
+    const int half = P;      // elements between rotate-half partners
+    const int64_t off = int64_t(h) * D + v * 8;
+
+    float c[8], s[8];
+    {
+        const float4* cp = reinterpret_cast<const float4*>(cos_s + t * P + v * 8);
+        const float4* sp = reinterpret_cast<const float4*>(sin_s + t * P + v * 8);
+        const float4 c0 = cp[0], c1 = cp[1], s0 = sp[0], s1 = sp[1];
+        c[0] = c0.x; c[1] = c0.y; c[2] = c0.z; c[3] = c0.w;
+        c[4] = c1.x; c[5] = c1.y; c[6] = c1.z; c[7] = c1.w;
+        s[0] = s0.x; s[1] = s0.y; s[2] = s0.z; s[3] = s0.w;
+        s[4] = s1.x; s[5] = s1.y; s[6] = s1.z; s[7] = s1.w;
+    }
+
+    const int l0 = blockIdx.y * a.layers_per_cta;
+    const int l1 = min(l0 + a.layers_per_cta, a.n_layers);
+    const int64_t sls = a.store_layer_stride;
+    const int64_t cls = a.cache_layer_stride;
+    const uint16_t* sk = a.store_k + src + int64_t(l0) * sls + off;
+    const uint16_t* sv = a.store_v + src + int64_t(l0) * sls + off;
+    uint16_t* ck = a.cache_k + dst + int64_t(l0) * cls + off;
+    uint16_t* cv = a.cache_v + dst + int64_t(l0) * cls + off;
+
+    int l = l0;
+    for (; l + 2 <= l1; l += 2) {
+        const uint4 k0a = ld_stream(sk), k1a = ld_stream(sk + half);
+        const uint4 v0a = ld_stream(sv), v1a = ld_stream(sv + half);
+        const uint4 k0b = ld_stream(sk + sls), k1b = ld_stream(sk + sls + half);
+        const uint4 v0b = ld_stream(sv + sls), v1b = ld_stream(sv + sls + half);
+        uint4 o0, o1;
+        rotate_vec(k0a, k1a, c, s, o0, o1);
+        st_row(ck, o0);
+        st_row(ck + half, o1);
+        st_row(cv, v0a);
+        st_row(cv + half, v1a);
+        rotate_vec(k0b, k1b, c, s, o0, o1);
+        st_row(ck + cls, o0);
+        st_row(ck + cls + half, o1);
+        st_row(cv + cls, v0b);
+        st_row(cv + cls + half, v1b);
+        sk += 2 * sls; sv += 2 * sls; ck += 2 * cls; cv += 2 * cls;
+    }
+    if (l < l1) {
+        const uint4 k0 = ld_stream(sk), k1 = ld_stream(sk + half);
+        const uint4 v0 = ld_stream(sv), v1 = ld_stream(sv + half);
+        uint4 o0, o1;
+        rotate_vec(k0, k1, c, s, o0, o1);
+        st_row(ck, o0);
+        st_row(ck + half, o1);
+        st_row(cv, v0);
+        st_row(cv + half, v1);
+    }
+}
+
+}  // namespace
+
+cudaError_t rebind_blocks_per_sm(int block, size_t smem, int* out) {
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, rebind_kernel, block, smem);
+}
+
+cudaError_t launch_rebind(const RebindArgs& a, dim3 grid, int block, size_t smem,
+                          cudaStream_t stream) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(block, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, rebind_kernel, a);
+}
+
+}  // namespace prcr

@@ -160,6 +160,12 @@ def selections(wl: Workload, rng) -> List[List[np.ndarray]]:
             _, _, rows, cols, _ = layout[0]
             r0 = int(rng.integers(0, rows - nr + 1)); c0 = int(rng.integers(0, cols - nc + 1))
             revs.append(_rect_ids(layout, 0, 0, 1, r0, nr, c0, nc))
+        elif wl.selection == "random":
+            # extra = (min revisits, max revisits, min K, max K): distinct random tokens
+            rmin, rmax, kmin, kmax = wl.extra
+            for _ in range(int(rng.integers(rmin, rmax + 1))):
+                k = min(int(rng.integers(kmin, kmax + 1)), wl.n_tokens)
+                revs.append(rng.choice(wl.n_tokens, size=k, replace=False).astype(np.int32))
         else:
             raise ValueError(wl.selection)
         out.append(revs)
