@@ -56,6 +56,8 @@ def parse():
     ap.add_argument("--workload", default="stress")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-samples", type=int, default=8,
+                    help="sequences the CPU oracle baseline is timed on")
     ap.add_argument("--no-check", action="store_true", help="skip the pre-timing parity check")
     return ap.parse_args()
 
@@ -152,13 +154,13 @@ def measured_peaks():
 # ----------------------------------------------------------------------------
 # the CPU oracle on a bounded sample
 # ----------------------------------------------------------------------------
-def sample_batch(wl, n_layers: int, n_tokens=None, device="cpu"):
+def sample_batch(wl, n_layers: int, n_tokens=None, device="cpu", seed: int = 0):
     """A bounded sample of the workload: its first sequence (same grids,
     selection recipe and value distribution) with n_layers layers, optionally
     cut to the first n_tokens selected tokens (one revisit), on the host."""
     from workloads import make_batch
     import torch
-    b = make_batch(dataclasses.replace(wl, n_seqs=1, n_layers=n_layers), device=device)
+    b = make_batch(dataclasses.replace(wl, n_seqs=1, n_layers=n_layers), device=device, seed=seed)
     if device != "cpu":
         b = dataclasses.replace(b, **{f: getattr(b, f).cpu() for f in (
             "store_k", "store_v", "coords", "seq_rev_off", "rev_tok_off", "idx", "p_txt",
@@ -194,12 +196,21 @@ def describe_sample(wl, batch):
             f"({batch.algorithmic_bytes() / 1e6:.1f} MB algorithmic); numpy float64, one thread")
 
 
-def cpu_baseline(wl, n_layers: int, device="cpu"):
-    batch = sample_batch(wl, n_layers, device=device)
-    t = oracle_step(batch)
-    nbytes = batch.algorithmic_bytes()
-    return dict(value=nbytes / t / 1e9, unit=UNIT, cores=1, kind="oracle",
-                sample=describe_sample(wl, batch), seconds=t)
+def cpu_baseline(wl, n_layers: int, n_samples: int = 1, device="cpu"):
+    """The oracle's whole call timed on n_samples sequences drawn like the
+    workload's (seeds 0 .. n_samples-1), one sequence per call."""
+    total_t, total_b, batch = 0.0, 0, None
+    for s in range(n_samples):
+        batch = sample_batch(wl, n_layers, device=device, seed=s)
+        total_t += oracle_step(batch)
+        total_b += batch.algorithmic_bytes()
+        del batch
+    return dict(value=total_b / total_t / 1e9, unit=UNIT, cores=1, kind="oracle",
+                sample=(f"{n_samples} sequence(s) drawn like '{wl.name}' (seeds 0..{n_samples - 1}), "
+                        f"all selected tokens x {n_layers} of {wl.n_layers} layers x "
+                        f"{wl.n_kv_heads} KV heads, one sequence per oracle call "
+                        f"({total_b / 1e9:.2f} GB algorithmic); numpy float64, one thread"),
+                seconds=total_t)
 
 
 # ----------------------------------------------------------------------------
@@ -328,7 +339,7 @@ def run_gpu(args):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(wl, 8, device=dev)
+        cpu = cpu_baseline(wl, wl.n_layers, n_samples=args.cpu_samples, device=dev)
 
     if rank == 0:
         R = batch.n_revisits
