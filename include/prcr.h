@@ -205,6 +205,27 @@ PRCR_API int prcr_rebind_apply(const prcr_rope_cfg* cfg, const prcr_store_desc* 
                       const prcr_outputs* out, int32_t mode, int32_t L, int32_t flags,
                       void* workspace, size_t workspace_bytes, void* stream);
 
+/* prcr_rebind_inject_static - prcr_rebind_inject without a caller workspace.
+ * The paper has no counterpart to this call; it exists for callers that cannot
+ * allocate device memory themselves (a plugin whose host framework owns all
+ * device memory through its own pool, or a decode loop where cudaMalloc and
+ * cudaFree, which can synchronise the device, are not allowed). It allocates
+ * nothing: the per-token plan lives in a fixed array inside the library, of
+ * PRCR_STATIC_MAX_TOKENS tokens (2.5 MiB), held on every GPU that loads the
+ * library until the process exits. Inputs and outputs are passed and owned by
+ * the caller exactly as for prcr_rebind_inject, with the same results.
+ *  - total_k > PRCR_STATIC_MAX_TOKENS returns PRCR_EWORKSPACE, nothing enqueued.
+ *  - The first call on a device looks up the array's device address (set-up
+ *    done once per device); make that first call before any stream capture.
+ *  - Every call shares the one array: calls whose work overlaps on the GPU
+ *    (other streams, other host threads) race and must be serialised by the
+ *    caller. Nothing in the array needs to start at zero.                    */
+#define PRCR_STATIC_MAX_TOKENS 65536
+PRCR_API int prcr_rebind_inject_static(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+                                       const prcr_cache_desc* cache,
+                                       const prcr_revisit_batch* batch, const prcr_outputs* out,
+                                       int32_t mode, int32_t L, int32_t flags, void* stream);
+
 /* prcr_store_raw - fill the raw visual memory (Sec. 3.1, Eq. "raw_kv" and
  * "global_raw_memory"): copy pre-rotation K/V of tokens m_begin ..
  * m_begin+m_count-1, layers layer_begin .. layer_begin+n_layers-1 of sequence

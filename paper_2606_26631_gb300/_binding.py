@@ -25,7 +25,9 @@ LAYOUT_SECTIONED, LAYOUT_INTERLEAVED = 0, 1
 CACHE_CONTIGUOUS, CACHE_PAGED = 0, 1
 
 EXPORTS = ("prcr_workspace_size", "prcr_rebind_inject", "prcr_plan", "prcr_rebind_apply",
-           "prcr_store_raw", "prcr_next_text_pos", "prcr_error_string", "prcr_version")
+           "prcr_store_raw", "prcr_next_text_pos", "prcr_error_string", "prcr_version",
+           "prcr_rebind_inject_static")
+STATIC_MAX_TOKENS = 65536
 
 
 class RopeCfg(C.Structure):
@@ -79,6 +81,8 @@ def lib():
     for name in ("prcr_rebind_inject", "prcr_plan", "prcr_rebind_apply"):
         getattr(L, name).argtypes = call
         getattr(L, name).restype = C.c_int
+    L.prcr_rebind_inject_static.argtypes = call[:8] + [C.c_void_p]
+    L.prcr_rebind_inject_static.restype = C.c_int
     L.prcr_store_raw.argtypes = [P(RopeCfg), P(StoreDesc), C.c_int32, C.c_int32, C.c_int32,
                                  C.c_int32, C.c_int32, C.c_void_p, C.c_void_p, C.c_int64,
                                  C.c_int64, C.c_void_p, C.c_void_p]
@@ -242,6 +246,17 @@ def rebind_apply(cfg, store, cache, batch, out, mode=MODE_PCR, L=2, flags=0, wor
                  stream=None):
     """prcr_rebind_apply: the row-moving half, consuming a preceding prcr_plan."""
     return _call("prcr_rebind_apply", cfg, store, cache, batch, out, mode, L, flags, workspace, stream)
+
+
+def rebind_inject_static(cfg, store, cache, batch, out, mode=MODE_PCR, L=2, flags=0, stream=None):
+    """prcr_rebind_inject_static: the same call with the library's own fixed
+    scratch instead of a caller workspace (for callers that cannot allocate
+    device memory); at most STATIC_MAX_TOKENS selected tokens per call, and
+    calls must not overlap on the GPU."""
+    rc = lib().prcr_rebind_inject_static(C.byref(cfg), C.byref(store), C.byref(cache),
+                                         C.byref(batch), C.byref(out), int(mode), int(L),
+                                         int(flags), _stream(stream))
+    return _check(rc, "prcr_rebind_inject_static")
 
 
 def store_raw(cfg, store, seq: int, layer_begin: int, m_begin: int, k_src: torch.Tensor,

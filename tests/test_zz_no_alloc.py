@@ -1,0 +1,89 @@
+"""GPU test of prcr_rebind_inject_static, the allocation-free form of the call.
+
+Some callers cannot allocate device memory themselves (a plugin whose host
+framework owns all device memory through its own pool, or a decode loop where
+cudaMalloc/cudaFree, which may synchronise the device, are not allowed). For
+them the library keeps the per-token plan in its own fixed device array
+instead of a caller workspace. This test calls that entry point through the C
+ABI twice in a row, on two different workloads, and checks each result
+against the workspace-based prcr_rebind_inject on the same inputs: positions,
+slots, lengths and V bit for bit, K within the tolerance the parity tests use,
+every row neither call should write left untouched. It also checks that a
+batch above the array's capacity is refused before anything runs.
+
+The file name sorts last so that a run stopping at the first failure has run
+every other test before this one; it passes alone in a fresh process too.
+"""
+import ctypes as C
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+
+
+def _compare_with_workspace_call(name):
+    import paper_2606_26631_gb300 as prcr
+    import parity_util as pu
+    from workloads import get, make_batch
+
+    batch = make_batch(get(name), device=DEV)
+    pristine_k = batch.cache_k.clone()
+    pristine_v = batch.cache_v.clone()
+
+    ref = pu.make_revisit(batch)  # caller-provided workspace
+    ref.run()
+    torch.cuda.synchronize()
+
+    other = dataclasses.replace(batch, cache_k=pristine_k, cache_v=pristine_v)
+    st = pu.make_revisit(other)
+    prcr.rebind_inject_static(st.cfg, st.store, st.cache, st.batch, st.out, st.mode, st.L, st.flags)
+    torch.cuda.synchronize()
+
+    assert ref.status_value() == 0 and st.status_value() == 0
+    assert torch.equal(st.pos.view(torch.int64), ref.pos.view(torch.int64))
+    assert torch.equal(st.slot, ref.slot)
+    assert torch.equal(st.cache_len_out, ref.cache_len_out)
+    assert torch.equal(st.next_pos, ref.next_pos)
+    assert torch.equal(other.cache_v.view(torch.int16), batch.cache_v.view(torch.int16))
+
+    pl = pu.oracle_plan(batch)
+    tokens = np.arange(batch.total_k)
+    layers = range(batch.wl.n_layers)
+    k_raw = pu.bits(pu.raw_rows(batch, batch.store_k, tokens, pl, layers))
+    k_ref = pu.bits(pu.gather_cache(batch, batch.cache_k, tokens, pl, layers))
+    k_st = pu.bits(pu.gather_cache(other, other.cache_k, tokens, pl, layers))
+    from oracle import prcr_oracle as O
+    e = pu.k_error(k_st, O.bf16_bits_to_f64(k_ref), k_raw)
+    assert e["max_err"] <= pu.K_TOL, e
+    pu.check_untouched(other, pl)
+    return st
+
+
+def test_static_scratch_two_calls_in_a_row():
+    first = _compare_with_workspace_call("qwen25vl-7b")   # paged, 4093 tokens
+    second = _compare_with_workspace_call("qwen2vl-2b")   # contiguous, 259 tokens
+    assert first.batch.total_k != second.batch.total_k
+
+
+def test_static_scratch_refuses_oversized_batch():
+    import paper_2606_26631_gb300 as prcr
+    import parity_util as pu
+    from paper_2606_26631_gb300 import _binding as B
+    from workloads import get, make_batch
+
+    batch = make_batch(get("tiny"), device=DEV)
+    rv = pu.make_revisit(batch)
+    big = B.RevisitBatch.from_buffer_copy(rv.batch)
+    big.total_k = B.STATIC_MAX_TOKENS + 1
+    rc = prcr.lib().prcr_rebind_inject_static(C.byref(rv.cfg), C.byref(rv.store),
+                                              C.byref(rv.cache), C.byref(big), C.byref(rv.out),
+                                              0, 2, 0, None)
+    assert rc == B.EWORKSPACE
+    torch.cuda.synchronize()
+    assert rv.status_value() == 0
+    assert bool((batch.cache_k.view(torch.int16) == -1).all().item())
