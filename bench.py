@@ -59,6 +59,9 @@ def parse():
     ap.add_argument("--cpu-samples", type=int, default=8,
                     help="sequences the CPU oracle baseline is timed on")
     ap.add_argument("--no-check", action="store_true", help="skip the pre-timing parity check")
+    ap.add_argument("--graph", action="store_true",
+                    help="replay the step from a CUDA graph (for small, launch-bound workloads)")
+    ap.add_argument("--graph-inner", type=int, default=20, help="steps captured per graph")
     return ap.parse_args()
 
 
@@ -295,22 +298,54 @@ def run_gpu(args):
     torch.cuda.synchronize()
 
     K = args.steps
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
-           torch.cuda.Event(enable_timing=True)) for _ in range(K)]
-    barrier(world)
-    torch.cuda.synchronize()
-    with Clocks(local) as clk:
-        for e0, e1, e2 in ev:
-            e0.record(stream)
-            rv.run_plan()
-            e1.record(stream)
-            rv.run_apply()
-            e2.record(stream)
+    if args.graph:
+        # K steps as K / inner replays of a graph holding `inner` steps
+        inner = max(1, args.graph_inner)
+        K = max(inner, (K + inner - 1) // inner * inner)
+        g = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            rv.run()
+        stream.wait_stream(side)
         torch.cuda.synchronize()
-    barrier(world)
-    step_ms = [e0.elapsed_time(e2) for e0, _, e2 in ev]
-    apply_ms = [e1.elapsed_time(e2) for _, e1, e2 in ev]
-    plan_ms = [e0.elapsed_time(e1) for e0, e1, _ in ev]
+        with torch.cuda.graph(g):
+            for _ in range(inner):
+                rv.run()
+        for _ in range(3):
+            g.replay()
+        torch.cuda.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(K // inner)]
+        barrier(world)
+        torch.cuda.synchronize()
+        with Clocks(local) as clk:
+            for e0, e2 in ev:
+                e0.record(stream)
+                g.replay()
+                e2.record(stream)
+            torch.cuda.synchronize()
+        barrier(world)
+        step_ms = [e0.elapsed_time(e2) / inner for e0, e2 in ev for _ in range(inner)]
+        apply_ms = None
+        plan_ms = None
+    else:
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+               torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+        barrier(world)
+        torch.cuda.synchronize()
+        with Clocks(local) as clk:
+            for e0, e1, e2 in ev:
+                e0.record(stream)
+                rv.run_plan()
+                e1.record(stream)
+                rv.run_apply()
+                e2.record(stream)
+            torch.cuda.synchronize()
+        barrier(world)
+        step_ms = [e0.elapsed_time(e2) for e0, _, e2 in ev]
+        apply_ms = [e1.elapsed_time(e2) for _, e1, e2 in ev]
+        plan_ms = [e0.elapsed_time(e1) for e0, e1, _ in ev]
     total_s = sum(step_ms) / 1e3
     total_s = max_over_ranks(total_s, world, dev)
     value = nbytes * world * K / total_s / 1e9
@@ -329,12 +364,17 @@ def run_gpu(args):
     e2e_value = nbytes * world * args.e2e_steps / e2e_s / 1e9
 
     peak, peak_kind = measured_peaks()
-    apply_avg_s = statistics.mean(apply_ms) / 1e3
+    if apply_ms is not None:
+        apply_avg_s = statistics.mean(apply_ms) / 1e3
+        kernel = "rebind_kernel"
+    else:  # graph replay: only whole steps are timed
+        apply_avg_s = statistics.mean(step_ms) / 1e3
+        kernel = "plan_kernel + rebind_kernel (graph step)"
     achieved = nbytes / apply_avg_s / 1e9
     src_sha = _sha(os.path.join(ROOT, "paper_2606_26631_gb300", "csrc", "prcr_rebind.cu"))
     traffic = TRAFFIC.get((wl.name, src_sha))
     roof = dict(bound="hbm", achieved=achieved, peak=peak, unit="GB/s", frac=achieved / peak,
-                traffic=traffic, kernel="rebind_kernel", peak_kind=f"{peak_kind} copy (hbm_gbs)",
+                traffic=traffic, kernel=kernel, peak_kind=f"{peak_kind} copy (hbm_gbs)",
                 bytes_per_launch=nbytes, avg_launch_us=1e6 * apply_avg_s)
 
     cpu = None
@@ -355,7 +395,9 @@ def run_gpu(args):
             pct_of_hbm_measured=100.0 * value / peak, pct_of_hbm_spec_8tbs=100.0 * value / SPEC_HBM_GBS,
             us_per_revisit=1e3 * ms_per_step / R,
             token_layers_per_s=batch.total_k * wl.n_layers * world * K / total_s,
-            plan_us_avg=1e3 * statistics.mean(plan_ms),
+            plan_us_avg=1e3 * statistics.mean(plan_ms) if plan_ms else None,
+            timing="cuda graph, %d steps per replay" % args.graph_inner if args.graph
+            else "stream launches, events around each step and kernel",
             roofline=roof, cpu_baseline=cpu,
             e2e=dict(value=e2e_value, unit=UNIT, h2d_bytes_per_step=rv.h2d_bytes(),
                      d2h_bytes_per_step=rv.d2h_bytes(), steps=args.e2e_steps),

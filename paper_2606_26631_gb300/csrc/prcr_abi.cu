@@ -168,6 +168,30 @@ int sm_count(int dev) {
     return n;
 }
 
+// Layers each rebind CTA walks. Every CTA of a grid does the same work, so
+// the grid runs in ceil(waves) rounds of `slots` resident CTAs: pick the
+// group size whose waves are fullest (counting a short last group), charging
+// each CTA's cos/sin prologue as about a tenth of one layer's rows, and
+// prefer the larger group on ties. A grid that fits in one wave uses one
+// layer per CTA (shortest CTAs, lowest latency).
+int layers_per_cta(int64_t tiles, int n_layers, int64_t slots) {
+    if (tiles * n_layers <= slots) return 1;
+    int best = n_layers;
+    double best_eff = -1.0;
+    for (int G = n_layers; G >= 1; --G) {
+        const int64_t groups = (n_layers + G - 1) / G;
+        if (groups > 65535) break;
+        const double waves = double(tiles * groups) / double(slots);
+        const double eff = waves / std::ceil(waves) * double(n_layers) / double(groups * G) /
+                           (1.0 + 0.1 / G);
+        if (eff > best_eff + 1e-9) {
+            best = G;
+            best_eff = eff;
+        }
+    }
+    return best;
+}
+
 int do_rebind(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
               const prcr_cache_desc* cache, const prcr_revisit_batch* b, const prcr_outputs* o,
               void* ws, cudaStream_t stream) {
@@ -207,13 +231,9 @@ int do_rebind(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return PRCR_ECUDA;
     const int64_t tiles = (b->total_k + T - 1) / T;
-    const int64_t target = int64_t(sm_count(dev)) * blocks_per_sm(dev, block, smem) * 4;
-    int64_t groups = 1;
-    if (tiles < target) groups = (target + tiles - 1) / tiles;
-    if (groups > cfg->n_layers) groups = cfg->n_layers;
-    if (groups > 65535) groups = 65535;
-    const int G = int((cfg->n_layers + groups - 1) / groups);
-    groups = (cfg->n_layers + G - 1) / G;
+    const int64_t slots = int64_t(sm_count(dev)) * blocks_per_sm(dev, block, smem);
+    const int G = layers_per_cta(tiles, cfg->n_layers, slots);
+    const int64_t groups = (cfg->n_layers + G - 1) / G;
     a.layers_per_cta = G;
     if (tiles > INT32_MAX) return PRCR_EINVAL;
     const dim3 grid(unsigned(tiles), unsigned(groups), 1);

@@ -10,7 +10,7 @@
 
 namespace prcr {
 
-constexpr int kPlanThreads = 256;
+constexpr int kPlanThreads = 512;
 constexpr int kMaxPairs = PRCR_MAX_HEAD_DIM / 2;
 constexpr int kRebindTargetThreads = 256;
 

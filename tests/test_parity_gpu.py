@@ -284,3 +284,26 @@ def test_full_size(name, seqs, layers):
     e = pu.check_rows(batch, rv, pl, tokens, layers)
     print(name, e)
     pu.check_untouched(batch, pl)
+
+
+@pytest.mark.parametrize("name", ["tiny", "qwen25vl-7b"])
+def test_graph_replay_matches(name):
+    """The call captured in a CUDA graph (plan + PDL-launched rebind) and
+    replayed gives the oracle's results."""
+    import parity_util as pu
+    batch = make_batch(get(name), device=DEV)
+    rv = pu.make_revisit(batch)
+    rv.run()  # warm-up outside capture (first-call set-up)
+    torch.cuda.synchronize()
+    batch.cache_k.view(torch.int16).fill_(-1)
+    batch.cache_v.view(torch.int16).fill_(-1)
+    rv.pos.zero_(); rv.slot.zero_(); rv.next_pos.zero_(); rv.cache_len_out.zero_()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        rv.run()
+    g.replay()
+    g.replay()
+    torch.cuda.synchronize()
+    assert rv.status_value() == 0
+    pu.full_check(batch, rv)
