@@ -39,7 +39,10 @@ SPEC_HBM_GBS = 8000.0
 # DRAM traffic (read + write bytes) of one rebind launch on the default
 # workload, from an ncu capture; valid only for the kernel source it was
 # measured on (its sha256 prefix), reported as null otherwise.
-TRAFFIC = {}
+TRAFFIC = {
+    # profiles/rebind_kernel_stress_dram.md: 19,304,776,704 B read + 19,268,871,168 B written
+    ("stress", "6b40ef09c2644b48"): 38573647872,
+}
 
 
 def _sha(path):

@@ -240,6 +240,29 @@ PRCR_API int prcr_store_raw(const prcr_rope_cfg* cfg, const prcr_store_desc* sto
                    const void* k_src, const void* v_src, int64_t src_layer_stride,
                    int64_t src_token_stride, const int32_t* coords_src, void* stream);
 
+/* prcr_prefill_capture - build the raw visual memory during prefill
+ * (Sec. 3.1, Eq. "raw_kv" and "global_raw_memory") in the same pass that
+ * writes the model's ordinary cache entries for those tokens (Eq.
+ * "historical_position_bound_kv": key rotated at the original coordinate,
+ * value unchanged). Tokens m_begin .. m_begin+m_count-1, layers layer_begin ..
+ * layer_begin+n_layers-1 of sequence `seq`:
+ *   - the pre-rotation rows are read once from k_src / v_src (device bf16;
+ *     row of (layer i, token j) at i*src_layer_stride + j*src_token_stride),
+ *   - copied unchanged into the store, with coords_src (device int32
+ *     [m_count][3], original (t, h, w)) into the store's coordinates,
+ *   - and written as RoPE(k, p_m) and v into the cache at slots
+ *     slot_begin .. slot_begin+m_count-1 of sequence `seq` (contiguous or
+ *     paged through the block table).
+ * Host-checked ranges return PRCR_EINVAL; a slot beyond the capacity or an
+ * unmapped block sets PRCR_ST_CAPACITY / PRCR_ST_NO_BLOCK in *status (device
+ * word) and skips that token's cache rows (its store rows are still written). */
+PRCR_API int prcr_prefill_capture(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+                                  const prcr_cache_desc* cache, int32_t seq, int32_t layer_begin,
+                                  int32_t n_layers, int32_t m_begin, int32_t m_count,
+                                  int64_t slot_begin, const void* k_src, const void* v_src,
+                                  int64_t src_layer_stride, int64_t src_token_stride,
+                                  const int32_t* coords_src, uint32_t* status, void* stream);
+
 /* prcr_next_text_pos - host helper: the position the next text token takes
  * after a revisit appended k_seq tokens to a sequence whose latest text token
  * is at p_txt: p_txt + 1 for PCR, ORIGINAL and UIR (Sec. 3.2, Sec. 3.3);

@@ -16,6 +16,7 @@ What it computes (paper sections / equations):
 * Concatenation onto the existing decoder cache                  (Sec. 3.3, Eq. "active_cache")
 * Next text position p_txt + 1                                   (Sec. 3.2 and 3.3, before Eq. "decode_with_active_cache")
 * The position-bound historical key RoPE(k_raw, p_m)             (Sec. 2.3, Eq. "historical_position_bound_kv")
+* Prefill capture: raw rows kept + position-bound cache rows       (Sec. 3.1, Eq. "raw_kv", "global_raw_memory")
 
 Readings taken where the paper is silent (each is a named choice below):
 
@@ -230,6 +231,20 @@ def position_bound_keys(k_raw_bits, coords, head_dim, sections, theta,
     """Eq. "historical_position_bound_kv": k_tilde = RoPE(k_raw, p_m)."""
     return rebind_keys(k_raw_bits, np.asarray(coords, dtype=np.float64), head_dim, sections,
                        theta, layout)
+
+
+def prefill_capture(k_raw_bits, v_raw_bits, coords, head_dim, sections, theta,
+                    layout: int = LAYOUT_SECTIONED):
+    """Sec. 3.1: during prefill the raw projections of every visual token are
+    kept as they are (Eq. "raw_kv", "global_raw_memory") while the ordinary
+    cache receives the position-bound entries of Eq.
+    "historical_position_bound_kv" (key rotated at the original coordinate,
+    value unchanged). Inputs [M, ..., D] bf16 bit patterns and [M, 3] coords;
+    returns (store K bits, store V bits, cache K float64, cache V bits)."""
+    k_raw_bits = np.asarray(k_raw_bits)
+    v_raw_bits = np.asarray(v_raw_bits)
+    k_cache = position_bound_keys(k_raw_bits, coords, head_dim, sections, theta, layout)
+    return k_raw_bits.copy(), v_raw_bits.copy(), k_cache, v_raw_bits.copy()
 
 
 # ----------------------------------------------------------------------------

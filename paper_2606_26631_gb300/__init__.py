@@ -9,7 +9,7 @@ from ._binding import (  # noqa: F401
     CACHE_CONTIGUOUS, CACHE_PAGED, EXPORTS, FLAG_DEGENERATE_CENTER, LAYOUT_INTERLEAVED,
     LAYOUT_SECTIONED, MODE_LPA, MODE_ORIGINAL, MODE_PCR, MODE_UIR, ST_CAPACITY, ST_CSR,
     ST_IDX_RANGE, ST_NO_BLOCK, ST_POS_RANGE, PrcrError, cache_contiguous, cache_paged, lib,
-    next_text_pos, outputs, plan, rebind_apply, rebind_inject, rebind_inject_static,
+    next_text_pos, outputs, plan, prefill_capture, rebind_apply, rebind_inject, rebind_inject_static,
     revisit_batch, rope_cfg,
     store_desc, store_raw, version, workspace_size)
 from .revisit import Revisit  # noqa: F401

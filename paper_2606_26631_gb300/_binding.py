@@ -26,7 +26,7 @@ CACHE_CONTIGUOUS, CACHE_PAGED = 0, 1
 
 EXPORTS = ("prcr_workspace_size", "prcr_rebind_inject", "prcr_plan", "prcr_rebind_apply",
            "prcr_store_raw", "prcr_next_text_pos", "prcr_error_string", "prcr_version",
-           "prcr_rebind_inject_static")
+           "prcr_rebind_inject_static", "prcr_prefill_capture")
 STATIC_MAX_TOKENS = 65536
 
 
@@ -87,6 +87,11 @@ def lib():
                                  C.c_int32, C.c_int32, C.c_void_p, C.c_void_p, C.c_int64,
                                  C.c_int64, C.c_void_p, C.c_void_p]
     L.prcr_store_raw.restype = C.c_int
+    L.prcr_prefill_capture.argtypes = [P(RopeCfg), P(StoreDesc), P(CacheDesc), C.c_int32,
+                                       C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int64,
+                                       C.c_void_p, C.c_void_p, C.c_int64, C.c_int64, C.c_void_p,
+                                       C.c_void_p, C.c_void_p]
+    L.prcr_prefill_capture.restype = C.c_int
     L.prcr_next_text_pos.argtypes = [C.c_int64, C.c_int64, C.c_int32]
     L.prcr_next_text_pos.restype = C.c_int64
     L.prcr_error_string.argtypes = [C.c_int]
@@ -272,6 +277,24 @@ def store_raw(cfg, store, seq: int, layer_begin: int, m_begin: int, k_src: torch
                               k_src.data_ptr(), v_src.data_ptr(), k_src.stride(0), k_src.stride(1),
                               _ptr(coords_src), _stream(stream))
     return _check(rc, "prcr_store_raw")
+
+
+def prefill_capture(cfg, store, cache, seq: int, layer_begin: int, m_begin: int, slot_begin: int,
+                    k_src: torch.Tensor, v_src: torch.Tensor, coords_src: torch.Tensor,
+                    status: torch.Tensor, stream=None):
+    """prcr_prefill_capture: k_src / v_src are the prefill's pre-rotation rows
+    [n_layers, m_count, H, D] bf16 (row-contiguous); coords_src [m_count, 3] int32."""
+    _bf16(k_src, "k_src"); _bf16(v_src, "v_src")
+    if k_src.stride() != v_src.stride() or k_src.shape != v_src.shape:
+        raise ValueError("k_src and v_src must have the same shape and strides")
+    if coords_src.dtype != torch.int32 or not coords_src.is_contiguous():
+        raise TypeError("coords_src must be a contiguous int32 [m_count, 3] tensor")
+    rc = lib().prcr_prefill_capture(C.byref(cfg), C.byref(store), C.byref(cache), int(seq),
+                                    int(layer_begin), int(k_src.shape[0]), int(m_begin),
+                                    int(k_src.shape[1]), int(slot_begin), k_src.data_ptr(),
+                                    v_src.data_ptr(), k_src.stride(0), k_src.stride(1),
+                                    coords_src.data_ptr(), status.data_ptr(), _stream(stream))
+    return _check(rc, "prcr_prefill_capture")
 
 
 def next_text_pos(p_txt: int, k_seq: int, mode: int = MODE_PCR) -> int:

@@ -135,18 +135,22 @@ PlanArgs make_plan_args(const prcr_store_desc* store, const prcr_cache_desc* cac
     return a;
 }
 
-// Occupancy of the rebind kernel per (device, block, smem), cached.
-int blocks_per_sm(int dev, int block, size_t smem) {
+enum KernelId { kRebind = 0, kCapture = 1 };
+
+// Resident CTAs per SM of a kernel per (device, kernel, block, smem), cached.
+int blocks_per_sm(int dev, int block, size_t smem, int kernel = kRebind) {
     static std::mutex mu;
-    static std::map<std::tuple<int, int, size_t>, int> cache;
-    const auto key = std::make_tuple(dev, block, smem);
+    static std::map<std::tuple<int, int, int, size_t>, int> cache;
+    const auto key = std::make_tuple(dev, kernel, block, smem);
     {
         std::lock_guard<std::mutex> g(mu);
         auto it = cache.find(key);
         if (it != cache.end()) return it->second;
     }
     int n = 0;
-    if (rebind_blocks_per_sm(block, smem, &n) != cudaSuccess || n < 1) n = 1;
+    const cudaError_t e = kernel == kRebind ? rebind_blocks_per_sm(block, smem, &n)
+                                            : capture_blocks_per_sm(block, smem, &n);
+    if (e != cudaSuccess || n < 1) n = 1;
     std::lock_guard<std::mutex> g(mu);
     cache[key] = n;
     return n;
@@ -247,6 +251,69 @@ int do_plan(const prcr_store_desc* store, const prcr_cache_desc* cache,
     return launch_plan(a, stream) == cudaSuccess ? PRCR_OK : PRCR_ECUDA;
 }
 
+int do_capture(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+               const prcr_cache_desc* cache, int32_t seq, int32_t layer_begin, int32_t n_layers,
+               int32_t m_begin, int32_t m_count, int64_t slot_begin, const void* k_src,
+               const void* v_src, int64_t src_layer_stride, int64_t src_token_stride,
+               const int32_t* coords_src, uint32_t* status, cudaStream_t stream) {
+    CaptureArgs a = {};
+    const int64_t sbase = int64_t(seq) * store->seq_stride + int64_t(layer_begin) * store->layer_stride +
+                          int64_t(m_begin) * store->token_stride;
+    a.src_k = static_cast<const uint16_t*>(k_src);
+    a.src_v = static_cast<const uint16_t*>(v_src);
+    a.src_layer_stride = src_layer_stride;
+    a.src_token_stride = src_token_stride;
+    a.store_k = static_cast<uint16_t*>(store->k) + sbase;
+    a.store_v = static_cast<uint16_t*>(store->v) + sbase;
+    a.store_layer_stride = store->layer_stride;
+    a.store_token_stride = store->token_stride;
+    a.store_coords = store->coords + int64_t(seq) * store->coord_seq_stride + 3 * int64_t(m_begin);
+    a.coords = coords_src;
+    a.cache_k = static_cast<uint16_t*>(cache->k) + int64_t(layer_begin) * cache->layer_stride;
+    a.cache_v = static_cast<uint16_t*>(cache->v) + int64_t(layer_begin) * cache->layer_stride;
+    a.cache_layer_stride = cache->layer_stride;
+    a.cache_kind = cache->kind;
+    a.slot_stride = cache->slot_stride;
+    a.slot_begin = slot_begin;
+    if (cache->kind == PRCR_CACHE_CONTIGUOUS) {
+        a.cache_seq_off = int64_t(seq) * cache->seq_stride;
+        a.capacity = cache->max_slots;
+        a.block_size = 1;
+    } else {
+        a.bt_row = cache->block_table + int64_t(seq) * cache->bt_stride;
+        a.block_size = cache->block_size;
+        a.block_stride = cache->block_stride;
+        a.n_blocks = cache->n_blocks;
+        a.capacity = int64_t(cache->bt_stride) * cache->block_size;
+    }
+    a.status = status;
+    a.m_count = m_count;
+    a.n_layers = n_layers;
+    a.head_dim = cfg->head_dim;
+    a.layout = cfg->layout;
+    a.sec_t = cfg->sections[0];
+    a.sec_h = cfg->sections[1];
+    a.sec_w = cfg->sections[2];
+    const int P = cfg->head_dim / 2;
+    for (int i = 0; i < P; ++i)
+        a.inv_freq[i] = std::pow(cfg->theta, -2.0 * double(i) / double(cfg->head_dim));
+    const int lanes = cfg->n_kv_heads * (cfg->head_dim / 16);
+    int T = kRebindTargetThreads / lanes;
+    if (T < 1) T = 1;
+    const int block = T * lanes;
+    const size_t smem = size_t(2) * T * P * sizeof(float) + size_t(T) * sizeof(int64_t);
+    a.lanes = lanes;
+    a.tok_per_cta = T;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return PRCR_ECUDA;
+    const int64_t tiles = (int64_t(m_count) + T - 1) / T;
+    const int64_t slots = int64_t(sm_count(dev)) * blocks_per_sm(dev, block, smem, kCapture);
+    const int G = layers_per_cta(tiles, n_layers, slots);
+    a.layers_per_cta = G;
+    const dim3 grid(unsigned(tiles), unsigned((n_layers + G - 1) / G), 1);
+    return launch_capture(a, grid, block, smem, stream) == cudaSuccess ? PRCR_OK : PRCR_ECUDA;
+}
+
 }  // namespace
 }  // namespace prcr
 
@@ -324,6 +391,33 @@ int prcr_store_raw(const prcr_rope_cfg* cfg, const prcr_store_desc* store, int32
     a.src_coords = coords_src;
     return launch_store(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? PRCR_OK
                                                                              : PRCR_ECUDA;
+}
+
+int prcr_prefill_capture(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+                         const prcr_cache_desc* cache, int32_t seq, int32_t layer_begin,
+                         int32_t n_layers, int32_t m_begin, int32_t m_count, int64_t slot_begin,
+                         const void* k_src, const void* v_src, int64_t src_layer_stride,
+                         int64_t src_token_stride, const int32_t* coords_src, uint32_t* status,
+                         void* stream) {
+    int rc = check_cfg(cfg);
+    if (rc) return rc;
+    if ((rc = check_store(cfg, store))) return rc;
+    if ((rc = check_cache(cfg, cache))) return rc;
+    if (seq < 0 || seq >= store->n_seqs || seq >= cache->n_seqs || layer_begin < 0 ||
+        n_layers < 0 || layer_begin + int64_t(n_layers) > cfg->n_layers || m_begin < 0 ||
+        m_count < 0 || m_begin + int64_t(m_count) > store->n_tokens || slot_begin < 0)
+        return PRCR_EINVAL;
+    if (n_layers == 0 || m_count == 0) return PRCR_OK;
+    const int64_t row = int64_t(cfg->n_kv_heads) * cfg->head_dim;
+    if (!k_src || !v_src || !coords_src || !status || src_token_stride < row ||
+        src_layer_stride < 0)
+        return PRCR_EINVAL;
+    if (!aligned16(k_src) || !aligned16(v_src) || !mult8(src_layer_stride) ||
+        !mult8(src_token_stride) || !aligned4(coords_src) || !aligned4(status))
+        return PRCR_EALIGN;
+    return do_capture(cfg, store, cache, seq, layer_begin, n_layers, m_begin, m_count, slot_begin,
+                      k_src, v_src, src_layer_stride, src_token_stride, coords_src, status,
+                      static_cast<cudaStream_t>(stream));
 }
 
 int64_t prcr_next_text_pos(int64_t p_txt, int64_t k_seq, int32_t mode) {

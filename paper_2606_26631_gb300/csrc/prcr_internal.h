@@ -118,6 +118,46 @@ struct StoreArgs {
     const int32_t* src_coords;
 };
 
+struct CaptureArgs {
+    const uint16_t* src_k;      // token 0 of layer 0 of the prefill rows
+    const uint16_t* src_v;
+    int64_t src_layer_stride;
+    int64_t src_token_stride;
+    uint16_t* store_k;          // store row of (seq, layer_begin, m_begin)
+    uint16_t* store_v;
+    int64_t store_layer_stride;
+    int64_t store_token_stride;
+    int32_t* store_coords;      // store coordinates of (seq, m_begin)
+    const int32_t* coords;      // [m_count][3] original (t, h, w)
+    uint16_t* cache_k;          // cache base shifted to layer_begin
+    uint16_t* cache_v;
+    int64_t cache_layer_stride;
+    int64_t cache_seq_off;      // contiguous: seq * seq_stride
+    int64_t block_stride;
+    int64_t slot_stride;
+    int64_t capacity;           // slots of this sequence
+    int64_t slot_begin;
+    const int32_t* bt_row;      // paged: block-table row of the sequence
+    int32_t cache_kind;
+    int32_t block_size;
+    int32_t n_blocks;
+    uint32_t* status;
+    int32_t m_count;
+    int32_t n_layers;
+    int32_t head_dim;
+    int32_t lanes;
+    int32_t tok_per_cta;
+    int32_t layers_per_cta;
+    int32_t layout;
+    int32_t sec_t;
+    int32_t sec_h;
+    int32_t sec_w;
+    double inv_freq[kMaxPairs];
+};
+
+cudaError_t launch_capture(const CaptureArgs& a, dim3 grid, int block, size_t smem,
+                           cudaStream_t stream);
+cudaError_t capture_blocks_per_sm(int block, size_t smem, int* out);
 cudaError_t launch_plan(const PlanArgs& a, cudaStream_t stream);
 cudaError_t launch_rebind(const RebindArgs& a, dim3 grid, int block, size_t smem,
                           cudaStream_t stream);

@@ -372,10 +372,31 @@ def pin_original_mode_is_position_bound_cache(o):
         assert np.allclose(got["k_hat"][j, 0, 0], y, rtol=0, atol=1e-12)
 
 
+def pin_prefill_capture(o):
+    """The store keeps the raw rows bit for bit; the cache key is the textbook
+    rotation at the original coordinate (Eq. "historical_position_bound_kv")."""
+    rng = np.random.default_rng(29)
+    D, sec = 16, (2, 3, 3)
+    kb = rng.integers(0x3C00, 0x4100, size=(5, 2, D)).astype(np.uint16)
+    vb = rng.integers(0x3C00, 0x4100, size=(5, 2, D)).astype(np.uint16)
+    coords = np.array([(7, 20 + m, 30 - m) for m in range(5)])
+    sk, sv, ck, cv = o.prefill_capture(kb, vb, coords, D, sec, 1e6)
+    assert np.array_equal(sk, kb) and np.array_equal(sv, vb) and np.array_equal(cv, vb)
+    P = D // 2
+    for m in range(5):
+        for h in range(2):
+            x = [_bf16_value(v) for v in kb[m, h]]
+            for i in range(P):
+                axis = 0 if i < sec[0] else (1 if i < sec[0] + sec[1] else 2)
+                z = complex(x[i], x[i + P]) * cmath.exp(1j * coords[m, axis] * 1e6 ** (-2.0 * i / D))
+                assert abs(ck[m, h, i] - z.real) < 1e-12 and abs(ck[m, h, i + P] - z.imag) < 1e-12
+
+
 PINS = [pin_worked_rect4x4, pin_worked_rect2x2, pin_pcr_closed_forms, pin_degenerate_center,
         pin_other_modes, pin_plan_slots_and_continuity, pin_rope_closed_forms,
         pin_mrope_equal_axes_is_textbook, pin_mrope_sections, pin_rope_invariants,
-        pin_bf16_helpers, pin_brute_force_2x2, pin_original_mode_is_position_bound_cache]
+        pin_bf16_helpers, pin_brute_force_2x2, pin_original_mode_is_position_bound_cache,
+        pin_prefill_capture]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
