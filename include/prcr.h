@@ -263,6 +263,33 @@ PRCR_API int prcr_prefill_capture(const prcr_rope_cfg* cfg, const prcr_store_des
                                   int64_t src_layer_stride, int64_t src_token_stride,
                                   const int32_t* coords_src, uint32_t* status, void* stream);
 
+/* prcr_decode_attention - the first decode step over the active cache
+ * (Sec. 3.3, Eq. "decode_with_active_cache"): for every sequence b, layer l
+ * and query head h,
+ *   out[b][l][h] = softmax(RoPE(q[b][l][h], (p, p, p)) K^T / sqrt(D)) V,
+ * p = q_pos[b], over cache slots [0, seq_len[b]) of sequence b (contiguous, or
+ * paged through the block table), the revisited rows included. Query head h
+ * reads KV head h / (n_q_heads / n_kv_heads) (grouped-query attention).
+ *   q:       device bf16 [n_seqs][n_layers][n_q_heads][D] raw (pre-rotation)
+ *   q_pos:   device int64 [n_seqs]  (the next text position, e.g. next_pos_out)
+ *   seq_len: device int32 [n_seqs]  (e.g. cache_len_out); max_len >= every
+ *            seq_len is a host bound used for the split of the sequence axis
+ *   out:     device float32 [n_seqs][n_layers][n_q_heads][D]
+ * Limits: D in {64, 128, 256}; n_q_heads a multiple of n_kv_heads, at most 8
+ * query heads per KV head and n_q_heads * D <= PRCR_DECODE_MAX_Q_ELEMS.
+ * workspace: device, >= prcr_decode_workspace_size(...) bytes (0 when the
+ * sequence axis is not split), 16-byte aligned. A seq_len beyond the
+ * capacity sets PRCR_ST_CAPACITY (clamped); an unmapped block in range sets
+ * PRCR_ST_NO_BLOCK and its slots are left out of the softmax.              */
+#define PRCR_DECODE_MAX_Q_ELEMS 8192
+PRCR_API size_t prcr_decode_workspace_size(const prcr_rope_cfg* cfg, int32_t n_seqs,
+                                           int32_t n_q_heads, int64_t max_len);
+PRCR_API int prcr_decode_attention(const prcr_rope_cfg* cfg, const prcr_cache_desc* cache,
+                                   int32_t n_seqs, int32_t n_q_heads, const void* q,
+                                   const int64_t* q_pos, const int32_t* seq_len, int64_t max_len,
+                                   float* out, uint32_t* status, void* workspace,
+                                   size_t workspace_bytes, void* stream);
+
 /* prcr_next_text_pos - host helper: the position the next text token takes
  * after a revisit appended k_seq tokens to a sequence whose latest text token
  * is at p_txt: p_txt + 1 for PCR, ORIGINAL and UIR (Sec. 3.2, Sec. 3.3);

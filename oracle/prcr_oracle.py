@@ -17,6 +17,7 @@ What it computes (paper sections / equations):
 * Next text position p_txt + 1                                   (Sec. 3.2 and 3.3, before Eq. "decode_with_active_cache")
 * The position-bound historical key RoPE(k_raw, p_m)             (Sec. 2.3, Eq. "historical_position_bound_kv")
 * Prefill capture: raw rows kept + position-bound cache rows       (Sec. 3.1, Eq. "raw_kv", "global_raw_memory")
+* First decode step over the active cache                         (Sec. 3.3, Eq. "decode_with_active_cache")
 
 Readings taken where the paper is silent (each is a named choice below):
 
@@ -245,6 +246,32 @@ def prefill_capture(k_raw_bits, v_raw_bits, coords, head_dim, sections, theta,
     v_raw_bits = np.asarray(v_raw_bits)
     k_cache = position_bound_keys(k_raw_bits, coords, head_dim, sections, theta, layout)
     return k_raw_bits.copy(), v_raw_bits.copy(), k_cache, v_raw_bits.copy()
+
+
+def decode_attention(q_raw: np.ndarray, q_pos: int, k_act: np.ndarray, v_act: np.ndarray,
+                     head_dim: int, sections, theta: float,
+                     layout: int = LAYOUT_SECTIONED) -> np.ndarray:
+    """Eq. "decode_with_active_cache" for one sequence and one layer:
+    o = softmax(RoPE(q_raw, p_next) K_act^T / sqrt(d_k)) V_act.
+
+    q_raw: [Hq, D] raw query (values); q_pos: the query's text position, the
+    triple (p, p, p) under M-RoPE; k_act, v_act: [S, H, D] active cache
+    (values). Query head hq reads KV head hq // (Hq / H). Returns [Hq, D]."""
+    q_raw = np.asarray(q_raw, dtype=np.float64)
+    k_act = np.asarray(k_act, dtype=np.float64)
+    v_act = np.asarray(v_act, dtype=np.float64)
+    Hq = q_raw.shape[0]
+    H = k_act.shape[1]
+    group = Hq // H
+    pos = np.full((Hq, 3), float(q_pos))
+    q = rope(q_raw, angles(pos, head_dim, sections, theta, layout))
+    out = np.zeros((Hq, head_dim))
+    for hq in range(Hq):
+        kh = hq // group
+        logits = k_act[:, kh, :] @ q[hq] / np.sqrt(head_dim)
+        w = np.exp(logits - logits.max())
+        out[hq] = (w / w.sum()) @ v_act[:, kh, :]
+    return out
 
 
 # ----------------------------------------------------------------------------

@@ -26,7 +26,8 @@ CACHE_CONTIGUOUS, CACHE_PAGED = 0, 1
 
 EXPORTS = ("prcr_workspace_size", "prcr_rebind_inject", "prcr_plan", "prcr_rebind_apply",
            "prcr_store_raw", "prcr_next_text_pos", "prcr_error_string", "prcr_version",
-           "prcr_rebind_inject_static", "prcr_prefill_capture")
+           "prcr_rebind_inject_static", "prcr_prefill_capture", "prcr_decode_workspace_size",
+           "prcr_decode_attention")
 STATIC_MAX_TOKENS = 65536
 
 
@@ -92,6 +93,13 @@ def lib():
                                        C.c_void_p, C.c_void_p, C.c_int64, C.c_int64, C.c_void_p,
                                        C.c_void_p, C.c_void_p]
     L.prcr_prefill_capture.restype = C.c_int
+    L.prcr_decode_workspace_size.argtypes = [P(RopeCfg), C.c_int32, C.c_int32, C.c_int64]
+    L.prcr_decode_workspace_size.restype = C.c_size_t
+    L.prcr_decode_attention.argtypes = [P(RopeCfg), P(CacheDesc), C.c_int32, C.c_int32,
+                                        C.c_void_p, C.c_void_p, C.c_void_p, C.c_int64,
+                                        C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t,
+                                        C.c_void_p]
+    L.prcr_decode_attention.restype = C.c_int
     L.prcr_next_text_pos.argtypes = [C.c_int64, C.c_int64, C.c_int32]
     L.prcr_next_text_pos.restype = C.c_int64
     L.prcr_error_string.argtypes = [C.c_int]
@@ -295,6 +303,31 @@ def prefill_capture(cfg, store, cache, seq: int, layer_begin: int, m_begin: int,
                                     v_src.data_ptr(), k_src.stride(0), k_src.stride(1),
                                     coords_src.data_ptr(), status.data_ptr(), _stream(stream))
     return _check(rc, "prcr_prefill_capture")
+
+
+def decode_workspace_size(cfg, n_seqs: int, n_q_heads: int, max_len: int) -> int:
+    return int(lib().prcr_decode_workspace_size(C.byref(cfg), int(n_seqs), int(n_q_heads),
+                                                int(max_len)))
+
+
+def decode_attention(cfg, cache, q: torch.Tensor, q_pos: torch.Tensor, seq_len: torch.Tensor,
+                     max_len: int, out: torch.Tensor, status: torch.Tensor,
+                     workspace: Optional[torch.Tensor] = None, stream=None):
+    """prcr_decode_attention: q [B, n_layers, Hq, D] bf16 (contiguous), q_pos int64 [B],
+    seq_len int32 [B], out float32 [B, n_layers, Hq, D]."""
+    if q.dtype != torch.bfloat16 or not q.is_contiguous():
+        raise TypeError("q must be a contiguous bfloat16 [B, n_layers, Hq, D] tensor")
+    if out.dtype != torch.float32 or not out.is_contiguous() or out.shape != q.shape:
+        raise TypeError("out must be a contiguous float32 tensor shaped like q")
+    if q_pos.dtype != torch.int64 or seq_len.dtype != torch.int32:
+        raise TypeError("q_pos must be int64 and seq_len int32")
+    ws = None if workspace is None else workspace.data_ptr()
+    nbytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    rc = lib().prcr_decode_attention(C.byref(cfg), C.byref(cache), int(q.shape[0]), int(q.shape[2]),
+                                     q.data_ptr(), q_pos.data_ptr(), seq_len.data_ptr(),
+                                     int(max_len), out.data_ptr(), status.data_ptr(), ws, nbytes,
+                                     _stream(stream))
+    return _check(rc, "prcr_decode_attention")
 
 
 def next_text_pos(p_txt: int, k_seq: int, mode: int = MODE_PCR) -> int:

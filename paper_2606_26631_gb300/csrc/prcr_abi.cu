@@ -314,6 +314,34 @@ int do_capture(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
     return launch_capture(a, grid, block, smem, stream) == cudaSuccess ? PRCR_OK : PRCR_ECUDA;
 }
 
+constexpr size_t kDecodeSmem = 48 * 1024;  // default dynamic shared memory limit
+
+// Chunking of the decode step: enough CTAs to fill the GPU a few times over,
+// chunks a multiple of 32 slots, at most kDecodeMaxChunk and small enough for
+// the chunk's row offsets to fit beside the rotated queries in shared memory.
+void decode_split(int64_t base_ctas, int64_t max_len, int sms, int64_t q_elems, int* splits,
+                  int* chunk) {
+    int64_t want = (int64_t(sms) * 4 + base_ctas - 1) / base_ctas;
+    if (want < 1) want = 1;
+    int64_t c = (max_len + want - 1) / want;
+    c = (c + 31) / 32 * 32;
+    if (c < 32) c = 32;
+    if (c > kDecodeMaxChunk) c = kDecodeMaxChunk;
+    const int64_t cap = (int64_t(kDecodeSmem) - q_elems * int64_t(sizeof(float))) / 8 / 32 * 32;
+    if (c > cap) c = cap;
+    *chunk = int(c);
+    *splits = int((max_len + c - 1) / c);
+    if (*splits < 1) *splits = 1;
+}
+
+bool decode_shape_ok(const prcr_rope_cfg* cfg, int32_t n_q_heads) {
+    const int D = cfg->head_dim;
+    if (D != 64 && D != 128 && D != 256) return false;
+    if (int64_t(n_q_heads) * D > PRCR_DECODE_MAX_Q_ELEMS) return false;
+    if (n_q_heads < cfg->n_kv_heads || n_q_heads % cfg->n_kv_heads) return false;
+    return n_q_heads / cfg->n_kv_heads <= 8;
+}
+
 }  // namespace
 }  // namespace prcr
 
@@ -418,6 +446,84 @@ int prcr_prefill_capture(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
     return do_capture(cfg, store, cache, seq, layer_begin, n_layers, m_begin, m_count, slot_begin,
                       k_src, v_src, src_layer_stride, src_token_stride, coords_src, status,
                       static_cast<cudaStream_t>(stream));
+}
+
+size_t prcr_decode_workspace_size(const prcr_rope_cfg* cfg, int32_t n_seqs, int32_t n_q_heads,
+                                  int64_t max_len) {
+    if (check_cfg(cfg) || n_seqs < 1 || max_len < 1 || !decode_shape_ok(cfg, n_q_heads)) return 0;
+    int dev = 0, sms = 1;
+    if (cudaGetDevice(&dev) == cudaSuccess) sms = sm_count(dev);
+    int splits = 1, chunk = 32;
+    decode_split(int64_t(n_seqs) * cfg->n_layers, max_len, sms, int64_t(n_q_heads) * cfg->head_dim,
+                 &splits, &chunk);
+    if (splits == 1) return 0;
+    return size_t(n_seqs) * cfg->n_layers * n_q_heads * splits * (cfg->head_dim + 2) * sizeof(float);
+}
+
+int prcr_decode_attention(const prcr_rope_cfg* cfg, const prcr_cache_desc* cache, int32_t n_seqs,
+                          int32_t n_q_heads, const void* q, const int64_t* q_pos,
+                          const int32_t* seq_len, int64_t max_len, float* out, uint32_t* status,
+                          void* workspace, size_t workspace_bytes, void* stream) {
+    int rc = check_cfg(cfg);
+    if (rc) return rc;
+    if ((rc = check_cache(cfg, cache))) return rc;
+    if (!decode_shape_ok(cfg, n_q_heads) || n_seqs < 0 || n_seqs > cache->n_seqs || max_len < 0)
+        return PRCR_EINVAL;
+    if (n_seqs == 0 || max_len == 0) return PRCR_OK;
+    if (!q || !q_pos || !seq_len || !out || !status) return PRCR_EINVAL;
+    if (!aligned4(q) || !aligned8(q_pos) || !aligned4(seq_len) || !aligned16(out) ||
+        !aligned4(status))
+        return PRCR_EALIGN;
+    const int64_t capacity = cache->kind == PRCR_CACHE_CONTIGUOUS
+                                 ? int64_t(cache->max_slots)
+                                 : int64_t(cache->bt_stride) * cache->block_size;
+    if (max_len > capacity) return PRCR_EINVAL;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return PRCR_ECUDA;
+    DecodeArgs a = {};
+    decode_split(int64_t(n_seqs) * cfg->n_layers, max_len, sm_count(dev),
+                 int64_t(n_q_heads) * cfg->head_dim, &a.splits, &a.chunk);
+    if (a.splits > 1) {
+        const size_t need = size_t(n_seqs) * cfg->n_layers * n_q_heads * a.splits *
+                            (cfg->head_dim + 2) * sizeof(float);
+        if (!workspace || workspace_bytes < need) return PRCR_EWORKSPACE;
+        if (!aligned16(workspace)) return PRCR_EALIGN;
+        a.partial = static_cast<float*>(workspace);
+    }
+    a.q = static_cast<const uint16_t*>(q);
+    a.q_pos = q_pos;
+    a.seq_len = seq_len;
+    a.cache_k = static_cast<const uint16_t*>(cache->k);
+    a.cache_v = static_cast<const uint16_t*>(cache->v);
+    a.layer_stride = cache->layer_stride;
+    a.seq_stride = cache->seq_stride;
+    a.block_stride = cache->block_stride;
+    a.slot_stride = cache->slot_stride;
+    a.capacity = capacity;
+    a.block_table = cache->block_table;
+    a.bt_stride = cache->bt_stride;
+    a.block_size = cache->kind == PRCR_CACHE_PAGED ? cache->block_size : 1;
+    a.n_blocks = cache->n_blocks;
+    a.cache_kind = cache->kind;
+    a.out = out;
+    a.status = status;
+    a.n_layers = cfg->n_layers;
+    a.n_kv_heads = cfg->n_kv_heads;
+    a.n_q_heads = n_q_heads;
+    a.head_dim = cfg->head_dim;
+    a.group = n_q_heads / cfg->n_kv_heads;
+    a.scale = float(1.0 / std::sqrt(double(cfg->head_dim)));
+    const int P = cfg->head_dim / 2;
+    for (int i = 0; i < P; ++i)
+        a.inv_freq[i] = std::pow(cfg->theta, -2.0 * double(i) / double(cfg->head_dim));
+    int gp = 1;
+    while (gp < a.group) gp <<= 1;
+    const size_t smem = size_t(n_q_heads) * cfg->head_dim * sizeof(float) +
+                        size_t(a.chunk) * sizeof(int64_t);
+    const dim3 grid(unsigned(a.splits), unsigned(cfg->n_layers), unsigned(n_seqs));
+    return launch_decode(a, gp, grid, smem, static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? PRCR_OK
+               : PRCR_ECUDA;
 }
 
 int64_t prcr_next_text_pos(int64_t p_txt, int64_t k_seq, int32_t mode) {

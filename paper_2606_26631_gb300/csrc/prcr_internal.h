@@ -155,6 +155,40 @@ struct CaptureArgs {
     double inv_freq[kMaxPairs];
 };
 
+struct DecodeArgs {
+    const uint16_t* q;          // [B][n_layers][n_q_heads][D] raw queries
+    const int64_t* q_pos;       // [B]
+    const int32_t* seq_len;     // [B]
+    const uint16_t* cache_k;
+    const uint16_t* cache_v;
+    int64_t layer_stride;
+    int64_t seq_stride;         // contiguous
+    int64_t block_stride;       // paged
+    int64_t slot_stride;
+    int64_t capacity;           // slots per sequence
+    const int32_t* block_table;
+    int32_t bt_stride;
+    int32_t block_size;
+    int32_t n_blocks;
+    int32_t cache_kind;
+    float* out;                 // [B][n_layers][n_q_heads][D]
+    float* partial;             // [B][n_layers][n_q_heads][splits][D + 2] when splits > 1
+    uint32_t* status;
+    int32_t n_layers;
+    int32_t n_kv_heads;
+    int32_t n_q_heads;
+    int32_t head_dim;
+    int32_t group;
+    int32_t splits;
+    int32_t chunk;
+    float scale;
+    double inv_freq[kMaxPairs];
+};
+
+constexpr int kDecodeMaxChunk = 4096;
+
+cudaError_t launch_decode(const DecodeArgs& a, int gp, dim3 grid, size_t smem,
+                          cudaStream_t stream);
 cudaError_t launch_capture(const CaptureArgs& a, dim3 grid, int block, size_t smem,
                            cudaStream_t stream);
 cudaError_t capture_blocks_per_sm(int block, size_t smem, int* out);

@@ -1,0 +1,153 @@
+"""GPU parity of prcr_decode_attention (Eq. "decode_with_active_cache")
+against the oracle's fp64 decode_attention.
+
+1. Decode over a populated input cache (contiguous and paged, GQA groups
+   1 / 4 / 7, head_dim 64 / 128 / 256, sequences long enough to be split).
+   Bar: max |o_gpu - o_ref| <= 1e-4 * max |V| (float32 logits, exp and
+   accumulation over at most a few thousand slots per chunk stay ~1e-6).
+2. End to end: revisit rows appended by prcr_rebind_inject into a cache whose
+   context rows are data, then decoded at next_pos over cache_len_out. The
+   expected cache is the context plus the oracle's rebound keys rounded to
+   bf16 (the value a correct kernel stores); bar 1e-3 * max |V|.
+3. Relative positions only (Eq. "direct_reuse_score"): a cache made only of
+   revisited rows decoded at p + 1 gives the same output when the text
+   position moves by a constant (up to the bf16 rounding of the keys).
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import prcr_oracle as O
+from workloads import Workload, get, make_batch, make_decode_inputs
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+
+
+def _f64(t):
+    return O.bf16_bits_to_f64(t.contiguous().view(torch.int16).cpu().numpy())
+
+
+def _cache_rows(cache_k, cache_v, block_table, b, n, paged):
+    """[n, n_L, H, D] value arrays of slots 0..n-1 of sequence b (input data)."""
+    s = torch.arange(n, device=cache_k.device)
+    if not paged:
+        return _f64(cache_k[b, :, :n].transpose(0, 1)), _f64(cache_v[b, :, :n].transpose(0, 1))
+    bs = cache_k.shape[2]
+    blk = block_table[b][s // bs].long()
+    off = s % bs
+    return _f64(cache_k[:, blk, off].transpose(0, 1)), _f64(cache_v[:, blk, off].transpose(0, 1))
+
+
+def _run_decode(cfg, cache_desc, q, q_pos, seq_len, max_len):
+    import paper_2606_26631_gb300 as prcr
+    out = torch.full(q.shape, float("nan"), dtype=torch.float32, device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    nbytes = prcr.decode_workspace_size(cfg, q.shape[0], q.shape[2], max_len)
+    ws = torch.empty(max(nbytes, 16), dtype=torch.uint8, device=DEV)
+    prcr.decode_attention(cfg, cache_desc, q, q_pos, seq_len, max_len, out, status, ws)
+    torch.cuda.synchronize()
+    return out, int(status.item())
+
+
+CASES = [  # (B, layers, H, Hq, D, max_len, paged)
+    (3, 3, 8, 32, 128, 3000, True),
+    (2, 2, 2, 14, 64, 700, False),
+    (2, 2, 4, 4, 256, 1200, True),
+    (5, 1, 4, 28, 128, 9000, True),
+]
+
+
+@pytest.mark.parametrize("case", CASES, ids=[f"B{c[0]}L{c[1]}H{c[2]}Hq{c[3]}D{c[4]}S{c[5]}{'p' if c[6] else 'c'}" for c in CASES])
+def test_decode_parity(case):
+    import paper_2606_26631_gb300 as prcr
+    B, nL, H, Hq, D, max_len, paged = case
+    sec = (D // 8, D // 8 + (D // 2 - 3 * (D // 8)) // 2, 0)
+    sec = (sec[0], sec[1], D // 2 - sec[0] - sec[1])
+    inp = make_decode_inputs(B, nL, H, Hq, D, max_len, paged, device=DEV, seed=7)
+    cfg = prcr.rope_cfg(nL, H, D, sec, 1e6)
+    cd = (prcr.cache_paged(inp["cache_k"], inp["cache_v"], inp["block_table"]) if paged
+          else prcr.cache_contiguous(inp["cache_k"], inp["cache_v"]))
+    out, st = _run_decode(cfg, cd, inp["q"], inp["q_pos"], inp["seq_len"], max_len)
+    assert st == 0
+    got = out.cpu().numpy()
+    qv = _f64(inp["q"])
+    for b in range(B):
+        n = int(inp["seq_len"][b])
+        K, V = _cache_rows(inp["cache_k"], inp["cache_v"], inp["block_table"], b, n, paged)
+        for l in range(nL):
+            ref = O.decode_attention(qv[b, l], int(inp["q_pos"][b]), K[:, l], V[:, l], D, sec, 1e6)
+            err = np.abs(got[b, l] - ref).max() / np.abs(V[:, l]).max()
+            assert err <= 1e-4, (b, l, err)
+
+
+def test_inject_then_decode():
+    import paper_2606_26631_gb300 as prcr
+    import parity_util as pu
+    for name in ("qwen2vl-2b", "qwen25vl-7b"):
+        wl = get(name)
+        batch = make_batch(wl, device=DEV, context="random")
+        B, nL, H, D = wl.n_seqs, wl.n_layers, wl.n_kv_heads, wl.head_dim
+        Hq = {"qwen2vl-2b": 12, "qwen25vl-7b": 28}[name]
+        # expected cache: context rows as given + the oracle's rows at the slots
+        ctx_k = batch.cache_k.clone()
+        ctx_v = batch.cache_v.clone()
+        rv = pu.make_revisit(batch)
+        rv.run()
+        torch.cuda.synchronize()
+        assert rv.status_value() == 0
+        pl = pu.oracle_plan(batch)
+        g = torch.Generator(device=DEV)
+        g.manual_seed(11)
+        q = torch.randn((B, nL, Hq, D), generator=g, device=DEV).to(torch.bfloat16)
+        max_len = int(pl["cache_len_out"].max())
+        cfg = rv.cfg
+        out, st = _run_decode(cfg, rv.cache, q, rv.next_pos, rv.cache_len_out, max_len)
+        assert st == 0
+        got = out.cpu().numpy()
+        qv = _f64(q)
+        idx = batch.idx.cpu().numpy()
+        for b in range(B):
+            n_ctx = int(batch.cache_len_in[b])
+            n_all = int(pl["cache_len_out"][b])
+            K, V = _cache_rows(ctx_k, ctx_v, batch.block_table, b, n_all, batch.paged)
+            toks = np.nonzero(pl["seq"] == b)[0]
+            slots = pl["slot"][toks]
+            k_raw = pu.bits(batch.store_k[b][:, torch.as_tensor(idx[toks], device=DEV).long()]
+                            .transpose(0, 1))
+            v_raw = pu.bits(batch.store_v[b][:, torch.as_tensor(idx[toks], device=DEV).long()]
+                            .transpose(0, 1))
+            k_hat = O.rebind_keys(k_raw, pl["pos"][toks], D, wl.sections, wl.theta)
+            K[slots] = O.f64_to_bf16_rne(k_hat)
+            V[slots] = O.bf16_bits_to_f64(v_raw)
+            assert n_ctx + len(toks) == n_all
+            for l in range(nL):
+                ref = O.decode_attention(qv[b, l], int(pl["next_pos"][b]), K[:, l], V[:, l], D,
+                                         wl.sections, wl.theta)
+                err = np.abs(got[b, l] - ref).max() / np.abs(V[:, l]).max()
+                assert err <= 1e-3, (name, b, l, err)
+
+
+def test_decode_sees_only_relative_positions():
+    import paper_2606_26631_gb300 as prcr
+    import parity_util as pu
+    wl = Workload(name="rel", n_layers=2, n_kv_heads=4, head_dim=128, sections=(16, 24, 24),
+                  n_seqs=2, grids=((1, 24, 24),), selection="random", cache="contiguous",
+                  cur_pos=("fixed", 3000), extra=(1, 1, 200, 300))
+    outs = []
+    for shift in (0, 12345):
+        batch = make_batch(wl, device=DEV, seed=3)
+        batch.p_txt += shift
+        batch.cache_len_in.zero_()  # the cache holds only the revisited rows
+        rv = pu.make_revisit(batch)
+        rv.run()
+        g = torch.Generator(device=DEV)
+        g.manual_seed(5)
+        q = torch.randn((2, 2, 16, 128), generator=g, device=DEV).to(torch.bfloat16)
+        out, st = _run_decode(rv.cfg, rv.cache, q, rv.next_pos, rv.cache_len_out,
+                              int(rv.cache_len_out.max()))
+        assert st == 0 and rv.status_value() == 0
+        outs.append(out.cpu().numpy())
+    vmax = float(torch.abs(batch.store_v.float()).max())
+    assert np.abs(outs[0] - outs[1]).max() / vmax <= 2e-3

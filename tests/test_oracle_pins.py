@@ -392,11 +392,52 @@ def pin_prefill_capture(o):
                 assert abs(ck[m, h, i] - z.real) < 1e-12 and abs(ck[m, h, i + P] - z.imag) < 1e-12
 
 
+def pin_decode_attention(o):
+    """Eq. "decode_with_active_cache": (1) one cached slot returns its value
+    row; (2) equal keys give the mean of the values; (3) against a direct
+    per-slot loop with math.exp; (4) a uniform shift of every position
+    (query and cached keys) leaves the output unchanged (Eq.
+    "direct_reuse_score": logits see only relative offsets); (5) GQA: query
+    head hq reads KV head hq // group."""
+    rng = np.random.default_rng(31)
+    D, sec, th = 16, (2, 3, 3), 1e6
+    q = rng.standard_normal((4, D))
+    v1 = rng.standard_normal((1, 2, D))
+    k1 = rng.standard_normal((1, 2, D))
+    out = o.decode_attention(q, 50, k1, v1, D, sec, th)
+    assert np.allclose(out, np.repeat(v1[0], 2, axis=0), atol=1e-14)
+    kk = np.repeat(rng.standard_normal((1, 2, D)), 5, axis=0)
+    vv = rng.standard_normal((5, 2, D))
+    out = o.decode_attention(q, 7, kk, vv, D, sec, th)
+    assert np.allclose(out, np.repeat(vv.mean(axis=0), 2, axis=0), atol=1e-12)
+    S = 9
+    k_raw = rng.standard_normal((S, 2, D))
+    v = rng.standard_normal((S, 2, D))
+    kpos = rng.uniform(0, 300, size=(S, 3))
+    k = o.rope(k_raw, o.angles(kpos, D, sec, th))
+    out = o.decode_attention(q, 301, k, v, D, sec, th)
+    P = D // 2
+    for hq in range(4):
+        kh = hq // 2
+        qz = [complex(q[hq, i], q[hq, i + P]) * cmath.exp(1j * 301 * th ** (-2.0 * i / D))
+              for i in range(P)]
+        qr = [z.real for z in qz] + [z.imag for z in qz]
+        lg = [sum(qr[d] * k[s, kh, d] for d in range(D)) / math.sqrt(D) for s in range(S)]
+        mx = max(lg)
+        w = [math.exp(x - mx) for x in lg]
+        ref = [sum(w[s] * v[s, kh, d] for s in range(S)) / sum(w) for d in range(D)]
+        assert np.allclose(out[hq], ref, rtol=0, atol=1e-12)
+    shift = 1234.0
+    k2 = o.rope(k_raw, o.angles(kpos + shift, D, sec, th))
+    out2 = o.decode_attention(q, 301 + shift, k2, v, D, sec, th)
+    assert np.allclose(out, out2, rtol=0, atol=1e-9)
+
+
 PINS = [pin_worked_rect4x4, pin_worked_rect2x2, pin_pcr_closed_forms, pin_degenerate_center,
         pin_other_modes, pin_plan_slots_and_continuity, pin_rope_closed_forms,
         pin_mrope_equal_axes_is_textbook, pin_mrope_sections, pin_rope_invariants,
         pin_bf16_helpers, pin_brute_force_2x2, pin_original_mode_is_position_bound_cache,
-        pin_prefill_capture]
+        pin_prefill_capture, pin_decode_attention]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -480,6 +521,26 @@ def _m_range_swapped_axes(sel):
     return lo, hi
 
 
+_orig_decode = O.decode_attention
+
+
+def _m_decode_no_scale(q_raw, q_pos, k_act, v_act, head_dim, sections, theta, layout=0):
+    return _orig_decode(q_raw, q_pos, k_act * np.sqrt(head_dim), v_act, head_dim, sections, theta,
+                        layout)
+
+
+def _m_decode_head_modulo(q_raw, q_pos, k_act, v_act, head_dim, sections, theta, layout=0):
+    H = k_act.shape[1]
+    Hq = q_raw.shape[0]
+    perm = np.array([(hq % H) * (Hq // H) + hq // H for hq in range(Hq)])
+    return _orig_decode(q_raw[perm], q_pos, k_act, v_act, head_dim, sections, theta, layout)[
+        np.argsort(perm)]
+
+
+def _m_decode_query_unrotated(q_raw, q_pos, k_act, v_act, head_dim, sections, theta, layout=0):
+    return _orig_decode(q_raw, 0, k_act, v_act, head_dim, sections, theta, layout)
+
+
 MUTANTS = [
     ("pcr_position", _m_pcr_k_not_k_minus_1),
     ("pcr_position", _m_pcr_denominator_k),
@@ -493,6 +554,9 @@ MUTANTS = [
     ("plan", _m_plan_slot_shift),
     ("next_text_pos", _m_next_pos_same),
     ("coord_range", _m_range_swapped_axes),
+    ("decode_attention", _m_decode_no_scale),
+    ("decode_attention", _m_decode_head_modulo),
+    ("decode_attention", _m_decode_query_unrotated),
 ]
 
 

@@ -212,7 +212,8 @@ def fill_store(wl: Workload, store_k: torch.Tensor, store_v: torch.Tensor, seed:
 # ----------------------------------------------------------------------------
 # whole batch
 # ----------------------------------------------------------------------------
-def make_batch(wl: Workload, device="cpu", seed: int = 0, store: bool = True) -> Batch:
+def make_batch(wl: Workload, device="cpu", seed: int = 0, store: bool = True,
+               context: str = "canary") -> Batch:
     device = torch.device(device)
     rng_sel = np.random.Generator(np.random.PCG64(seed + 1))
     rng_pos = np.random.Generator(np.random.PCG64(seed + 2))
@@ -245,6 +246,11 @@ def make_batch(wl: Workload, device="cpu", seed: int = 0, store: bool = True) ->
     else:
         store_k = store_v = torch.empty((0,), dtype=torch.bfloat16, device=device)
 
+    # context="canary": only the appended span is backed (paged) and every
+    # cache row holds the canary; context="random": every slot up to the end of
+    # the appended span is backed and the existing context rows hold N(0, 1)
+    # values standing in for the model's already-rotated entries.
+    full = context == "random"
     bs = wl.block_size
     if wl.cache == "contiguous":
         S = int(np.max(cache_len_in.astype(np.int64) + k_per_seq))
@@ -254,7 +260,12 @@ def make_batch(wl: Workload, device="cpu", seed: int = 0, store: bool = True) ->
     else:
         first = cache_len_in.astype(np.int64) // bs
         last = (cache_len_in.astype(np.int64) + k_per_seq - 1) // bs
-        n_span = np.where(k_per_seq > 0, last - first + 1, 0)
+        if full:
+            last = np.maximum(last, (cache_len_in.astype(np.int64) - 1) // bs)
+            first = np.zeros_like(first)
+            n_span = last - first + 1
+        else:
+            n_span = np.where(k_per_seq > 0, last - first + 1, 0)
         n_blocks = int(n_span.sum())
         max_blocks = int(np.max(np.where(k_per_seq > 0, last + 1, first + 1))) + 1
         perm = rng_pos.permutation(n_blocks).astype(np.int32)
@@ -266,8 +277,14 @@ def make_batch(wl: Workload, device="cpu", seed: int = 0, store: bool = True) ->
                 k += 1
         cshape = (nL, max(n_blocks, 1), bs, H, D)
         block_table = torch.from_numpy(bt).to(device)
-    cache_k = torch.full(cshape, CANARY_BITS, dtype=torch.int16, device=device).view(torch.bfloat16)
-    cache_v = torch.full(cshape, CANARY_BITS, dtype=torch.int16, device=device).view(torch.bfloat16)
+    if full:
+        g = torch.Generator(device=device)
+        g.manual_seed(seed + 3)
+        cache_k = torch.randn(cshape, generator=g, device=device, dtype=torch.float32).to(torch.bfloat16)
+        cache_v = torch.randn(cshape, generator=g, device=device, dtype=torch.float32).to(torch.bfloat16)
+    else:
+        cache_k = torch.full(cshape, CANARY_BITS, dtype=torch.int16, device=device).view(torch.bfloat16)
+        cache_v = torch.full(cshape, CANARY_BITS, dtype=torch.int16, device=device).view(torch.bfloat16)
 
     t = lambda a, dt: torch.as_tensor(np.asarray(a), dtype=dt).to(device)
     return Batch(
@@ -277,3 +294,41 @@ def make_batch(wl: Workload, device="cpu", seed: int = 0, store: bool = True) ->
         idx=t(idx, torch.int32), p_txt=t(p_txt, torch.int64),
         cache_len_in=t(cache_len_in, torch.int32),
         cache_k=cache_k, cache_v=cache_v, block_table=block_table, revisits=revisits)
+
+
+def make_decode_inputs(n_seqs: int, n_layers: int, n_kv_heads: int, n_q_heads: int, head_dim: int,
+                       max_len: int, paged: bool, device="cpu", seed: int = 0,
+                       block_size: int = 16) -> dict:
+    """A populated decoder cache (N(0, 1) bf16 rows in every slot each sequence
+    attends), raw queries N(0, 1) bf16 [B, n_L, Hq, D], per-sequence lengths
+    (the last sequence at max_len) and query positions at or after them."""
+    device = torch.device(device)
+    rng = np.random.Generator(np.random.PCG64(seed + 1))
+    seq_len = rng.integers(1, max_len + 1, size=n_seqs)
+    seq_len[-1] = max_len
+    q_pos = seq_len + rng.integers(0, 20000, size=n_seqs)
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    H, D = n_kv_heads, head_dim
+    if paged:
+        nblk = [(int(n) + block_size - 1) // block_size for n in seq_len]
+        total = sum(nblk)
+        perm = rng.permutation(total + 3)[:total]  # a few pool blocks stay unused
+        bt = np.full((n_seqs, max(nblk) + 2), -1, dtype=np.int32)
+        k = 0
+        for b in range(n_seqs):
+            bt[b, :nblk[b]] = perm[k:k + nblk[b]]
+            k += nblk[b]
+        shape = (n_layers, total + 3, block_size, H, D)
+        block_table = torch.from_numpy(bt).to(device)
+    else:
+        shape = (n_seqs, n_layers, max_len + 8, H, D)
+        block_table = None
+    cache_k = torch.randn(shape, generator=g, device=device, dtype=torch.float32).to(torch.bfloat16)
+    cache_v = torch.randn(shape, generator=g, device=device, dtype=torch.float32).to(torch.bfloat16)
+    q = torch.randn((n_seqs, n_layers, n_q_heads, D), generator=g, device=device,
+                    dtype=torch.float32).to(torch.bfloat16)
+    return dict(cache_k=cache_k, cache_v=cache_v, block_table=block_table, q=q,
+                q_pos=torch.as_tensor(q_pos, dtype=torch.int64).to(device),
+                seq_len=torch.as_tensor(seq_len, dtype=torch.int32).to(device),
+                max_len=int(max_len), block_size=block_size)
