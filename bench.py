@@ -57,6 +57,10 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["prcr", "reference"], default="prcr")
     ap.add_argument("--workload", default="stress")
+    ap.add_argument("--path", choices=["revisit", "capture", "decode"], default="revisit",
+                    help="revisit: the rebind+inject step (default); capture: prefill capture; "
+                         "decode: the first decode step over the active cache")
+    ap.add_argument("--seqs", type=int, default=0, help="capture/decode: sequences (0 = workload's)")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-samples", type=int, default=8,
@@ -411,10 +415,136 @@ def run_gpu(args):
         dist.destroy_process_group()
 
 
+def _timed(fn, steps, warmup, local):
+    import torch
+    stream = torch.cuda.current_stream()
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(steps)]
+    with Clocks(local) as clk:
+        for e0, e1 in ev:
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+        torch.cuda.synchronize()
+    ms = [e0.elapsed_time(e1) for e0, e1 in ev]
+    return ms, clk.summary()
+
+
+def run_capture_path(args):
+    """Prefill capture: every visual token of every sequence, all layers."""
+    import torch
+    _, _, local = dist_env()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    from paper_2606_26631_gb300 import _build
+    if not _build.up_to_date():
+        _build.build()
+    import paper_2606_26631_gb300 as prcr
+    from workloads import get, make_batch
+    wl = get(args.workload)
+    if args.seqs:
+        wl = dataclasses.replace(wl, n_seqs=args.seqs)
+    src = make_batch(wl, device=dev)  # its raw store stands in for the prefill projections
+    B, nL, M, H, D = wl.n_seqs, wl.n_layers, wl.n_tokens, wl.n_kv_heads, wl.head_dim
+    store_k = torch.empty_like(src.store_k); store_v = torch.empty_like(src.store_v)
+    coords = torch.empty_like(src.coords)
+    bs = 16
+    nblk = (M + bs - 1) // bs
+    perm = torch.randperm(B * nblk, device=dev, generator=torch.Generator(device=dev).manual_seed(2))
+    bt = perm.view(B, nblk).to(torch.int32).contiguous()
+    cache_k = torch.empty((nL, B * nblk, bs, H, D), dtype=torch.bfloat16, device=dev)
+    cache_v = torch.empty_like(cache_k)
+    cfg = prcr.rope_cfg(nL, H, D, wl.sections, wl.theta)
+    sd = prcr.store_desc(store_k, store_v, coords)
+    cd = prcr.cache_paged(cache_k, cache_v, bt)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+
+    def step():
+        for b in range(B):
+            prcr.prefill_capture(cfg, sd, cd, b, 0, 0, 0, src.store_k[b], src.store_v[b],
+                                 src.coords[b], status)
+
+    step()
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    assert torch.equal(store_k.view(torch.int16), src.store_k.view(torch.int16))
+    ms, clk = _timed(step, args.steps, args.warmup, local)
+    nbytes = B * M * nL * H * D * 2 * 6  # read k, v; write store k, v and cache k, v
+    t = sum(ms) / 1e3
+    peak, kind = measured_peaks()
+    value = nbytes * args.steps / t / 1e9
+    print(json.dumps(dict(
+        metric="prefill capture GB/s (read+write)", value=value, unit=UNIT, n_gpus=1,
+        steps=args.steps, warmup=args.warmup, ms_per_step=1e3 * t / args.steps,
+        higher_is_better=True, scaling="weak", vs_baseline=None, dtype="f32", io_dtype="bf16",
+        data="synthetic", config=dict(workload=wl.name, batch=B, tokens_per_seq=M, n_layers=nL,
+                                      cache="paged/16", bytes_per_step=nbytes),
+        roofline=dict(bound="hbm", achieved=value, peak=peak, unit="GB/s", frac=value / peak,
+                      traffic=None, kernel="capture_kernel", peak_kind=f"{kind} copy (hbm_gbs)"),
+        gpu_launches=B * args.steps, clocks=clk)), flush=True)
+
+
+def run_decode_path(args):
+    """First decode step over a populated paged cache of the workload's shape."""
+    import torch
+    _, _, local = dist_env()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    from paper_2606_26631_gb300 import _build
+    if not _build.up_to_date():
+        _build.build()
+    import paper_2606_26631_gb300 as prcr
+    from workloads import get, make_decode_inputs
+    wl = get(args.workload)
+    B = args.seqs or wl.n_seqs
+    Hq = 4 * wl.n_kv_heads
+    max_len = 8192
+    inp = make_decode_inputs(B, wl.n_layers, wl.n_kv_heads, Hq, wl.head_dim, max_len, True,
+                             device=dev, seed=1)
+    cfg = prcr.rope_cfg(wl.n_layers, wl.n_kv_heads, wl.head_dim, wl.sections, wl.theta)
+    cd = prcr.cache_paged(inp["cache_k"], inp["cache_v"], inp["block_table"])
+    out = torch.empty(inp["q"].shape, dtype=torch.float32, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    nws = prcr.decode_workspace_size(cfg, B, Hq, max_len)
+    ws = torch.empty(max(nws, 16), dtype=torch.uint8, device=dev)
+
+    def step():
+        prcr.decode_attention(cfg, cd, inp["q"], inp["q_pos"], inp["seq_len"], max_len, out,
+                              status, ws)
+
+    step()
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    ms, clk = _timed(step, args.steps, args.warmup, local)
+    slots = int(inp["seq_len"].sum())
+    nbytes = slots * wl.n_layers * wl.n_kv_heads * wl.head_dim * 2 * 2
+    t = sum(ms) / 1e3
+    peak, kind = measured_peaks()
+    value = nbytes * args.steps / t / 1e9
+    print(json.dumps(dict(
+        metric="decode attention GB/s (K/V read)", value=value, unit=UNIT, n_gpus=1,
+        steps=args.steps, warmup=args.warmup, ms_per_step=1e3 * t / args.steps,
+        higher_is_better=True, scaling="weak", vs_baseline=None, dtype="f32", io_dtype="bf16",
+        data="synthetic", config=dict(workload=wl.name, batch=B, n_q_heads=Hq, max_len=max_len,
+                                      slots=slots, cache="paged/16", bytes_per_step=nbytes,
+                                      workspace_bytes=nws),
+        roofline=dict(bound="hbm", achieved=value, peak=peak, unit="GB/s", frac=value / peak,
+                      traffic=None, kernel="decode_kernel (+ merge)",
+                      peak_kind=f"{kind} copy (hbm_gbs)"),
+        gpu_launches=(2 if nws else 1) * args.steps, clocks=clk)), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         run_reference(args)
+    elif args.path == "capture":
+        run_capture_path(args)
+    elif args.path == "decode":
+        run_decode_path(args)
     else:
         run_gpu(args)
 
