@@ -290,6 +290,32 @@ PRCR_API int prcr_decode_attention(const prcr_rope_cfg* cfg, const prcr_cache_de
                                    float* out, uint32_t* status, void* workspace,
                                    size_t workspace_bytes, void* stream);
 
+/* prcr_select_topk - the revisited index set I_tau (Sec. 2.1, Eq. 3) chosen
+ * by attention. The paper names an attention-driven selection (it ranks the
+ * visual tokens by relevance to the current decoding context and keeps K);
+ * its formula is not in the paper. Reading implemented: for sequence b the
+ * relevance of visual token m is the trigger query's attention on m at layer
+ * `layer`: per query head h, softmax over the store's M tokens of
+ * RoPE(q[b][h], (p, p, p)) . RoPE(k_raw[b][layer][m][h / group], p_m) / sqrt(D),
+ * p = q_pos[b], averaged over the heads. The k most relevant tokens (equal
+ * relevance: lower index first) are written in ascending token order as one
+ * revisit per sequence, ready for prcr_rebind_inject:
+ *   idx_out     device int32 [n_seqs * k]   selected token ids
+ *   seq_rev_off device int32 [n_seqs + 1]   b
+ *   rev_tok_off device int32 [n_seqs + 1]   b * k
+ *   score_out   optional device float32 [n_seqs][n_tokens] relevance
+ *   q           device bf16 [n_seqs][n_q_heads][D] raw trigger queries of `layer`
+ * Limits: 1 <= k <= n_tokens <= PRCR_SELECT_MAX_TOKENS; n_q_heads a multiple of
+ * n_kv_heads, <= 8 per KV head, n_q_heads * D <= PRCR_DECODE_MAX_Q_ELEMS.
+ * workspace: device >= prcr_select_workspace_size(...) bytes (the logits).   */
+#define PRCR_SELECT_MAX_TOKENS 32768
+PRCR_API size_t prcr_select_workspace_size(int32_t n_seqs, int32_t n_q_heads, int32_t n_tokens);
+PRCR_API int prcr_select_topk(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+                              int32_t n_seqs, int32_t layer, int32_t n_q_heads, const void* q,
+                              const int64_t* q_pos, int32_t k, int32_t* idx_out,
+                              int32_t* seq_rev_off, int32_t* rev_tok_off, float* score_out,
+                              void* workspace, size_t workspace_bytes, void* stream);
+
 /* prcr_next_text_pos - host helper: the position the next text token takes
  * after a revisit appended k_seq tokens to a sequence whose latest text token
  * is at p_txt: p_txt + 1 for PCR, ORIGINAL and UIR (Sec. 3.2, Sec. 3.3);

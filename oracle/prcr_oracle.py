@@ -18,6 +18,7 @@ What it computes (paper sections / equations):
 * The position-bound historical key RoPE(k_raw, p_m)             (Sec. 2.3, Eq. "historical_position_bound_kv")
 * Prefill capture: raw rows kept + position-bound cache rows       (Sec. 3.1, Eq. "raw_kv", "global_raw_memory")
 * First decode step over the active cache                         (Sec. 3.3, Eq. "decode_with_active_cache")
+* Attention-driven selection of the revisited set I_tau            (Sec. 2.1, Eq. 3; reading below)
 
 Readings taken where the paper is silent (each is a named choice below):
 
@@ -39,6 +40,11 @@ Readings taken where the paper is silent (each is a named choice below):
 * LPA (Sec. 3.2, Table 2; formula not printed): the r-th token appended to a
   sequence in this call goes to p_txt + r (r = 1, 2, ...) on all axes, and the
   next text position becomes p_txt + K_seq + 1.
+* Attention-driven selection (Sec. 2.1 names it, its formula is outside the
+  paper): the relevance of visual token m is the trigger query's attention
+  on m at one layer, softmax over the M visual tokens' position-bound keys
+  RoPE(k_raw, p_m), averaged over the query heads; the K most relevant tokens
+  are selected (ties to the lower index) and listed in ascending token order.
 
 Parity pins for every function here live in tests/test_oracle_pins.py; every
 function is pinned (no function is "parity unpinned").
@@ -272,6 +278,34 @@ def decode_attention(q_raw: np.ndarray, q_pos: int, k_act: np.ndarray, v_act: np
         w = np.exp(logits - logits.max())
         out[hq] = (w / w.sum()) @ v_act[:, kh, :]
     return out
+
+
+def ads_relevance(q_raw: np.ndarray, q_pos: int, k_raw_bits: np.ndarray, coords, head_dim: int,
+                  sections, theta: float, layout: int = LAYOUT_SECTIONED) -> np.ndarray:
+    """Relevance of each visual token to the trigger query (the reading of the
+    attention-driven selection named in Sec. 2.1): q_raw [Hq, D] values at
+    text position q_pos; k_raw_bits [M, H, D] raw keys of one layer; coords
+    [M, 3]. r_m = mean over query heads h of softmax_m(RoPE(q_h, (p,p,p)) .
+    RoPE(k_m, p_m) / sqrt(D)), query head h reading KV head h // (Hq / H)."""
+    q_raw = np.asarray(q_raw, dtype=np.float64)
+    Hq = q_raw.shape[0]
+    k = position_bound_keys(k_raw_bits, coords, head_dim, sections, theta, layout)  # [M, H, D]
+    H = k.shape[1]
+    group = Hq // H
+    q = rope(q_raw, angles(np.full((Hq, 3), float(q_pos)), head_dim, sections, theta, layout))
+    r = np.zeros(k.shape[0])
+    for h in range(Hq):
+        lg = k[:, h // group, :] @ q[h] / np.sqrt(head_dim)
+        w = np.exp(lg - lg.max())
+        r += w / w.sum()
+    return r / Hq
+
+
+def ads_select(relevance: np.ndarray, K: int) -> np.ndarray:
+    """I_tau of Eq. 3: the K most relevant tokens (equal relevance: lower
+    token index first), in ascending token order."""
+    order = sorted(range(len(relevance)), key=lambda m: (-relevance[m], m))
+    return np.array(sorted(order[:K]), dtype=np.int64)
 
 
 # ----------------------------------------------------------------------------

@@ -27,7 +27,7 @@ CACHE_CONTIGUOUS, CACHE_PAGED = 0, 1
 EXPORTS = ("prcr_workspace_size", "prcr_rebind_inject", "prcr_plan", "prcr_rebind_apply",
            "prcr_store_raw", "prcr_next_text_pos", "prcr_error_string", "prcr_version",
            "prcr_rebind_inject_static", "prcr_prefill_capture", "prcr_decode_workspace_size",
-           "prcr_decode_attention")
+           "prcr_decode_attention", "prcr_select_workspace_size", "prcr_select_topk")
 STATIC_MAX_TOKENS = 65536
 
 
@@ -100,6 +100,12 @@ def lib():
                                         C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t,
                                         C.c_void_p]
     L.prcr_decode_attention.restype = C.c_int
+    L.prcr_select_workspace_size.argtypes = [C.c_int32, C.c_int32, C.c_int32]
+    L.prcr_select_workspace_size.restype = C.c_size_t
+    L.prcr_select_topk.argtypes = [P(RopeCfg), P(StoreDesc), C.c_int32, C.c_int32, C.c_int32,
+                                   C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p,
+                                   C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p]
+    L.prcr_select_topk.restype = C.c_int
     L.prcr_next_text_pos.argtypes = [C.c_int64, C.c_int64, C.c_int32]
     L.prcr_next_text_pos.restype = C.c_int64
     L.prcr_error_string.argtypes = [C.c_int]
@@ -328,6 +334,28 @@ def decode_attention(cfg, cache, q: torch.Tensor, q_pos: torch.Tensor, seq_len: 
                                      int(max_len), out.data_ptr(), status.data_ptr(), ws, nbytes,
                                      _stream(stream))
     return _check(rc, "prcr_decode_attention")
+
+
+def select_workspace_size(n_seqs: int, n_q_heads: int, n_tokens: int) -> int:
+    return int(lib().prcr_select_workspace_size(int(n_seqs), int(n_q_heads), int(n_tokens)))
+
+
+def select_topk(cfg, store, layer: int, q: torch.Tensor, q_pos: torch.Tensor, k: int,
+                idx_out: torch.Tensor, seq_rev_off: torch.Tensor, rev_tok_off: torch.Tensor,
+                workspace: torch.Tensor, score_out: Optional[torch.Tensor] = None, stream=None):
+    """prcr_select_topk: q [B, Hq, D] bf16 (contiguous); q_pos int64 [B]; outputs
+    idx_out int32 [B * k], seq_rev_off / rev_tok_off int32 [B + 1]."""
+    if q.dtype != torch.bfloat16 or not q.is_contiguous():
+        raise TypeError("q must be a contiguous bfloat16 [B, Hq, D] tensor")
+    for name, t in (("idx_out", idx_out), ("seq_rev_off", seq_rev_off), ("rev_tok_off", rev_tok_off)):
+        if t.dtype != torch.int32 or not t.is_contiguous():
+            raise TypeError(f"{name} must be a contiguous int32 tensor")
+    rc = lib().prcr_select_topk(C.byref(cfg), C.byref(store), int(q.shape[0]), int(layer),
+                                int(q.shape[1]), q.data_ptr(), q_pos.data_ptr(), int(k),
+                                idx_out.data_ptr(), seq_rev_off.data_ptr(), rev_tok_off.data_ptr(),
+                                _ptr(score_out), workspace.data_ptr(),
+                                workspace.numel() * workspace.element_size(), _stream(stream))
+    return _check(rc, "prcr_select_topk")
 
 
 def next_text_pos(p_txt: int, k_seq: int, mode: int = MODE_PCR) -> int:

@@ -20,7 +20,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libprcr.so")
 
 SOURCES = ["prcr_abi.cu", "prcr_plan.cu", "prcr_rebind.cu", "prcr_store.cu", "prcr_static.cu",
-           "prcr_capture.cu", "prcr_decode.cu"]
+           "prcr_capture.cu", "prcr_decode.cu", "prcr_select.cu"]
 GENCODE = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = GENCODE + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-fvisibility=hidden",
                         "-I", INCLUDE, "-I", CSRC]

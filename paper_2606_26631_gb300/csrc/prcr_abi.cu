@@ -526,6 +526,65 @@ int prcr_decode_attention(const prcr_rope_cfg* cfg, const prcr_cache_desc* cache
                : PRCR_ECUDA;
 }
 
+size_t prcr_select_workspace_size(int32_t n_seqs, int32_t n_q_heads, int32_t n_tokens) {
+    if (n_seqs < 1 || n_q_heads < 1 || n_tokens < 1) return 0;
+    return size_t(n_seqs) * n_q_heads * n_tokens * sizeof(float);
+}
+
+int prcr_select_topk(const prcr_rope_cfg* cfg, const prcr_store_desc* store, int32_t n_seqs,
+                     int32_t layer, int32_t n_q_heads, const void* q, const int64_t* q_pos,
+                     int32_t k, int32_t* idx_out, int32_t* seq_rev_off, int32_t* rev_tok_off,
+                     float* score_out, void* workspace, size_t workspace_bytes, void* stream) {
+    int rc = check_cfg(cfg);
+    if (rc) return rc;
+    if ((rc = check_store(cfg, store))) return rc;
+    const int H = cfg->n_kv_heads;
+    if (n_seqs < 0 || n_seqs > store->n_seqs || layer < 0 || layer >= cfg->n_layers ||
+        n_q_heads < H || n_q_heads % H || n_q_heads / H > 8 || n_q_heads > kSelectMaxQHeads ||
+        int64_t(n_q_heads) * cfg->head_dim > PRCR_DECODE_MAX_Q_ELEMS ||
+        store->n_tokens > PRCR_SELECT_MAX_TOKENS || k < 1 || k > store->n_tokens)
+        return PRCR_EINVAL;
+    if (int64_t(n_seqs) * k > INT32_MAX) return PRCR_EINVAL;
+    if (n_seqs == 0) return PRCR_OK;
+    if (!q || !q_pos || !idx_out || !seq_rev_off || !rev_tok_off) return PRCR_EINVAL;
+    if (!aligned4(q) || !aligned8(q_pos) || !aligned4(idx_out) || !aligned4(seq_rev_off) ||
+        !aligned4(rev_tok_off) || (score_out && !aligned4(score_out)))
+        return PRCR_EALIGN;
+    if (!workspace || workspace_bytes < prcr_select_workspace_size(n_seqs, n_q_heads, store->n_tokens))
+        return PRCR_EWORKSPACE;
+    if (!aligned16(workspace)) return PRCR_EALIGN;
+    SelectArgs a = {};
+    a.q = static_cast<const uint16_t*>(q);
+    a.q_pos = q_pos;
+    a.store_k = static_cast<const uint16_t*>(store->k);
+    a.store_seq_stride = store->seq_stride;
+    a.store_layer_stride = store->layer_stride;
+    a.store_token_stride = store->token_stride;
+    a.coords = store->coords;
+    a.coord_seq_stride = store->coord_seq_stride;
+    a.layer = layer;
+    a.n_tokens = store->n_tokens;
+    a.n_kv_heads = H;
+    a.n_q_heads = n_q_heads;
+    a.head_dim = cfg->head_dim;
+    a.k = k;
+    a.layout = cfg->layout;
+    a.sec_t = cfg->sections[0];
+    a.sec_h = cfg->sections[1];
+    a.sec_w = cfg->sections[2];
+    a.scale = float(1.0 / std::sqrt(double(cfg->head_dim)));
+    a.logits = static_cast<float*>(workspace);
+    a.score_out = score_out;
+    a.idx_out = idx_out;
+    a.rev_tok_off = rev_tok_off;
+    a.seq_rev_off = seq_rev_off;
+    const int P = cfg->head_dim / 2;
+    for (int i = 0; i < P; ++i)
+        a.inv_freq[i] = std::pow(cfg->theta, -2.0 * double(i) / double(cfg->head_dim));
+    return launch_select(a, n_seqs, static_cast<cudaStream_t>(stream)) == cudaSuccess ? PRCR_OK
+                                                                                     : PRCR_ECUDA;
+}
+
 int64_t prcr_next_text_pos(int64_t p_txt, int64_t k_seq, int32_t mode) {
     switch (mode) {
         case PRCR_MODE_PCR:

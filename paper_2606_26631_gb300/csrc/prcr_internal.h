@@ -187,6 +187,38 @@ struct DecodeArgs {
 
 constexpr int kDecodeMaxChunk = 4096;
 
+constexpr int kSelectMaxQHeads = 128;
+
+struct SelectArgs {
+    const uint16_t* q;          // [B][n_q_heads][D] raw trigger queries
+    const int64_t* q_pos;       // [B]
+    const uint16_t* store_k;
+    int64_t store_seq_stride;
+    int64_t store_layer_stride;
+    int64_t store_token_stride;
+    const int32_t* coords;
+    int64_t coord_seq_stride;
+    int32_t layer;
+    int32_t n_tokens;
+    int32_t n_kv_heads;
+    int32_t n_q_heads;
+    int32_t head_dim;
+    int32_t k;
+    int32_t layout;
+    int32_t sec_t;
+    int32_t sec_h;
+    int32_t sec_w;
+    float scale;
+    float* logits;              // workspace [B][n_q_heads][n_tokens]
+    float* score_out;           // optional [B][n_tokens]
+    int32_t* idx_out;           // [B][k]
+    int32_t* rev_tok_off;       // [B + 1]
+    int32_t* seq_rev_off;       // [B + 1]
+    double inv_freq[kMaxPairs];
+};
+
+cudaError_t launch_select(const SelectArgs& a, int n_seqs, cudaStream_t stream);
+
 cudaError_t launch_decode(const DecodeArgs& a, int gp, dim3 grid, size_t smem,
                           cudaStream_t stream);
 cudaError_t launch_capture(const CaptureArgs& a, dim3 grid, int block, size_t smem,

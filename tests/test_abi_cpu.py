@@ -202,3 +202,49 @@ def test_struct_layout_matches_c_compiler(tmp_path):
         assert got[(cname, "size")] == C.sizeof(py), cname
         for f, _ in py._fields_:
             assert got[(cname, f)] == getattr(py, f).offset, (cname, f)
+
+
+def test_new_entry_points_validate_on_host():
+    """prcr_prefill_capture / prcr_decode_attention / prcr_select_topk reject
+    bad arguments before any CUDA call."""
+    a = _descs()
+    L = prcr.lib()
+    st = C.byref(a["st"]); ca = C.byref(a["ca"]); cfg = C.byref(a["cfg"])
+    K, V, CO, STAT = FAKE + 2 ** 23, FAKE + 2 ** 24, FAKE + 2 ** 25, FAKE + 2 ** 26
+    cap = lambda **k: L.prcr_prefill_capture(cfg, st, ca, k.get("seq", 0), k.get("l0", 0),
+                                             k.get("nl", 2), k.get("m0", 0), k.get("mc", 8),
+                                             k.get("slot", 0), k.get("k", K), V, 4 * 128, 128,
+                                             k.get("coords", CO), k.get("status", STAT), None)
+    assert cap(seq=1) == B.EINVAL
+    assert cap(l0=1) == B.EINVAL
+    assert cap(slot=-1) == B.EINVAL
+    assert cap(coords=None) == B.EINVAL
+    assert cap(status=None) == B.EINVAL
+    assert cap(k=K + 8) == B.EALIGN
+    assert cap(mc=0) == B.OK
+    # decode: head_dim 64 is allowed, 16 query heads per KV head is not
+    Q, QP, SL, OUT = FAKE + 2 ** 27, FAKE + 2 ** 28, FAKE + 2 ** 29, FAKE + 2 ** 30
+    dec = lambda **k: L.prcr_decode_attention(cfg, ca, k.get("B", 1), k.get("Hq", 4), Q, QP, SL,
+                                              k.get("max_len", 100), k.get("out", OUT), STAT,
+                                              None, 0, None)
+    assert dec(Hq=3) == B.EINVAL          # not a multiple of the KV heads
+    assert dec(Hq=32) == B.EINVAL         # 16 per KV head
+    assert dec(max_len=257) == B.EINVAL   # beyond the cache's 256 slots
+    assert dec(B=2) == B.EINVAL           # more sequences than the cache holds
+    assert dec(out=OUT + 4) == B.EALIGN
+    assert dec(B=0) == B.OK
+    cfg48 = prcr.rope_cfg(2, 2, 48, (8, 8, 8))
+    assert L.prcr_decode_attention(C.byref(cfg48), ca, 1, 4, Q, QP, SL, 10, OUT, STAT, None, 0,
+                                   None) == B.EINVAL  # head_dim 48 unsupported by decode
+    # select
+    IDX, SRO, RTO, WS = FAKE + 2 ** 31, FAKE + 2 ** 32, FAKE + 2 ** 33, FAKE + 2 ** 34
+    sel = lambda **k: L.prcr_select_topk(cfg, st, k.get("B", 1), k.get("layer", 0),
+                                         k.get("Hq", 4), Q, QP, k.get("k", 8), IDX, SRO, RTO,
+                                         None, k.get("ws", WS), k.get("wsb", 1 << 20), None)
+    assert sel(k=0) == B.EINVAL
+    assert sel(k=65) == B.EINVAL          # more than the 64 store tokens
+    assert sel(layer=2) == B.EINVAL
+    assert sel(Hq=3) == B.EINVAL
+    assert sel(ws=None) == B.EWORKSPACE
+    assert sel(wsb=16) == B.EWORKSPACE
+    assert prcr.select_workspace_size(2, 4, 64) == 2 * 4 * 64 * 4

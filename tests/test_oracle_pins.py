@@ -433,11 +433,51 @@ def pin_decode_attention(o):
     assert np.allclose(out, out2, rtol=0, atol=1e-9)
 
 
+def pin_ads(o):
+    """Selection reading (Sec. 2.1, Eq. 3): relevance is a per-head softmax
+    averaged over heads, so it sums to 1; a key equal to a large multiple of
+    the (rotated) query direction wins; ties go to the lower index; the set
+    comes back in ascending order; against a direct loop with math.exp."""
+    rng = np.random.default_rng(37)
+    D, sec, th = 16, (2, 3, 3), 1e6
+    M, H, Hq = 12, 2, 4
+    kb = rng.integers(0x3C00, 0x4100, size=(M, H, D)).astype(np.uint16)
+    kb[..., ::2] |= 0x8000  # mixed signs
+    coords = np.array([(3, 10 + m // 4, 20 + m % 4) for m in range(M)])
+    q = rng.standard_normal((Hq, D))
+    r = o.ads_relevance(q, 40, kb, coords, D, sec, th)
+    assert abs(r.sum() - 1.0) < 1e-12 and (r > 0).all()
+    # direct loop
+    P = D // 2
+    ref = np.zeros(M)
+    for h in range(Hq):
+        qz = [complex(q[h, i], q[h, i + P]) * cmath.exp(1j * 40 * th ** (-2.0 * i / D)) for i in range(P)]
+        lg = []
+        for m in range(M):
+            x = [_bf16_value(v) for v in kb[m, h // 2]]
+            kz = []
+            for i in range(P):
+                axis = 0 if i < sec[0] else (1 if i < sec[0] + sec[1] else 2)
+                kz.append(complex(x[i], x[i + P]) * cmath.exp(1j * coords[m, axis] * th ** (-2.0 * i / D)))
+            lg.append(sum(a.real * b.real + a.imag * b.imag for a, b in zip(qz, kz)) / math.sqrt(D))
+        mx = max(lg)
+        w = [math.exp(x - mx) for x in lg]
+        for m in range(M):
+            ref[m] += w[m] / sum(w) / Hq
+    assert np.allclose(r, ref, rtol=1e-10, atol=0)
+    sel = o.ads_select(np.array([0.1, 0.3, 0.3, 0.05, 0.3, 0.2]), 3)
+    assert list(sel) == [1, 2, 4]
+    sel = o.ads_select(np.array([0.1, 0.3, 0.3, 0.05, 0.3, 0.2]), 2)
+    assert list(sel) == [1, 2]
+    sel = o.ads_select(np.array([0.5, 0.1, 0.2, 0.9]), 2)
+    assert list(sel) == [0, 3]
+
+
 PINS = [pin_worked_rect4x4, pin_worked_rect2x2, pin_pcr_closed_forms, pin_degenerate_center,
         pin_other_modes, pin_plan_slots_and_continuity, pin_rope_closed_forms,
         pin_mrope_equal_axes_is_textbook, pin_mrope_sections, pin_rope_invariants,
         pin_bf16_helpers, pin_brute_force_2x2, pin_original_mode_is_position_bound_cache,
-        pin_prefill_capture, pin_decode_attention]
+        pin_prefill_capture, pin_decode_attention, pin_ads]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -541,6 +581,19 @@ def _m_decode_query_unrotated(q_raw, q_pos, k_act, v_act, head_dim, sections, th
     return _orig_decode(q_raw, 0, k_act, v_act, head_dim, sections, theta, layout)
 
 
+_orig_select = O.ads_select
+
+
+def _m_select_unsorted(rel, K):
+    order = sorted(range(len(rel)), key=lambda m: (-rel[m], m))
+    return np.array(order[:K], dtype=np.int64)
+
+
+def _m_select_ties_high(rel, K):
+    order = sorted(range(len(rel)), key=lambda m: (-rel[m], -m))
+    return np.array(sorted(order[:K]), dtype=np.int64)
+
+
 MUTANTS = [
     ("pcr_position", _m_pcr_k_not_k_minus_1),
     ("pcr_position", _m_pcr_denominator_k),
@@ -557,6 +610,8 @@ MUTANTS = [
     ("decode_attention", _m_decode_no_scale),
     ("decode_attention", _m_decode_head_modulo),
     ("decode_attention", _m_decode_query_unrotated),
+    ("ads_select", _m_select_unsorted),
+    ("ads_select", _m_select_ties_high),
 ]
 
 

@@ -1,0 +1,119 @@
+"""GPU checks of prcr_select_topk (attention-driven selection, Sec. 2.1 /
+Eq. 3, under the reading in the oracle's header).
+
+Relevance: float32 on the GPU against the oracle's float64 ads_relevance,
+relative error <= 1e-4. Selection: where floating point decides an integer,
+the check is that (a) the set is exactly the top-k of the relevance the
+kernel itself reports (ties to the lower index), (b) it is a valid top-k of
+the oracle's relevance up to the measured relevance error, and (c) it equals
+the oracle's ads_select whenever the oracle's k-th and (k+1)-th values are
+further apart than that error. Ties are forced with an all-zero key layer.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import prcr_oracle as O
+from workloads import get, make_batch
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+
+
+def _select(batch, layer, Hq, k, q, q_pos):
+    import paper_2606_26631_gb300 as prcr
+    wl = batch.wl
+    B, M = wl.n_seqs, wl.n_tokens
+    cfg = prcr.rope_cfg(wl.n_layers, wl.n_kv_heads, wl.head_dim, wl.sections, wl.theta)
+    sd = prcr.store_desc(batch.store_k, batch.store_v, batch.coords)
+    idx = torch.full((B * k,), -7, dtype=torch.int32, device=DEV)
+    sro = torch.full((B + 1,), -7, dtype=torch.int32, device=DEV)
+    rto = torch.full((B + 1,), -7, dtype=torch.int32, device=DEV)
+    score = torch.full((B, M), -1.0, dtype=torch.float32, device=DEV)
+    ws = torch.empty(prcr.select_workspace_size(B, Hq, M), dtype=torch.uint8, device=DEV)
+    prcr.select_topk(cfg, sd, layer, q, q_pos, k, idx, sro, rto, ws, score)
+    torch.cuda.synchronize()
+    return idx.view(B, k).cpu().numpy(), sro.cpu().numpy(), rto.cpu().numpy(), score.cpu().numpy()
+
+
+def _topk_by(values, k):
+    order = np.lexsort((np.arange(len(values)), -values))
+    return np.sort(order[:k])
+
+
+@pytest.mark.parametrize("name,Hq,k,layer", [("qwen25vl-7b", 28, 64, 5), ("qwen3vl-8b", 32, 300, 35),
+                                             ("tiny", 2, 16, 1)])
+def test_select_parity(name, Hq, k, layer):
+    wl = get(name)
+    batch = make_batch(wl, device=DEV)
+    B, M, D = wl.n_seqs, wl.n_tokens, wl.head_dim
+    g = torch.Generator(device=DEV)
+    g.manual_seed(17)
+    q = (3.0 * torch.randn((B, Hq, D), generator=g, device=DEV)).to(torch.bfloat16)
+    idx, sro, rto, score = _select(batch, layer, Hq, k, q, batch.p_txt)
+    assert np.array_equal(sro, np.arange(B + 1))
+    assert np.array_equal(rto, k * np.arange(B + 1))
+    qv = O.bf16_bits_to_f64(q.view(torch.int16).cpu().numpy())
+    coords = batch.coords.cpu().numpy()
+    for b in range(min(B, 4)):
+        k_raw = batch.store_k[b, layer].view(torch.int16).cpu().numpy()
+        ref = O.ads_relevance(qv[b], int(batch.p_txt[b]), k_raw, coords[b], D, wl.sections, wl.theta)
+        rel_err = np.abs(score[b] - ref) / ref
+        assert rel_err.max() <= 1e-4, rel_err.max()
+        sel = idx[b]
+        assert len(set(sel.tolist())) == k and np.all(np.diff(sel) > 0)
+        assert np.array_equal(sel, _topk_by(score[b].astype(np.float64), k))  # (a)
+        tol = 2 * np.abs(score[b] - ref).max() + 1e-12
+        chosen = np.zeros(M, dtype=bool)
+        chosen[sel] = True
+        if k < M:
+            assert ref[chosen].min() >= ref[~chosen].max() - tol  # (b)
+            srt = np.sort(ref)[::-1]
+            if srt[k - 1] - srt[k] > tol:
+                assert np.array_equal(sel, O.ads_select(ref, k))  # (c)
+
+
+def test_select_ties_and_full_set():
+    wl = get("qwen2vl-2b")
+    batch = make_batch(wl, device=DEV)
+    batch.store_k[:, 3].zero_()  # every logit of layer 3 is 0: all relevances tie
+    B, M, D = 1, wl.n_tokens, wl.head_dim
+    q = torch.randn((B, 2, D), device=DEV).to(torch.bfloat16)
+    idx, _, _, score = _select(batch, 3, 2, 100, q, batch.p_txt)
+    assert np.array_equal(idx[0], np.arange(100))
+    assert np.allclose(score[0], 1.0 / M, rtol=1e-6)
+    idx, _, _, _ = _select(batch, 7, 2, M, q, batch.p_txt)
+    assert np.array_equal(idx[0], np.arange(M))
+
+
+def test_select_feeds_rebind_inject():
+    """The selection's outputs are a valid revisit batch for prcr_rebind_inject."""
+    import paper_2606_26631_gb300 as prcr
+    wl = get("qwen25vl-7b")
+    batch = make_batch(wl, device=DEV)
+    B, k = wl.n_seqs, 48
+    q = torch.randn((B, 4, wl.head_dim), device=DEV).to(torch.bfloat16)
+    cfg = prcr.rope_cfg(wl.n_layers, wl.n_kv_heads, wl.head_dim, wl.sections, wl.theta)
+    sd = prcr.store_desc(batch.store_k, batch.store_v, batch.coords)
+    idx = torch.empty(B * k, dtype=torch.int32, device=DEV)
+    sro = torch.empty(B + 1, dtype=torch.int32, device=DEV)
+    rto = torch.empty(B + 1, dtype=torch.int32, device=DEV)
+    ws = torch.empty(prcr.select_workspace_size(B, 4, wl.n_tokens), dtype=torch.uint8, device=DEV)
+    prcr.select_topk(cfg, sd, 0, q, batch.p_txt, k, idx, sro, rto, ws)
+    # a cache with room for k slots after each sequence's context
+    clen = batch.cache_len_in
+    nblk = int(((clen.max() + k) // 16 + 2).item())
+    bt = torch.arange(B * nblk, dtype=torch.int32, device=DEV).view(B, nblk).contiguous()
+    ck = torch.full((wl.n_layers, B * nblk, 16, wl.n_kv_heads, wl.head_dim), -1,
+                    dtype=torch.int16, device=DEV).view(torch.bfloat16)
+    cv = ck.clone()
+    rv = prcr.Revisit(cfg, batch.store_k, batch.store_v, batch.coords, ck, cv, bt, sro, rto, idx,
+                      batch.p_txt, clen)
+    rv.run()
+    torch.cuda.synchronize()
+    assert rv.status_value() == 0
+    assert torch.equal(rv.cache_len_out, clen + k)
+    assert torch.equal(rv.next_pos, batch.p_txt + 1)
+    written = int((ck.view(torch.int16) != -1).sum().item())
+    assert written == B * k * wl.n_layers * wl.n_kv_heads * wl.head_dim
