@@ -314,7 +314,9 @@ int do_capture(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
     return launch_capture(a, grid, block, smem, stream) == cudaSuccess ? PRCR_OK : PRCR_ECUDA;
 }
 
-constexpr size_t kDecodeSmem = 48 * 1024;  // default dynamic shared memory limit
+// dynamic shared memory of the decode kernel: under the 48 KiB default limit
+// with room for its 1 KiB of static cos/sin
+constexpr size_t kDecodeSmem = 46 * 1024;
 
 // Chunking of the decode step: enough CTAs to fill the GPU a few times over,
 // chunks a multiple of 32 slots, at most kDecodeMaxChunk and small enough for

@@ -11,7 +11,7 @@
 // then serves one KV head and the `group` query heads that share it (GQA):
 // lane i holds D/32 consecutive dimensions, so every K or V row of the head
 // is one fully coalesced warp load. S = 32 / GP slots are processed per
-// iteration (GP = group rounded up to a power of two): each lane forms its
+// iteration (GP = 4 for groups up to 4, else 8): each lane forms its
 // partial dot products for all GP x S (head, slot) pairs, and a butterfly
 // transpose-reduction (31 shuffles) leaves lane l with the complete logit of
 // pair l. The online softmax then runs per head, and P V accumulates in
@@ -30,6 +30,7 @@ constexpr double kTwoPiHi = 6.283185307179586;
 constexpr double kTwoPiLo = 2.4492935982947064e-16;
 constexpr double kInvTwoPi = 0.15915494309189535;
 constexpr unsigned kFull = 0xffffffffu;
+constexpr int kDecodeThreads = 128;
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
@@ -49,7 +50,7 @@ __device__ __forceinline__ void load_row(const uint16_t* p, uint32_t (&w)[EPL / 
 }
 
 template <int GP, int EPL>
-__global__ void __launch_bounds__(256) decode_kernel(const __grid_constant__ DecodeArgs a) {
+__global__ void __launch_bounds__(kDecodeThreads, 3) decode_kernel(const __grid_constant__ DecodeArgs a) {
     constexpr int S = 32 / GP;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int D = a.head_dim;
@@ -71,17 +72,23 @@ __global__ void __launch_bounds__(256) decode_kernel(const __grid_constant__ Dec
     const int64_t s_end = min(len, s_begin + a.chunk);
 
     // Query heads of (b, l), rotated at (p, p, p) and scaled by 1/sqrt(D).
+    // With the same position on every axis, pair i turns by p * inv_freq_i
+    // whatever its band, so each pair's cos/sin serves all heads.
+    __shared__ float s_cos[kMaxPairs], s_sin[kMaxPairs];
     const int64_t p = a.q_pos[b];
-    const uint16_t* qb = a.q + (int64_t(b) * a.n_layers + l) * Hq * D;
-    for (int e = threadIdx.x; e < Hq * P; e += blockDim.x) {
-        const int hq = e / P;
-        const int i = e - hq * P;
+    for (int i = threadIdx.x; i < P; i += blockDim.x) {
         const double ang = double(p) * a.inv_freq[i];
         const double k = rint(ang * kInvTwoPi);
         double r = fma(-k, kTwoPiHi, ang);
         r = fma(-k, kTwoPiLo, r);
-        float sn, cs;
-        sincosf(float(r), &sn, &cs);
+        sincosf(float(r), &s_sin[i], &s_cos[i]);
+    }
+    __syncthreads();
+    const uint16_t* qb = a.q + (int64_t(b) * a.n_layers + l) * Hq * D;
+    for (int e = threadIdx.x; e < Hq * P; e += blockDim.x) {
+        const int hq = e / P;
+        const int i = e - hq * P;
+        const float sn = s_sin[i], cs = s_cos[i];
         const float x = __uint_as_float(uint32_t(qb[hq * D + i]) << 16);
         const float y = __uint_as_float(uint32_t(qb[hq * D + i + P]) << 16);
         q_s[hq * D + i] = fmaf(x, cs, -y * sn) * a.scale;
@@ -133,22 +140,40 @@ __global__ void __launch_bounds__(256) decode_kernel(const __grid_constant__ Dec
         const uint16_t* kbase = a.cache_k + lstride + int64_t(kh) * D + lane * EPL;
         const uint16_t* vbase = a.cache_v + lstride + int64_t(kh) * D + lane * EPL;
 
+        // Software pipeline: the K/V rows of the next S slots are requested
+        // before the current S slots are reduced, so every warp keeps its
+        // loads in flight while it runs the shuffle and softmax work.
+        uint32_t kn[S][EPL / 2], vn[S][EPL / 2];
+        bool okn[S];
+        auto fetch = [&](int64_t s0) {
+#pragma unroll
+            for (int si = 0; si < S; ++si) {
+                const int64_t s = s0 + si;
+                const int64_t row = s < s_end ? row_s[s - s_begin] : -1;
+                okn[si] = row >= 0;
+                if (okn[si]) {
+                    load_row<EPL>(kbase + row, kn[si]);
+                    load_row<EPL>(vbase + row, vn[si]);
+                } else {
+#pragma unroll
+                    for (int w = 0; w < EPL / 2; ++w) kn[si][w] = vn[si][w] = 0u;
+                }
+            }
+        };
+        if (s_begin < s_end) fetch(s_begin);
         for (int64_t s0 = s_begin; s0 < s_end; s0 += S) {
             uint32_t kw[S][EPL / 2], vw[S][EPL / 2];
             bool ok[S];
 #pragma unroll
             for (int si = 0; si < S; ++si) {
-                const int64_t s = s0 + si;
-                const int64_t row = s < s_end ? row_s[s - s_begin] : -1;
-                ok[si] = row >= 0;
-                if (ok[si]) {
-                    load_row<EPL>(kbase + row, kw[si]);
-                    load_row<EPL>(vbase + row, vw[si]);
-                } else {
+                ok[si] = okn[si];
 #pragma unroll
-                    for (int w = 0; w < EPL / 2; ++w) kw[si][w] = vw[si][w] = 0u;
+                for (int w = 0; w < EPL / 2; ++w) {
+                    kw[si][w] = kn[si][w];
+                    vw[si][w] = vn[si][w];
                 }
             }
+            if (s0 + S < s_end) fetch(s0 + S);
             // partial dot products of this lane's dimensions, index h * S + si
             float val[32];
 #pragma unroll
@@ -263,9 +288,9 @@ __global__ void __launch_bounds__(256) decode_merge_kernel(const __grid_constant
 template <int GP>
 cudaError_t launch_gp(const DecodeArgs& a, dim3 grid, size_t smem, cudaStream_t stream) {
     switch (a.head_dim) {
-        case 64: decode_kernel<GP, 2><<<grid, 256, smem, stream>>>(a); break;
-        case 128: decode_kernel<GP, 4><<<grid, 256, smem, stream>>>(a); break;
-        default: decode_kernel<GP, 8><<<grid, 256, smem, stream>>>(a); break;
+        case 64: decode_kernel<GP, 2><<<grid, kDecodeThreads, smem, stream>>>(a); break;
+        case 128: decode_kernel<GP, 4><<<grid, kDecodeThreads, smem, stream>>>(a); break;
+        default: decode_kernel<GP, 8><<<grid, kDecodeThreads, smem, stream>>>(a); break;
     }
     return cudaGetLastError();
 }
@@ -274,13 +299,10 @@ cudaError_t launch_gp(const DecodeArgs& a, dim3 grid, size_t smem, cudaStream_t 
 
 cudaError_t launch_decode(const DecodeArgs& a, int gp, dim3 grid, size_t smem,
                           cudaStream_t stream) {
-    cudaError_t e;
-    switch (gp) {
-        case 1: e = launch_gp<1>(a, grid, smem, stream); break;
-        case 2: e = launch_gp<2>(a, grid, smem, stream); break;
-        case 4: e = launch_gp<4>(a, grid, smem, stream); break;
-        default: e = launch_gp<8>(a, grid, smem, stream); break;
-    }
+    // groups of 1, 2 and 4 query heads run as 4 (padded) heads x 8 slots per
+    // warp iteration, groups of 5..8 as 8 heads x 4 slots
+    const cudaError_t e = gp <= 4 ? launch_gp<4>(a, grid, smem, stream)
+                                  : launch_gp<8>(a, grid, smem, stream);
     if (e != cudaSuccess || a.splits == 1) return e;
     const unsigned n = unsigned(int64_t(grid.z) * a.n_layers * a.n_q_heads);
     decode_merge_kernel<<<n, a.head_dim < 256 ? a.head_dim : 256, 0, stream>>>(a);

@@ -57,12 +57,15 @@ __global__ void __launch_bounds__(256) ads_logits_kernel(const __grid_constant__
     const int b = blockIdx.y;
     const int m0 = blockIdx.x * kTokTile;
 
+    // the query sits at (p, p, p): pair i turns by p * inv_freq_i for every head
+    __shared__ float s_qc[kMaxPairs], s_qs[kMaxPairs];
     const int64_t p = a.q_pos[b];
+    for (int i = threadIdx.x; i < P; i += blockDim.x) sincos_reduced(double(p) * a.inv_freq[i], &s_qs[i], &s_qc[i]);
+    __syncthreads();
     const uint16_t* qb = a.q + int64_t(b) * Hq * D;
     for (int e = threadIdx.x; e < Hq * P; e += blockDim.x) {
         const int hq = e / P, i = e - (e / P) * P;
-        float sn, cn;
-        sincos_reduced(double(p) * a.inv_freq[i], &sn, &cn);
+        const float sn = s_qs[i], cn = s_qc[i];
         const float x = __uint_as_float(uint32_t(qb[hq * D + i]) << 16);
         const float y = __uint_as_float(uint32_t(qb[hq * D + i + P]) << 16);
         q_s[hq * qs + i] = fmaf(x, cn, -y * sn) * a.scale;
