@@ -57,9 +57,10 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["prcr", "reference"], default="prcr")
     ap.add_argument("--workload", default="stress")
-    ap.add_argument("--path", choices=["revisit", "capture", "decode"], default="revisit",
+    ap.add_argument("--path", choices=["revisit", "capture", "decode", "select"], default="revisit",
                     help="revisit: the rebind+inject step (default); capture: prefill capture; "
-                         "decode: the first decode step over the active cache")
+                         "decode: the first decode step over the active cache; select: the "
+                         "attention-driven selection of the revisited set")
     ap.add_argument("--seqs", type=int, default=0, help="capture/decode: sequences (0 = workload's)")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -537,6 +538,53 @@ def run_decode_path(args):
         gpu_launches=(2 if nws else 1) * args.steps, clocks=clk)), flush=True)
 
 
+def run_select_path(args):
+    """Attention-driven selection of K tokens per sequence at one layer."""
+    import torch
+    _, _, local = dist_env()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    from paper_2606_26631_gb300 import _build
+    if not _build.up_to_date():
+        _build.build()
+    import paper_2606_26631_gb300 as prcr
+    from workloads import get, make_batch
+    wl = get(args.workload)
+    if args.seqs:
+        wl = dataclasses.replace(wl, n_seqs=args.seqs)
+    batch = make_batch(wl, device=dev)
+    B, M, H, D = wl.n_seqs, wl.n_tokens, wl.n_kv_heads, wl.head_dim
+    Hq, k, layer = 4 * H, max(1, batch.total_k // B), wl.n_layers - 1
+    q = torch.randn((B, Hq, D), device=dev, generator=torch.Generator(device=dev).manual_seed(3)
+                    ).to(torch.bfloat16)
+    cfg = prcr.rope_cfg(wl.n_layers, H, D, wl.sections, wl.theta)
+    sd = prcr.store_desc(batch.store_k, batch.store_v, batch.coords)
+    idx = torch.empty(B * k, dtype=torch.int32, device=dev)
+    sro = torch.empty(B + 1, dtype=torch.int32, device=dev)
+    rto = torch.empty(B + 1, dtype=torch.int32, device=dev)
+    ws = torch.empty(prcr.select_workspace_size(B, Hq, M), dtype=torch.uint8, device=dev)
+
+    def step():
+        prcr.select_topk(cfg, sd, layer, q, batch.p_txt, k, idx, sro, rto, ws)
+
+    ms, clk = _timed(step, args.steps, args.warmup, local)
+    nbytes = B * M * H * D * 2  # the layer's raw keys, read once
+    t = sum(ms) / 1e3
+    peak, kind = measured_peaks()
+    value = nbytes * args.steps / t / 1e9
+    print(json.dumps(dict(
+        metric="selection GB/s (raw keys read)", value=value, unit=UNIT, n_gpus=1,
+        steps=args.steps, warmup=args.warmup, ms_per_step=1e3 * t / args.steps,
+        us_per_sequence=1e6 * t / args.steps / B, higher_is_better=True, scaling="weak",
+        vs_baseline=None, dtype="f32", io_dtype="bf16", data="synthetic",
+        config=dict(workload=wl.name, batch=B, tokens_per_seq=M, n_q_heads=Hq, k=k, layer=layer,
+                    bytes_per_step=nbytes),
+        roofline=dict(bound="hbm", achieved=value, peak=peak, unit="GB/s", frac=value / peak,
+                      traffic=None, kernel="ads_logits_kernel + ads_select_kernel",
+                      peak_kind=f"{kind} copy (hbm_gbs)"),
+        gpu_launches=2 * args.steps, clocks=clk)), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -545,6 +593,8 @@ def main():
         run_capture_path(args)
     elif args.path == "decode":
         run_decode_path(args)
+    elif args.path == "select":
+        run_select_path(args)
     else:
         run_gpu(args)
 
