@@ -265,6 +265,280 @@ __global__ void __launch_bounds__(kDecodeThreads, 3) decode_kernel(const __grid_
     }
 }
 
+// ---------------------------------------------------------------------------
+// Tensor-core variant (head_dim 64 and 128), mma.sync m16n8k16 bf16 -> fp32.
+//
+// A warp serves one KV head and its group of g <= 8 query heads over 16 slots
+// per iteration; the next 16 slots' K rows (registers) and V rows (shared
+// memory) are requested right after the current QK, so they are in flight
+// during the softmax and P V of the current slots.
+//   QK:  S (16 heads x 8 slots, rows >= g zero) = Q (16 x 16 dims) x K^T, two
+//        n-tiles of 8 slots, D/16 k-steps. The dot product does not depend on
+//        the order of the dimensions, so k-step j of lane group t uses the four
+//        dimensions t*D/4 + 4j .. +3: each lane then loads its slot's 64
+//        contiguous bytes (D = 128) straight into B fragments.
+//   PV:  O^T (16 dims x 8 heads) += V^T (16 dims x 16 slots) x P^T (16 slots x
+//        8 heads). The QK accumulator of lane (g, t) holds head g at slots 2t,
+//        2t+1 (tile 0) and 2t+8, 2t+9 (tile 1): exactly the P^T B fragment.
+//        V tiles are staged in shared memory with cp.async (double-buffered)
+//        and read as A fragments with ldmatrix.trans.
+// bf16 operands hold only 8 significant bits, so the float32 query and the
+// float32 probabilities are each split into a bf16 head and a bf16 remainder
+// (two MMAs each): products stay exact and the result keeps ~16 bits per
+// operand, float32-accumulated. K and V are bf16 already and enter exactly.
+__device__ __forceinline__ void mma_bf16(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                         uint32_t a3, uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+        "{%8,%9}, {%0,%1,%2,%3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+// (head, remainder) bf16 pairs of two floats
+__device__ __forceinline__ void split2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+    hi = pack2(x0, x1);
+    lo = pack2(x0 - bf16_lo(hi), x1 - bf16_hi(hi));
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+                 "r"(src_bytes)
+                 : "memory");
+}
+
+template <int D>
+__global__ void __launch_bounds__(kDecodeThreads, 3)
+    decode_mma_kernel(const __grid_constant__ DecodeArgs a) {
+    constexpr int KS = D / 16;     // k-steps of QK, m-tiles of PV
+    constexpr int LV = D / 32;     // 16-byte K loads per lane per slot
+    constexpr int PITCH = D + 8;   // bf16 per staged V row (pad: conflict-free ldmatrix)
+    constexpr int VCH = D / 8;     // 16-byte chunks per V row
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int Hq = a.n_q_heads;
+    const int P = D / 2;
+    float* q_s = reinterpret_cast<float*>(smem_raw);
+    uint16_t* vbuf = reinterpret_cast<uint16_t*>(smem_raw + size_t(Hq) * D * sizeof(float));
+    const int b = blockIdx.z;
+    const int l = blockIdx.y;
+    const int split = blockIdx.x;
+    uint32_t err = 0;
+
+    int64_t len = a.seq_len[b];
+    if (len < 0 || len > a.capacity) {
+        err |= PRCR_ST_CAPACITY;
+        len = len < 0 ? 0 : a.capacity;
+    }
+    const int64_t s_begin = int64_t(split) * a.chunk;
+    const int64_t s_end = min(len, s_begin + a.chunk);
+
+    __shared__ float s_cos[kMaxPairs], s_sin[kMaxPairs];
+    const int64_t p = a.q_pos[b];
+    for (int i = threadIdx.x; i < P; i += blockDim.x) {
+        const double ang = double(p) * a.inv_freq[i];
+        const double k = rint(ang * kInvTwoPi);
+        double r = fma(-k, kTwoPiHi, ang);
+        r = fma(-k, kTwoPiLo, r);
+        sincosf(float(r), &s_sin[i], &s_cos[i]);
+    }
+    __syncthreads();
+    const uint16_t* qb = a.q + (int64_t(b) * a.n_layers + l) * Hq * D;
+    for (int e = threadIdx.x; e < Hq * P; e += blockDim.x) {
+        const int hq = e / P;
+        const int i = e - hq * P;
+        const float sn = s_sin[i], cs = s_cos[i];
+        const float x = __uint_as_float(uint32_t(qb[hq * D + i]) << 16);
+        const float y = __uint_as_float(uint32_t(qb[hq * D + i + P]) << 16);
+        q_s[hq * D + i] = fmaf(x, cs, -y * sn) * a.scale;
+        q_s[hq * D + i + P] = fmaf(y, cs, x * sn) * a.scale;
+    }
+    __syncthreads();
+
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    const int nwarps = blockDim.x >> 5;
+    const int gid = lane >> 2;
+    const int t = lane & 3;
+    const int g = a.group;
+    const int64_t lstride = int64_t(l) * a.layer_stride;
+    uint16_t* wv = vbuf + size_t(warp) * 2 * 16 * PITCH;
+    const uint32_t wv_s = uint32_t(__cvta_generic_to_shared(wv));
+
+    for (int kh = warp; kh < a.n_kv_heads; kh += nwarps) {
+        // Q A-fragments (rows = heads of the group; rows >= g and 8..15 are zero)
+        uint32_t qh[KS][2], ql[KS][2];
+        {
+            const bool hv = gid < g;
+            const float* qr = q_s + (kh * g + (hv ? gid : 0)) * D + t * (D / 4);
+#pragma unroll
+            for (int j = 0; j < KS; ++j) {
+                const float x0 = hv ? qr[4 * j] : 0.0f, x1 = hv ? qr[4 * j + 1] : 0.0f;
+                const float x2 = hv ? qr[4 * j + 2] : 0.0f, x3 = hv ? qr[4 * j + 3] : 0.0f;
+                split2(x0, x1, qh[j][0], ql[j][0]);
+                split2(x2, x3, qh[j][1], ql[j][1]);
+            }
+        }
+        float o[KS][4];
+#pragma unroll
+        for (int mt = 0; mt < KS; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.0f;
+        float m_run = -INFINITY, l_run = 0.0f;
+        const uint16_t* kbase = a.cache_k + lstride + int64_t(kh) * D;
+        const uint16_t* vbase = a.cache_v + lstride + int64_t(kh) * D;
+
+        uint4 kn[2][LV];
+        uint32_t mask_n = 0u;
+        // Requests tile s0 (16 slots): K rows into registers, V rows into stage st.
+        auto fetch = [&](int64_t s0, int st) {
+            const int64_t s = s0 + (lane & 15);
+            int64_t row = -1;
+            if (s < s_end) {
+                if (a.cache_kind == PRCR_CACHE_CONTIGUOUS) {
+                    row = int64_t(b) * a.seq_stride + s * a.slot_stride;
+                } else {
+                    const int64_t lb = s / a.block_size;
+                    const int32_t blk = a.block_table[int64_t(b) * a.bt_stride + lb];
+                    if (blk < 0 || blk >= a.n_blocks) err |= PRCR_ST_NO_BLOCK;
+                    else row = int64_t(blk) * a.block_stride + (s - lb * a.block_size) * a.slot_stride;
+                }
+            }
+            mask_n = __ballot_sync(kFull, row >= 0) & 0xffffu;
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) {
+                const int64_t rr = __shfl_sync(kFull, row, nt * 8 + gid);
+#pragma unroll
+                for (int u = 0; u < LV; ++u)
+                    kn[nt][u] = rr >= 0 ? __ldg(reinterpret_cast<const uint4*>(kbase + rr + t * (D / 4) + 8 * u))
+                                        : make_uint4(0u, 0u, 0u, 0u);
+            }
+#pragma unroll
+            for (int i = 0; i < (16 * VCH) / 32; ++i) {
+                const int c = lane + 32 * i;
+                const int slot = c / VCH;
+                const int piece = c - slot * VCH;
+                const int64_t rr = __shfl_sync(kFull, row, slot);
+                const uint32_t dst = wv_s + uint32_t(((st * 16 + slot) * PITCH + piece * 8) * 2);
+                cp_async16(dst, rr >= 0 ? vbase + rr + piece * 8 : vbase, rr >= 0 ? 16 : 0);
+            }
+            asm volatile("cp.async.commit_group;" ::: "memory");
+        };
+
+        int st = 0;
+        if (s_begin < s_end) fetch(s_begin, 0);
+        for (int64_t s0 = s_begin; s0 < s_end; s0 += 16, st ^= 1) {
+            const uint32_t mask = mask_n;
+            const bool more = s0 + 16 < s_end;
+
+            // S = Q K^T for the two slot tiles
+            float sc[2][4];
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) {
+                sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.0f;
+#pragma unroll
+                for (int j = 0; j < KS; ++j) {
+                    const uint4& w = kn[nt][j >> 1];
+                    const uint32_t b0 = (j & 1) ? w.z : w.x;
+                    const uint32_t b1 = (j & 1) ? w.w : w.y;
+                    mma_bf16(sc[nt], qh[j][0], 0u, qh[j][1], 0u, b0, b1);
+                    mma_bf16(sc[nt], ql[j][0], 0u, ql[j][1], 0u, b0, b1);
+                }
+            }
+            // the next tile's K and V are in flight during the softmax and P V
+            if (more) fetch(s0 + 16, st ^ 1);
+
+            // online softmax of head row gid over the 16 slots
+            float v[4] = {sc[0][0], sc[0][1], sc[1][0], sc[1][1]};
+            const int sl[4] = {2 * t, 2 * t + 1, 8 + 2 * t, 9 + 2 * t};
+            float mx = -INFINITY;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                if (!((mask >> sl[i]) & 1u)) v[i] = -INFINITY;
+                mx = fmaxf(mx, v[i]);
+            }
+            mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 1));
+            mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 2));
+            const float m_new = fmaxf(m_run, mx);
+            const float alpha = m_new == -INFINITY ? 1.0f : expf(m_run - m_new);
+            float ps = 0.0f;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                v[i] = v[i] == -INFINITY ? 0.0f : expf(v[i] - m_new);
+                ps += v[i];
+            }
+            ps += __shfl_xor_sync(kFull, ps, 1);
+            ps += __shfl_xor_sync(kFull, ps, 2);
+            l_run = l_run * alpha + ps;
+            m_run = m_new;
+            // O^T columns are heads 2t, 2t+1: their rescale factors live in rows 2t, 2t+1
+            const float a0 = __shfl_sync(kFull, alpha, (2 * t) * 4);
+            const float a1 = __shfl_sync(kFull, alpha, (2 * t + 1) * 4);
+#pragma unroll
+            for (int mt = 0; mt < KS; ++mt) {
+                o[mt][0] *= a0; o[mt][1] *= a1; o[mt][2] *= a0; o[mt][3] *= a1;
+            }
+            uint32_t pb0h, pb0l, pb1h, pb1l;
+            split2(v[0], v[1], pb0h, pb0l);
+            split2(v[2], v[3], pb1h, pb1l);
+
+            // O^T += V^T P^T
+            if (more) asm volatile("cp.async.wait_group 1;" ::: "memory");
+            else asm volatile("cp.async.wait_group 0;" ::: "memory");
+            __syncwarp();
+            const int lslot = (lane & 7) + ((lane >> 4) & 1) * 8;
+            const int ldim = ((lane >> 3) & 1) * 8;
+#pragma unroll
+            for (int mt = 0; mt < KS; ++mt) {
+                uint32_t r0, r1, r2, r3;
+                const uint32_t addr = wv_s + uint32_t(((st * 16 + lslot) * PITCH + mt * 16 + ldim) * 2);
+                asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                             : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                             : "r"(addr));
+                mma_bf16(o[mt], r0, r1, r2, r3, pb0h, pb1h);
+                mma_bf16(o[mt], r0, r1, r2, r3, pb0l, pb1l);
+            }
+            __syncwarp();
+        }
+
+        // heads 2t, 2t+1 of this lane's O^T columns
+        const float l0 = __shfl_sync(kFull, l_run, (2 * t) * 4);
+        const float l1 = __shfl_sync(kFull, l_run, (2 * t + 1) * 4);
+        const float m0 = __shfl_sync(kFull, m_run, (2 * t) * 4);
+        const float m1 = __shfl_sync(kFull, m_run, (2 * t + 1) * 4);
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int h = 2 * t + hh;
+            if (h >= g) continue;
+            const int64_t o_idx = (int64_t(b) * a.n_layers + l) * Hq + kh * g + h;
+            const float lh = hh ? l1 : l0;
+            if (a.splits == 1) {
+                const float inv = lh > 0.0f ? 1.0f / lh : 0.0f;
+                float* out = a.out + o_idx * D;
+#pragma unroll
+                for (int mt = 0; mt < KS; ++mt) {
+                    out[mt * 16 + gid] = o[mt][hh] * inv;
+                    out[mt * 16 + gid + 8] = o[mt][2 + hh] * inv;
+                }
+            } else {
+                float* part = a.partial + (o_idx * a.splits + split) * (D + 2);
+#pragma unroll
+                for (int mt = 0; mt < KS; ++mt) {
+                    part[mt * 16 + gid] = o[mt][hh];
+                    part[mt * 16 + gid + 8] = o[mt][2 + hh];
+                }
+                if (gid == 0) {
+                    part[D] = hh ? m1 : m0;
+                    part[D + 1] = lh;
+                }
+            }
+        }
+    }
+    if (err) atomicOr(a.status, err);
+}
+
 // Merge the chunks of one (sequence, layer, query head): thread d owns one dimension.
 __global__ void __launch_bounds__(256) decode_merge_kernel(const __grid_constant__ DecodeArgs a) {
     const int D = a.head_dim;
@@ -299,10 +573,24 @@ cudaError_t launch_gp(const DecodeArgs& a, dim3 grid, size_t smem, cudaStream_t 
 
 cudaError_t launch_decode(const DecodeArgs& a, int gp, dim3 grid, size_t smem,
                           cudaStream_t stream) {
-    // groups of 1, 2 and 4 query heads run as 4 (padded) heads x 8 slots per
-    // warp iteration, groups of 5..8 as 8 heads x 4 slots
-    const cudaError_t e = gp <= 4 ? launch_gp<4>(a, grid, smem, stream)
-                                  : launch_gp<8>(a, grid, smem, stream);
+    cudaError_t e;
+    if (a.head_dim == 64 || a.head_dim == 128) {
+        // tensor-core kernel: rotated queries + two staged V tiles per warp
+        const size_t sm = size_t(a.n_q_heads) * a.head_dim * sizeof(float) +
+                          size_t(kDecodeThreads / 32) * 2 * 16 * (a.head_dim + 8) * sizeof(uint16_t);
+        if (a.head_dim == 64) {
+            e = cudaFuncSetAttribute(decode_mma_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
+            if (e == cudaSuccess) decode_mma_kernel<64><<<grid, kDecodeThreads, sm, stream>>>(a);
+        } else {
+            e = cudaFuncSetAttribute(decode_mma_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
+            if (e == cudaSuccess) decode_mma_kernel<128><<<grid, kDecodeThreads, sm, stream>>>(a);
+        }
+        if (e == cudaSuccess) e = cudaGetLastError();
+    } else {
+        // groups of 1, 2 and 4 query heads run as 4 (padded) heads x 8 slots per
+        // warp iteration, groups of 5..8 as 8 heads x 4 slots
+        e = gp <= 4 ? launch_gp<4>(a, grid, smem, stream) : launch_gp<8>(a, grid, smem, stream);
+    }
     if (e != cudaSuccess || a.splits == 1) return e;
     const unsigned n = unsigned(int64_t(grid.z) * a.n_layers * a.n_q_heads);
     decode_merge_kernel<<<n, a.head_dim < 256 ? a.head_dim : 256, 0, stream>>>(a);
