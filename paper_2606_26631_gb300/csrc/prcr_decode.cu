@@ -392,18 +392,25 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
 
         uint4 kn[2][LV];
         uint32_t mask_n = 0u;
+        // Block id of slot s0 + (lane & 15) (paged caches), requested before
+        // the current tile's QK so that its latency hides behind the MMAs.
+        auto block_of = [&](int64_t s0) -> int32_t {
+            const int64_t s = s0 + (lane & 15);
+            if (a.cache_kind != PRCR_CACHE_PAGED || s >= s_end) return 0;
+            return a.block_table[int64_t(b) * a.bt_stride + s / a.block_size];
+        };
         // Requests tile s0 (16 slots): K rows into registers, V rows into stage st.
-        auto fetch = [&](int64_t s0, int st) {
+        auto fetch = [&](int64_t s0, int st, int32_t blk) {
             const int64_t s = s0 + (lane & 15);
             int64_t row = -1;
             if (s < s_end) {
                 if (a.cache_kind == PRCR_CACHE_CONTIGUOUS) {
                     row = int64_t(b) * a.seq_stride + s * a.slot_stride;
+                } else if (blk < 0 || blk >= a.n_blocks) {
+                    err |= PRCR_ST_NO_BLOCK;
                 } else {
                     const int64_t lb = s / a.block_size;
-                    const int32_t blk = a.block_table[int64_t(b) * a.bt_stride + lb];
-                    if (blk < 0 || blk >= a.n_blocks) err |= PRCR_ST_NO_BLOCK;
-                    else row = int64_t(blk) * a.block_stride + (s - lb * a.block_size) * a.slot_stride;
+                    row = int64_t(blk) * a.block_stride + (s - lb * a.block_size) * a.slot_stride;
                 }
             }
             mask_n = __ballot_sync(kFull, row >= 0) & 0xffffu;
@@ -428,10 +435,11 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
         };
 
         int st = 0;
-        if (s_begin < s_end) fetch(s_begin, 0);
+        if (s_begin < s_end) fetch(s_begin, 0, block_of(s_begin));
         for (int64_t s0 = s_begin; s0 < s_end; s0 += 16, st ^= 1) {
             const uint32_t mask = mask_n;
             const bool more = s0 + 16 < s_end;
+            const int32_t blk_next = more ? block_of(s0 + 16) : 0;
 
             // S = Q K^T for the two slot tiles
             float sc[2][4];
@@ -448,7 +456,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
                 }
             }
             // the next tile's K and V are in flight during the softmax and P V
-            if (more) fetch(s0 + 16, st ^ 1);
+            if (more) fetch(s0 + 16, st ^ 1, blk_next);
 
             // online softmax of head row gid over the 16 slots
             float v[4] = {sc[0][0], sc[0][1], sc[1][0], sc[1][1]};
