@@ -318,16 +318,18 @@ int do_capture(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
 // with room for its 1 KiB of static cos/sin
 constexpr size_t kDecodeSmem = 46 * 1024;
 
-// Chunking of the decode step: enough CTAs to fill the GPU a few times over,
-// chunks a multiple of 32 slots, at most kDecodeMaxChunk and small enough for
+// Chunking of the decode step. Sequence lengths differ, so CTAs differ in
+// work: aim at ~8 waves of resident CTAs (3 per SM) so that the last wave is
+// short, with chunks of at least 256 slots (to amortise each CTA's query
+// rotation), a multiple of 32, at most kDecodeMaxChunk, and small enough for
 // the chunk's row offsets to fit beside the rotated queries in shared memory.
 void decode_split(int64_t base_ctas, int64_t max_len, int sms, int64_t q_elems, int* splits,
                   int* chunk) {
-    int64_t want = (int64_t(sms) * 4 + base_ctas - 1) / base_ctas;
+    int64_t want = (int64_t(sms) * 24 + base_ctas - 1) / base_ctas;
     if (want < 1) want = 1;
     int64_t c = (max_len + want - 1) / want;
     c = (c + 31) / 32 * 32;
-    if (c < 32) c = 32;
+    if (c < 256) c = 256;
     if (c > kDecodeMaxChunk) c = kDecodeMaxChunk;
     const int64_t cap = (int64_t(kDecodeSmem) - q_elems * int64_t(sizeof(float))) / 8 / 32 * 32;
     if (c > cap) c = cap;
