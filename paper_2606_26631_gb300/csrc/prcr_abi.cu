@@ -1,7 +1,9 @@
 // extern "C" entry points of libprcr.so: argument checks, launch planning
 // and the two-kernel revisit path (plan, then rebind + inject).
+#include <array>
 #include <cmath>
 #include <cstdint>
+#include <cstring>
 #include <map>
 #include <mutex>
 #include <tuple>
@@ -10,6 +12,24 @@
 
 namespace prcr {
 namespace {
+
+// Turn rates of a (theta, head_dim) pair, computed once (long double pow is
+// slow where long double is a software type) and kept for the process.
+void copy_turn_freq(const prcr_rope_cfg* cfg, uint64_t* out) {
+    static std::mutex mu;
+    static std::map<std::pair<uint64_t, int>, std::array<uint64_t, kMaxPairs>> cache;
+    uint64_t tbits;
+    std::memcpy(&tbits, &cfg->theta, sizeof(tbits));
+    const auto key = std::make_pair(tbits, int(cfg->head_dim));
+    std::lock_guard<std::mutex> g(mu);
+    auto it = cache.find(key);
+    if (it == cache.end()) {
+        std::array<uint64_t, kMaxPairs> t{};
+        fill_turn_freq(cfg, t.data());
+        it = cache.emplace(key, t).first;
+    }
+    std::memcpy(out, it->second.data(), sizeof(uint64_t) * size_t(cfg->head_dim / 2));
+}
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 inline bool aligned4(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; }
@@ -220,8 +240,7 @@ int do_rebind(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
     a.sec_h = cfg->sections[1];
     a.sec_w = cfg->sections[2];
     const int P = cfg->head_dim / 2;
-    for (int i = 0; i < P; ++i)
-        a.inv_freq[i] = std::pow(cfg->theta, -2.0 * double(i) / double(cfg->head_dim));
+    copy_turn_freq(cfg, a.turn_freq);
 
     // One thread per (token, head, 16-byte vector of the first half row).
     const int lanes = cfg->n_kv_heads * (cfg->head_dim / 16);
@@ -295,8 +314,7 @@ int do_capture(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
     a.sec_h = cfg->sections[1];
     a.sec_w = cfg->sections[2];
     const int P = cfg->head_dim / 2;
-    for (int i = 0; i < P; ++i)
-        a.inv_freq[i] = std::pow(cfg->theta, -2.0 * double(i) / double(cfg->head_dim));
+    copy_turn_freq(cfg, a.turn_freq);
     const int lanes = cfg->n_kv_heads * (cfg->head_dim / 16);
     int T = kRebindTargetThreads / lanes;
     if (T < 1) T = 1;
@@ -517,9 +535,7 @@ int prcr_decode_attention(const prcr_rope_cfg* cfg, const prcr_cache_desc* cache
     a.head_dim = cfg->head_dim;
     a.group = n_q_heads / cfg->n_kv_heads;
     a.scale = float(1.0 / std::sqrt(double(cfg->head_dim)));
-    const int P = cfg->head_dim / 2;
-    for (int i = 0; i < P; ++i)
-        a.inv_freq[i] = std::pow(cfg->theta, -2.0 * double(i) / double(cfg->head_dim));
+    copy_turn_freq(cfg, a.turn_freq);
     int gp = 1;
     while (gp < a.group) gp <<= 1;
     const size_t smem = size_t(n_q_heads) * cfg->head_dim * sizeof(float) +
@@ -532,7 +548,7 @@ int prcr_decode_attention(const prcr_rope_cfg* cfg, const prcr_cache_desc* cache
 
 size_t prcr_select_workspace_size(int32_t n_seqs, int32_t n_q_heads, int32_t n_tokens) {
     if (n_seqs < 1 || n_q_heads < 1 || n_tokens < 1) return 0;
-    return size_t(n_seqs) * n_q_heads * n_tokens * sizeof(float);
+    return select_workspace_bytes(n_seqs, n_q_heads, n_tokens);
 }
 
 int prcr_select_topk(const prcr_rope_cfg* cfg, const prcr_store_desc* store, int32_t n_seqs,
@@ -577,14 +593,30 @@ int prcr_select_topk(const prcr_rope_cfg* cfg, const prcr_store_desc* store, int
     a.sec_h = cfg->sections[1];
     a.sec_w = cfg->sections[2];
     a.scale = float(1.0 / std::sqrt(double(cfg->head_dim)));
-    a.logits = static_cast<float*>(workspace);
+    {
+        char* w = static_cast<char*>(workspace);
+        const int64_t Bn = n_seqs, Hn = n_q_heads, M = store->n_tokens;
+        // one thread per (token, KV head) in a 256-thread CTA
+        int tile = 256 / H;
+        tile = tile < kSelectTokTile ? kSelectTokTile : (tile > 64 ? 64 : tile);
+        a.tok_tile = tile;
+        a.n_tiles = int32_t((M + tile - 1) / tile);
+        const int64_t max_tiles = (M + kSelectTokTile - 1) / kSelectTokTile;
+        a.logits = reinterpret_cast<float*>(w);
+        w += align256(size_t(4 * Bn * Hn * M));
+        a.tile_stats = reinterpret_cast<float*>(w);
+        w += align256(size_t(8 * Bn * Hn * max_tiles));
+        a.norm = reinterpret_cast<float*>(w);
+        w += align256(size_t(8 * Bn * Hn));
+        a.rel = reinterpret_cast<float*>(w);
+        w += align256(size_t(4 * Bn * M));
+        a.qrot = reinterpret_cast<float*>(w);
+    }
     a.score_out = score_out;
     a.idx_out = idx_out;
     a.rev_tok_off = rev_tok_off;
     a.seq_rev_off = seq_rev_off;
-    const int P = cfg->head_dim / 2;
-    for (int i = 0; i < P; ++i)
-        a.inv_freq[i] = std::pow(cfg->theta, -2.0 * double(i) / double(cfg->head_dim));
+    copy_turn_freq(cfg, a.turn_freq);
     return launch_select(a, n_seqs, static_cast<cudaStream_t>(stream)) == cudaSuccess ? PRCR_OK
                                                                                      : PRCR_ECUDA;
 }

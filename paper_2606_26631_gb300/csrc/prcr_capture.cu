@@ -10,8 +10,8 @@
 //
 // Work layout as in the rebind kernel: a CTA owns T tokens x G layers; its
 // prologue resolves each token's cache row (block-table lookup for paged
-// caches) and the float32 cos/sin of every (token, pair) from a float64
-// angle reduced modulo 2*pi; each thread then owns one (token, head, 16-byte
+// caches) and the float32 cos/sin of every (token, pair) from the angle
+// reduced modulo a turn in fixed point; each thread then owns one (token, head, 16-byte
 // vector) and its rotate-half partner, for all G layers.
 #include <cmath>
 
@@ -21,10 +21,6 @@
 
 namespace prcr {
 namespace {
-
-constexpr double kTwoPiHi = 6.283185307179586;
-constexpr double kTwoPiLo = 2.4492935982947064e-16;
-constexpr double kInvTwoPi = 0.15915494309189535;
 
 __device__ __forceinline__ uint4 ld_stream(const uint16_t* p) {
     uint4 r;
@@ -114,11 +110,7 @@ __global__ void __launch_bounds__(512) capture_kernel(const __grid_constant__ Ca
         float c = 1.0f, s = 0.0f;
         if (j < a.m_count) {
             const int ax = pair_axis(i, a.layout, a.sec_t, a.sec_h, a.sec_w);
-            const double ang = double(a.coords[3 * int64_t(j) + ax]) * a.inv_freq[i];
-            const double k = rint(ang * kInvTwoPi);
-            double r = fma(-k, kTwoPiHi, ang);
-            r = fma(-k, kTwoPiLo, r);
-            sincosf(float(r), &s, &c);
+            sincos_turns(double(a.coords[3 * int64_t(j) + ax]), a.turn_freq[i], &s, &c);
         }
         cos_s[q] = c;
         sin_s[q] = s;

@@ -5,8 +5,8 @@
 //
 // Work layout (memory-bound: every cached K/V row is read once per step).
 // A CTA owns (sequence, layer, slot chunk). Its prologue rotates the layer's
-// query heads at the text position (float64 angle reduced modulo 2*pi,
-// float32 sincos), pre-scales them by 1/sqrt(D) into shared memory, and
+// query heads at the text position (angle reduced modulo a turn in fixed
+// point, float32 sincos), pre-scales them by 1/sqrt(D) into shared memory, and
 // resolves the chunk's cache rows (block table for paged caches). Each warp
 // then serves one KV head and the `group` query heads that share it (GQA):
 // lane i holds D/32 consecutive dimensions, so every K or V row of the head
@@ -26,9 +26,6 @@
 namespace prcr {
 namespace {
 
-constexpr double kTwoPiHi = 6.283185307179586;
-constexpr double kTwoPiLo = 2.4492935982947064e-16;
-constexpr double kInvTwoPi = 0.15915494309189535;
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kDecodeThreads = 128;
 
@@ -77,11 +74,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3) decode_kernel(const __grid_
     __shared__ float s_cos[kMaxPairs], s_sin[kMaxPairs];
     const int64_t p = a.q_pos[b];
     for (int i = threadIdx.x; i < P; i += blockDim.x) {
-        const double ang = double(p) * a.inv_freq[i];
-        const double k = rint(ang * kInvTwoPi);
-        double r = fma(-k, kTwoPiHi, ang);
-        r = fma(-k, kTwoPiLo, r);
-        sincosf(float(r), &s_sin[i], &s_cos[i]);
+        sincos_turns(double(p), a.turn_freq[i], &s_sin[i], &s_cos[i]);
     }
     __syncthreads();
     const uint16_t* qb = a.q + (int64_t(b) * a.n_layers + l) * Hq * D;
@@ -340,11 +333,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     __shared__ float s_cos[kMaxPairs], s_sin[kMaxPairs];
     const int64_t p = a.q_pos[b];
     for (int i = threadIdx.x; i < P; i += blockDim.x) {
-        const double ang = double(p) * a.inv_freq[i];
-        const double k = rint(ang * kInvTwoPi);
-        double r = fma(-k, kTwoPiHi, ang);
-        r = fma(-k, kTwoPiLo, r);
-        sincosf(float(r), &s_sin[i], &s_cos[i]);
+        sincos_turns(double(p), a.turn_freq[i], &s_sin[i], &s_cos[i]);
     }
     __syncthreads();
     const uint16_t* qb = a.q + (int64_t(b) * a.n_layers + l) * Hq * D;

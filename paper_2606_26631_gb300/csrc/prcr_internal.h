@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cstddef>
+#include <cmath>
 #include <cstdint>
 
 #include <cuda_runtime.h>
@@ -23,6 +24,34 @@ struct PlanView {
 };
 
 inline size_t align256(size_t n) { return (n + 255) & ~size_t(255); }
+
+// Rotation rates of the pairs as fractions of a turn per unit of position,
+// in unsigned 0.64 fixed point: round(theta^(-2i/D) / (2 pi) * 2^64) (< 2^63).
+inline void fill_turn_freq(const prcr_rope_cfg* cfg, uint64_t* out) {
+    const long double two_pi = 6.283185307179586476925286766559005768L;
+    const long double two64 = 18446744073709551616.0L;
+    const int P = cfg->head_dim / 2;
+    for (int i = 0; i < P; ++i) {
+        const long double w = powl(static_cast<long double>(cfg->theta),
+                                   -2.0L * static_cast<long double>(i) / cfg->head_dim);
+        out[i] = static_cast<uint64_t>(llroundl(w / two_pi * two64));
+    }
+}
+
+#ifdef __CUDACC__
+// sin and cos of pos * inv_freq_i. The angle modulo one turn is formed
+// exactly in integers: pos in 32.32 fixed point times the 0.64 turn rate is
+// the number of turns with 96 fractional bits; the top 32 of those (the low
+// half of the 128-bit product's high word, read as signed) are the angle in
+// [-pi, pi) to 2^-32 of a turn. Needs |pos| < 2^31. Only the final sin/cos
+// runs in float32 (CUDA's sincosf).
+__device__ __forceinline__ void sincos_turns(double pos, uint64_t turn_freq, float* s, float* c) {
+    const long long pf = __double2ll_rn(pos * 4294967296.0);
+    const long long hi = __mul64hi(pf, static_cast<long long>(turn_freq));
+    const int frac = static_cast<int>(static_cast<unsigned int>(static_cast<unsigned long long>(hi)));
+    sincosf(static_cast<float>(frac) * 1.46291807926715968e-09f, s, c);  // 2 pi / 2^32
+}
+#endif
 
 inline size_t workspace_bytes(int64_t total_k) {
     if (total_k <= 0) return 0;
@@ -99,7 +128,7 @@ struct RebindArgs {
     int32_t sec_t;
     int32_t sec_h;
     int32_t sec_w;
-    double inv_freq[kMaxPairs];
+    uint64_t turn_freq[kMaxPairs];  // pair i: round(inv_freq_i / (2 pi) * 2^64)
 };
 
 struct StoreArgs {
@@ -152,7 +181,7 @@ struct CaptureArgs {
     int32_t sec_t;
     int32_t sec_h;
     int32_t sec_w;
-    double inv_freq[kMaxPairs];
+    uint64_t turn_freq[kMaxPairs];  // pair i: round(inv_freq_i / (2 pi) * 2^64)
 };
 
 struct DecodeArgs {
@@ -182,12 +211,20 @@ struct DecodeArgs {
     int32_t splits;
     int32_t chunk;
     float scale;
-    double inv_freq[kMaxPairs];
+    uint64_t turn_freq[kMaxPairs];  // pair i: round(inv_freq_i / (2 pi) * 2^64)
 };
 
 constexpr int kDecodeMaxChunk = 4096;
 
 constexpr int kSelectMaxQHeads = 128;
+constexpr int kSelectTokTile = 16;   // smallest tile of the logits kernel (sizes the workspace)
+
+inline size_t select_workspace_bytes(int64_t B, int64_t Hq, int64_t M) {
+    const int64_t tiles = (M + kSelectTokTile - 1) / kSelectTokTile;
+    return align256(size_t(4 * B * Hq * M)) + align256(size_t(8 * B * Hq * tiles)) +
+           align256(size_t(8 * B * Hq)) + align256(size_t(4 * B * M)) +
+           align256(size_t(4 * B * Hq) * kMaxPairs * 2);
+}
 
 struct SelectArgs {
     const uint16_t* q;          // [B][n_q_heads][D] raw trigger queries
@@ -210,11 +247,17 @@ struct SelectArgs {
     int32_t sec_w;
     float scale;
     float* logits;              // workspace [B][n_q_heads][n_tokens]
+    float* tile_stats;          // workspace [B][n_q_heads][n_tiles][2] (max, sum of exp)
+    float* norm;                // workspace [B][n_q_heads][2] (max, 1 / (sum * n_q_heads))
+    float* rel;                 // workspace [B][n_tokens] relevance
+    float* qrot;                // workspace [B][n_q_heads][D] rotated, scaled queries
+    int32_t n_tiles;            // token tiles of the logits kernel
+    int32_t tok_tile;           // tokens per tile
     float* score_out;           // optional [B][n_tokens]
     int32_t* idx_out;           // [B][k]
     int32_t* rev_tok_off;       // [B + 1]
     int32_t* seq_rev_off;       // [B + 1]
-    double inv_freq[kMaxPairs];
+    uint64_t turn_freq[kMaxPairs];  // pair i: round(inv_freq_i / (2 pi) * 2^64)
 };
 
 cudaError_t launch_select(const SelectArgs& a, int n_seqs, cudaStream_t stream);

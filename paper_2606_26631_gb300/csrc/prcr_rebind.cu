@@ -8,10 +8,10 @@
 //
 // Work layout. A CTA owns T tokens x G layers. Its threads first build the
 // float32 cos/sin of every (token, rotation pair) of the tile in shared
-// memory, once for all G layers and all heads: the angle is formed in float64
-// (position x inverse frequency), reduced modulo 2*pi in float64 (Cody-Waite
-// with a two-term 2*pi), and only then handed to float32 sincosf, so a
-// position near 3e4 keeps a ~1e-7 rad angle error instead of ~2e-3.
+// memory, once for all G layers and all heads: the angle modulo a turn is
+// formed exactly in fixed-point integers (sincos_turns) and only then handed
+// to float32 sincosf, so a position near 3e4 keeps a ~2e-7 rad angle error
+// instead of the ~2e-3 of a float32 product.
 // Then each thread owns one (token, head, 16-byte vector v) slot of the row:
 // it loads the 8 bf16 of the first half at v and the 8 bf16 of the second
 // half at v + D/2 (the rotate-half partners), for K and V, and walks the G
@@ -28,11 +28,6 @@
 
 namespace prcr {
 namespace {
-
-// 2*pi split into a float64 head and the float64 nearest to the remainder.
-constexpr double kTwoPiHi = 6.283185307179586;
-constexpr double kTwoPiLo = 2.4492935982947064e-16;
-constexpr double kInvTwoPi = 0.15915494309189535;
 
 __device__ __forceinline__ uint4 ld_stream(const uint16_t* p) {
     uint4 r;
@@ -106,11 +101,7 @@ __global__ void __launch_bounds__(512) rebind_kernel(const __grid_constant__ Reb
         float c = 1.0f, s = 0.0f;
         if (tok < a.total_k) {
             const int ax = pair_axis(i, a.layout, a.sec_t, a.sec_h, a.sec_w);
-            const double ang = a.plan_pos[3 * tok + ax] * a.inv_freq[i];
-            const double k = rint(ang * kInvTwoPi);
-            double r = fma(-k, kTwoPiHi, ang);
-            r = fma(-k, kTwoPiLo, r);
-            sincosf(float(r), &s, &c);
+            sincos_turns(a.plan_pos[3 * tok + ax], a.turn_freq[i], &s, &c);
         }
         cos_s[q] = c;
         sin_s[q] = s;

@@ -247,4 +247,4 @@ def test_new_entry_points_validate_on_host():
     assert sel(Hq=3) == B.EINVAL
     assert sel(ws=None) == B.EWORKSPACE
     assert sel(wsb=16) == B.EWORKSPACE
-    assert prcr.select_workspace_size(2, 4, 64) == 2 * 4 * 64 * 4
+    assert prcr.select_workspace_size(2, 4, 64) >= 2 * 4 * 64 * 4 + 2 * 64 * 4
