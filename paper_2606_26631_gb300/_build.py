@@ -20,7 +20,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libprcr.so")
 
 SOURCES = ["prcr_abi.cu", "prcr_plan.cu", "prcr_rebind.cu", "prcr_store.cu", "prcr_static.cu",
-           "prcr_capture.cu", "prcr_decode.cu", "prcr_select.cu"]
+           "prcr_capture.cu", "prcr_decode.cu", "prcr_select.cu", "prcr_fused.cu"]
 GENCODE = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = GENCODE + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-fvisibility=hidden",
                         "-I", INCLUDE, "-I", CSRC]
@@ -35,7 +35,8 @@ def nvcc() -> str:
 
 def _inputs():
     deps = [os.path.join(CSRC, s) for s in SOURCES]
-    deps += [os.path.join(CSRC, "prcr_internal.h"), os.path.join(INCLUDE, "prcr.h"), __file__]
+    deps += [os.path.join(CSRC, "prcr_internal.h"), os.path.join(CSRC, "prcr_device.cuh"),
+             os.path.join(INCLUDE, "prcr.h"), __file__]
     return deps
 
 

@@ -216,11 +216,11 @@ int layers_per_cta(int64_t tiles, int n_layers, int64_t slots) {
     return best;
 }
 
-int do_rebind(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
-              const prcr_cache_desc* cache, const prcr_revisit_batch* b, const prcr_outputs* o,
-              void* ws, cudaStream_t stream) {
-    if (b->total_k == 0) return PRCR_OK;
-    RebindArgs a = {};
+// Arguments and launch shape of the row-moving kernel (rebind or fused).
+int rebind_setup(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+                 const prcr_cache_desc* cache, const prcr_revisit_batch* b, const prcr_outputs* o,
+                 void* ws, RebindArgs& a, dim3& grid, int& block, size_t& smem) {
+    a = RebindArgs{};
     a.store_k = static_cast<const uint16_t*>(store->k);
     a.store_v = static_cast<const uint16_t*>(store->v);
     a.cache_k = static_cast<uint16_t*>(cache->k);
@@ -246,8 +246,8 @@ int do_rebind(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
     const int lanes = cfg->n_kv_heads * (cfg->head_dim / 16);
     int T = kRebindTargetThreads / lanes;
     if (T < 1) T = 1;
-    const int block = T * lanes;
-    const size_t smem = size_t(2) * T * P * sizeof(float);
+    block = T * lanes;
+    smem = size_t(2) * T * P * sizeof(float);
     a.lanes = lanes;
     a.tok_per_cta = T;
 
@@ -259,7 +259,20 @@ int do_rebind(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
     const int64_t groups = (cfg->n_layers + G - 1) / G;
     a.layers_per_cta = G;
     if (tiles > INT32_MAX) return PRCR_EINVAL;
-    const dim3 grid(unsigned(tiles), unsigned(groups), 1);
+    grid = dim3(unsigned(tiles), unsigned(groups), 1);
+    return PRCR_OK;
+}
+
+int do_rebind(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+              const prcr_cache_desc* cache, const prcr_revisit_batch* b, const prcr_outputs* o,
+              void* ws, cudaStream_t stream) {
+    if (b->total_k == 0) return PRCR_OK;
+    RebindArgs a;
+    dim3 grid;
+    int block = 0;
+    size_t smem = 0;
+    const int rc = rebind_setup(cfg, store, cache, b, o, ws, a, grid, block, smem);
+    if (rc) return rc;
     return launch_rebind(a, grid, block, smem, stream) == cudaSuccess ? PRCR_OK : PRCR_ECUDA;
 }
 
@@ -399,6 +412,18 @@ int prcr_rebind_inject(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
     int rc = check_call(cfg, store, cache, batch, out, mode, L, flags, workspace, workspace_bytes);
     if (rc || batch->n_seqs == 0) return rc;
     const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (batch->total_k > 0 && batch->total_k <= kFusedMaxTokens &&
+        batch->n_revisits <= kFusedMaxRevisits && batch->n_seqs <= kFusedMaxSeqs) {
+        // a few small revisits: one kernel plans and moves them (no plan round trip)
+        FusedArgs fa;
+        fa.plan = make_plan_args(store, cache, batch, out, mode, L, flags, workspace);
+        dim3 grid;
+        int block = 0;
+        size_t smem = 0;
+        rc = rebind_setup(cfg, store, cache, batch, out, workspace, fa.rebind, grid, block, smem);
+        if (rc) return rc;
+        return launch_fused(fa, grid, block, smem, s) == cudaSuccess ? PRCR_OK : PRCR_ECUDA;
+    }
     rc = do_plan(store, cache, batch, out, mode, L, flags, workspace, s);
     if (rc) return rc;
     return do_rebind(cfg, store, cache, batch, out, workspace, s);

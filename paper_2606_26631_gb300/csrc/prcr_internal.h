@@ -267,6 +267,18 @@ cudaError_t launch_decode(const DecodeArgs& a, int gp, dim3 grid, size_t smem,
 cudaError_t launch_capture(const CaptureArgs& a, dim3 grid, int block, size_t smem,
                            cudaStream_t stream);
 cudaError_t capture_blocks_per_sm(int block, size_t smem, int* out);
+// Small batches: the whole revisit in one kernel (plan part + rebind part;
+// the rebind part's plan pointers are unused).
+struct FusedArgs {
+    PlanArgs plan;
+    RebindArgs rebind;
+};
+constexpr int64_t kFusedMaxTokens = 2048;
+constexpr int kFusedMaxRevisits = 64;
+constexpr int kFusedMaxSeqs = 64;
+
+cudaError_t launch_fused(const FusedArgs& a, dim3 grid, int block, size_t smem,
+                         cudaStream_t stream);
 cudaError_t launch_plan(const PlanArgs& a, cudaStream_t stream);
 cudaError_t launch_rebind(const RebindArgs& a, dim3 grid, int block, size_t smem,
                           cudaStream_t stream);

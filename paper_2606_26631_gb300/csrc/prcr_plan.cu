@@ -17,90 +17,10 @@
 #include <climits>
 #include <cmath>
 
-#include "prcr_internal.h"
+#include "prcr_device.cuh"
 
 namespace prcr {
 namespace {
-
-constexpr double kExactLimit = 4503599627370496.0;  // 2^52
-constexpr int kTokPerThread = 4;   // tokens of a revisit each thread keeps in registers
-constexpr int kPosTable = 1024;    // exact PCR positions tabulated per axis when span < this
-
-// True when every integer formed for p_hat = ((p - L) * Q + tail) / Q with
-// 0 <= tail <= (L+1) * Q stays below 2^52 in magnitude, so that the integer
-// products cannot overflow and the float64 division sees exact operands.
-__device__ __forceinline__ bool exact_ok(int64_t p_minus_l, int32_t L, double Q) {
-    return (fabs(double(p_minus_l)) + double(L) + 1.0) * Q < kExactLimit;
-}
-
-__device__ __forceinline__ double pcr_position(int64_t p, int32_t L, int64_t K, int32_t c,
-                                               int32_t lo, int32_t hi, bool center,
-                                               uint32_t& err) {
-    const int64_t span = int64_t(hi) - int64_t(lo);
-    const int64_t pl = p - L;
-    if (span > 0) {
-        if (exact_ok(pl, L, double(K + 1) * double(span))) {
-            const int64_t Q = (K + 1) * span;
-            const int64_t tail = int64_t(L + 1) * (span + (K - 1) * (int64_t(c) - lo));
-            return double(pl * Q + tail) / double(Q);
-        }
-        err |= PRCR_ST_POS_RANGE;
-        const double u = double(int64_t(c) - lo) / double(span);
-        return double(pl) + double(L + 1) * (1.0 + double(K - 1) * u) / double(K + 1);
-    }
-    // degenerate axis: u = 0, or u = 1/2 with the centre reading
-    const int64_t Q = center ? 2 * (K + 1) : K + 1;
-    const int64_t tail = center ? int64_t(L + 1) * (K + 1) : int64_t(L + 1);
-    if (exact_ok(pl, L, double(Q))) return double(pl * Q + tail) / double(Q);
-    err |= PRCR_ST_POS_RANGE;
-    return double(pl) + double(tail) / double(Q);
-}
-
-// p + num / (K + 1), exact while representable (UIR).
-__device__ __forceinline__ double uir_position(int64_t p, int64_t num, int64_t K, uint32_t& err) {
-    if (exact_ok(p, 0, double(K + 1))) return double(p * (K + 1) + num) / double(K + 1);
-    err |= PRCR_ST_POS_RANGE;
-    return double(p) + double(num) / double(K + 1);
-}
-
-__device__ __forceinline__ void block_minmax(int (&mn)[3], int (&mx)[3], int* s_part) {
-    const int lane = threadIdx.x & 31;
-    const int warp = threadIdx.x >> 5;
-    const int nwarps = (blockDim.x + 31) >> 5;
-#pragma unroll
-    for (int a = 0; a < 3; ++a) {
-        mn[a] = __reduce_min_sync(0xffffffffu, mn[a]);
-        mx[a] = __reduce_max_sync(0xffffffffu, mx[a]);
-    }
-    if (lane == 0) {
-#pragma unroll
-        for (int a = 0; a < 3; ++a) {
-            s_part[warp * 6 + a] = mn[a];
-            s_part[warp * 6 + 3 + a] = mx[a];
-        }
-    }
-    __syncthreads();
-    if (warp == 0) {
-#pragma unroll
-        for (int a = 0; a < 3; ++a) {
-            int vmn = lane < nwarps ? s_part[lane * 6 + a] : INT_MAX;
-            int vmx = lane < nwarps ? s_part[lane * 6 + 3 + a] : INT_MIN;
-            vmn = __reduce_min_sync(0xffffffffu, vmn);
-            vmx = __reduce_max_sync(0xffffffffu, vmx);
-            if (lane == 0) {
-                s_part[32 * 6 + a] = vmn;
-                s_part[32 * 6 + 3 + a] = vmx;
-            }
-        }
-    }
-    __syncthreads();
-#pragma unroll
-    for (int a = 0; a < 3; ++a) {
-        mn[a] = s_part[32 * 6 + a];
-        mx[a] = s_part[32 * 6 + 3 + a];
-    }
-    __syncthreads();  // s_part is reused by the next revisit
-}
 
 // Per-token outputs of one selected token (plan entry, optional position and
 // slot outputs). pos[] must already hold the reassigned position.
@@ -121,115 +41,22 @@ __device__ __forceinline__ void emit(const PlanArgs& a, int j, int64_t slot, int
     if (a.slot_out) a.slot_out[j] = int32_t(slot > INT_MAX ? INT_MAX : slot);
 }
 
-struct RevisitCtx {
-    int b, beg, end, t0;
-    int64_t K, p, clen, capacity;
-    int lo[3], hi[3];
-    bool tab[3];
-    bool center;
-};
-
-// Physical destination row offset of `slot` (layer term excluded), or -1.
-__device__ __forceinline__ int64_t dest_row(const PlanArgs& a, const RevisitCtx& r, int64_t slot,
-                                            int32_t blk, uint32_t& err) {
-    if (r.clen < 0 || slot >= r.capacity) {
-        err |= PRCR_ST_CAPACITY;
-        return -1;
-    }
-    if (a.cache_kind == PRCR_CACHE_CONTIGUOUS)
-        return int64_t(r.b) * a.cache_seq_stride + slot * a.slot_stride;
-    if (blk < 0 || blk >= a.n_blocks) {
-        err |= PRCR_ST_NO_BLOCK;
-        return -1;
-    }
-    const int64_t lb = slot / a.block_size;
-    return int64_t(blk) * a.block_stride + (slot - lb * a.block_size) * a.slot_stride;
-}
-
-// Block id holding `slot` (paged caches), read early so the load overlaps others.
-__device__ __forceinline__ int32_t block_of(const PlanArgs& a, const RevisitCtx& r, int64_t slot) {
-    if (a.cache_kind != PRCR_CACHE_PAGED || r.clen < 0 || slot >= r.capacity) return -1;
-    return a.block_table[int64_t(r.b) * a.bt_stride + slot / a.block_size];
-}
-
 __device__ __forceinline__ void place_token(const PlanArgs& a, const RevisitCtx& r,
                                             const double (*tab)[kPosTable], int j, int m,
                                             const int (&c)[3], int32_t blk, uint32_t& err) {
-    const int64_t slot = r.clen + (j - r.t0);
     double pos[3];
-    int64_t src = 0, dst = -1;
-    if (m < 0 || m >= a.n_tokens) {
-        err |= PRCR_ST_IDX_RANGE;
-        pos[0] = pos[1] = pos[2] = __longlong_as_double(0x7ff8000000000000LL);
-    } else {
-        switch (a.mode) {
-            case PRCR_MODE_PCR:
-#pragma unroll
-                for (int ax = 0; ax < 3; ++ax)
-                    pos[ax] = r.tab[ax] ? tab[ax][c[ax] - r.lo[ax]]
-                                        : pcr_position(r.p, a.L, r.K, c[ax], r.lo[ax], r.hi[ax],
-                                                       r.center, err);
-                break;
-            case PRCR_MODE_ORIGINAL:
-#pragma unroll
-                for (int ax = 0; ax < 3; ++ax) pos[ax] = double(c[ax]);
-                break;
-            case PRCR_MODE_UIR: {
-                // p + (j' + 1) / (K + 1), j' the token's rank in its revisit
-                const double v = uir_position(r.p, int64_t(j - r.beg + 1), r.K, err);
-                pos[0] = pos[1] = pos[2] = v;
-                break;
-            }
-            default: {  // PRCR_MODE_LPA: p + rank in sequence + 1
-                const double v = double(r.p + (j - r.t0) + 1);
-                pos[0] = pos[1] = pos[2] = v;
-                break;
-            }
-        }
-        src = int64_t(r.b) * a.store_seq_stride + int64_t(m) * a.store_token_stride;
-        dst = dest_row(a, r, slot, blk, err);
-    }
+    int64_t src, dst, slot;
+    token_plan(a, r, tab, j, m, c, blk, err, pos, src, dst, slot);
     emit(a, j, slot, src, dst, pos);
-}
-
-__device__ __forceinline__ void load_coords(const int32_t* crd, int m, int n_tokens, int (&c)[3]) {
-    if (m >= 0 && m < n_tokens) {
-        const int32_t* q = crd + 3 * int64_t(m);
-        c[0] = q[0];
-        c[1] = q[1];
-        c[2] = q[2];
-    } else {
-        c[0] = c[1] = c[2] = 0;
-    }
 }
 
 __device__ void plan_revisit(const PlanArgs& a, int r, int* s_part, double (*s_tab)[kPosTable],
                              uint32_t& err) {
     RevisitCtx x;
-    x.beg = a.rev_tok_off[r];
-    x.end = a.rev_tok_off[r + 1];
-    // sequence owning revisit r: last b with seq_rev_off[b] <= r
-    int lo = 0, hi = a.n_seqs;
-    while (hi - lo > 1) {
-        const int mid = (lo + hi) >> 1;
-        if (a.seq_rev_off[mid] <= r) lo = mid; else hi = mid;
-    }
-    x.b = lo;
-    const int r_first = a.seq_rev_off[x.b];
-    bool ok = x.beg >= 0 && x.beg <= x.end && int64_t(x.end) <= a.total_k &&
-              r_first <= r && r < a.seq_rev_off[x.b + 1] && r_first >= 0;
-    x.t0 = ok ? a.rev_tok_off[r_first] : 0;
-    ok = ok && x.t0 >= 0 && x.t0 <= x.beg;
-    if (!ok) {  // uniform over the CTA
+    if (!revisit_ctx(a, r, x)) {  // uniform over the CTA
         err |= PRCR_ST_CSR;
         return;
     }
-    x.K = x.end - x.beg;
-    x.p = a.p_txt[x.b];
-    x.clen = a.cache_len_in[x.b];
-    x.center = (a.flags & PRCR_FLAG_DEGENERATE_CENTER) != 0;
-    x.capacity = a.cache_kind == PRCR_CACHE_CONTIGUOUS ? int64_t(a.max_slots)
-                                                       : int64_t(a.bt_stride) * a.block_size;
     const int32_t* crd = a.coords + int64_t(x.b) * a.coord_seq_stride;
 
     // Pass 1: the first kTokPerThread * blockDim tokens stay in registers

@@ -24,63 +24,10 @@
 
 #include <cuda_bf16.h>
 
-#include "prcr_internal.h"
+#include "prcr_device.cuh"
 
 namespace prcr {
 namespace {
-
-__device__ __forceinline__ uint4 ld_stream(const uint16_t* p) {
-    uint4 r;
-    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
-                 : "l"(p));
-    return r;
-}
-
-__device__ __forceinline__ void st_row(uint16_t* p, const uint4& v) {
-    asm volatile("st.global.v4.u32 [%0], {%1, %2, %3, %4};"
-                 :
-                 : "l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
-                 : "memory");
-}
-
-__device__ __forceinline__ float lo_f32(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float hi_f32(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
-
-__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
-    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<const uint32_t*>(&v);
-}
-
-// Rotate four bf16 pairs held as (first-half word x, second-half word y):
-// x' = x cos - y sin, y' = y cos + x sin, float32, bf16 round-to-nearest-even.
-__device__ __forceinline__ void rotate_word(uint32_t x, uint32_t y, float c0, float s0, float c1,
-                                           float s1, uint32_t& xo, uint32_t& yo) {
-    const float x0 = lo_f32(x), x1 = hi_f32(x);
-    const float y0 = lo_f32(y), y1 = hi_f32(y);
-    const float a0 = fmaf(x0, c0, -y0 * s0);
-    const float a1 = fmaf(x1, c1, -y1 * s1);
-    const float b0 = fmaf(y0, c0, x0 * s0);
-    const float b1 = fmaf(y1, c1, x1 * s1);
-    xo = pack_bf16x2(a0, a1);
-    yo = pack_bf16x2(b0, b1);
-}
-
-__device__ __forceinline__ void rotate_vec(const uint4& x, const uint4& y, const float (&c)[8],
-                                           const float (&s)[8], uint4& xo, uint4& yo) {
-    rotate_word(x.x, y.x, c[0], s[0], c[1], s[1], xo.x, yo.x);
-    rotate_word(x.y, y.y, c[2], s[2], c[3], s[3], xo.y, yo.y);
-    rotate_word(x.z, y.z, c[4], s[4], c[5], s[5], xo.z, yo.z);
-    rotate_word(x.w, y.w, c[6], s[6], c[7], s[7], xo.w, yo.w);
-}
-
-__device__ __forceinline__ int pair_axis(int i, int layout, int st, int sh, int sw) {
-    if (layout == PRCR_LAYOUT_SECTIONED) return i < st ? 0 : (i < st + sh ? 1 : 2);
-    const int r = i % 3;
-    if (r == 1 && i < 3 * sh) return 1;
-    if (r == 2 && i < 3 * sw) return 2;
-    return 0;
-}
 
 __global__ void __launch_bounds__(512) rebind_kernel(const __grid_constant__ RebindArgs a) {
     extern __shared__ float smem[];
@@ -143,35 +90,7 @@ __global__ void __launch_bounds__(512) rebind_kernel(const __grid_constant__ Reb
     uint16_t* ck = a.cache_k + dst + int64_t(l0) * cls + off;
     uint16_t* cv = a.cache_v + dst + int64_t(l0) * cls + off;
 
-    int l = l0;
-    for (; l + 2 <= l1; l += 2) {
-        const uint4 k0a = ld_stream(sk), k1a = ld_stream(sk + half);
-        const uint4 v0a = ld_stream(sv), v1a = ld_stream(sv + half);
-        const uint4 k0b = ld_stream(sk + sls), k1b = ld_stream(sk + sls + half);
-        const uint4 v0b = ld_stream(sv + sls), v1b = ld_stream(sv + sls + half);
-        uint4 o0, o1;
-        rotate_vec(k0a, k1a, c, s, o0, o1);
-        st_row(ck, o0);
-        st_row(ck + half, o1);
-        st_row(cv, v0a);
-        st_row(cv + half, v1a);
-        rotate_vec(k0b, k1b, c, s, o0, o1);
-        st_row(ck + cls, o0);
-        st_row(ck + cls + half, o1);
-        st_row(cv + cls, v0b);
-        st_row(cv + cls + half, v1b);
-        sk += 2 * sls; sv += 2 * sls; ck += 2 * cls; cv += 2 * cls;
-    }
-    if (l < l1) {
-        const uint4 k0 = ld_stream(sk), k1 = ld_stream(sk + half);
-        const uint4 v0 = ld_stream(sv), v1 = ld_stream(sv + half);
-        uint4 o0, o1;
-        rotate_vec(k0, k1, c, s, o0, o1);
-        st_row(ck, o0);
-        st_row(ck + half, o1);
-        st_row(cv, v0);
-        st_row(cv + half, v1);
-    }
+    stream_layers(sk, sv, ck, cv, sls, cls, half, l1 - l0, c, s);
 }
 
 }  // namespace

@@ -307,3 +307,62 @@ def test_graph_replay_matches(name):
     torch.cuda.synchronize()
     assert rv.status_value() == 0
     pu.full_check(batch, rv)
+
+
+SMALL = ["tiny", "qwen2vl-2b", "paper-8b-k32", "paper-8b-k128", "edge-d16", "edge-odd"]
+
+
+def _small_wl(name):
+    return {w.name: w for w in EDGE}.get(name) or get(name)
+
+
+@pytest.mark.parametrize("mode", [O.MODE_PCR, O.MODE_ORIGINAL, O.MODE_UIR, O.MODE_LPA])
+@pytest.mark.parametrize("name", SMALL)
+def test_fused_path_matches_two_kernel_path(name, mode):
+    """Small batches take the one-kernel path in prcr_rebind_inject; its
+    results equal the plan + rebind kernels' bit for bit (prcr_plan followed
+    by prcr_rebind_apply always runs the two kernels)."""
+    import parity_util as pu
+    batch = make_batch(_small_wl(name), device=DEV, seed=21)
+    assert batch.total_k <= 2048 and batch.n_revisits <= 64
+    pristine_k = batch.cache_k.clone(); pristine_v = batch.cache_v.clone()
+    fused = pu.make_revisit(batch, mode=mode)
+    fused.run()
+    torch.cuda.synchronize()
+    fk, fv = batch.cache_k.clone(), batch.cache_v.clone()
+    batch.cache_k.copy_(pristine_k); batch.cache_v.copy_(pristine_v)
+    two = pu.make_revisit(batch, mode=mode)
+    two.run_plan(); two.run_apply()
+    torch.cuda.synchronize()
+    assert fused.status_value() == two.status_value() == 0
+    assert torch.equal(fk.view(torch.int16), batch.cache_k.view(torch.int16))
+    assert torch.equal(fv.view(torch.int16), batch.cache_v.view(torch.int16))
+    assert torch.equal(fused.pos.view(torch.int64), two.pos.view(torch.int64))
+    assert torch.equal(fused.slot, two.slot)
+    assert torch.equal(fused.cache_len_out, two.cache_len_out)
+    assert torch.equal(fused.next_pos, two.next_pos)
+
+
+def test_malformed_offsets_small_batch_write_nothing():
+    import parity_util as pu
+    batch = make_batch(_small_wl("edge-odd"), device=DEV, seed=5)
+    r = int(batch.rev_tok_off.numel()) - 1
+    assert r >= 3 and batch.total_k <= 2048
+    batch.rev_tok_off[2] = batch.rev_tok_off[3] + 1  # not monotone
+    rv = _run(batch)
+    assert rv.status_value() & pu.prcr.ST_CSR
+    for c in (batch.cache_k, batch.cache_v):
+        assert bool((c.view(torch.int16) == -1).all().item())
+
+
+def test_bad_index_small_batch():
+    """Fused path: an out-of-range index is reported and its rows skipped;
+    the other revisits' rows are right."""
+    import parity_util as pu
+    batch = make_batch(get("paper-8b-k128"), device=DEV)
+    pl = pu.oracle_plan(batch)
+    batch.idx[7] = batch.wl.n_tokens + 1
+    rv = _run(batch)
+    assert rv.status_value() & pu.prcr.ST_IDX_RANGE
+    written = np.array([j for j in range(batch.total_k) if j != 7])
+    pu.check_untouched(batch, pl, written=written)

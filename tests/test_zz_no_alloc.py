@@ -26,12 +26,14 @@ pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
 
 
-def _compare_with_workspace_call(name):
+def _compare_with_workspace_call(wl):
     import paper_2606_26631_gb300 as prcr
     import parity_util as pu
-    from workloads import get, make_batch
+    from workloads import make_batch
 
-    batch = make_batch(get(name), device=DEV)
+    batch = make_batch(wl, device=DEV)
+    # batches this large use the plan kernel and its per-token scratch
+    assert batch.total_k > 2048
     pristine_k = batch.cache_k.clone()
     pristine_v = batch.cache_v.clone()
 
@@ -65,8 +67,10 @@ def _compare_with_workspace_call(name):
 
 
 def test_static_scratch_two_calls_in_a_row():
-    first = _compare_with_workspace_call("qwen25vl-7b")   # paged, 4093 tokens
-    second = _compare_with_workspace_call("qwen2vl-2b")   # contiguous, 259 tokens
+    from workloads import get
+    first = _compare_with_workspace_call(get("qwen25vl-7b"))  # paged, 4093 tokens
+    second = _compare_with_workspace_call(                    # contiguous, 12 x 259 tokens
+        dataclasses.replace(get("qwen2vl-2b"), n_seqs=12))
     assert first.batch.total_k != second.batch.total_k
 
 
