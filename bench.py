@@ -40,14 +40,19 @@ SPEC_HBM_GBS = 8000.0
 # workload, from an ncu capture; valid only for the kernel source it was
 # measured on (its sha256 prefix), reported as null otherwise.
 TRAFFIC = {
-    # profiles/rebind_kernel_stress_dram.md: 19,304,776,704 B read + 19,268,871,168 B written
-    ("stress", "6b40ef09c2644b48"): 38573647872,
+    # profiles/rebind_kernel_stress_dram.md: 19,312,595,968 B read + 19,268,798,464 B written
+    ("stress", "b0312a34cc78aa78"): 38581394432,
 }
 
 
-def _sha(path):
-    with open(path, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+def _sha(*paths):
+    """Hash of the rebind kernel's sources: a stored traffic figure is used
+    only while they are the ones it was measured on."""
+    h = hashlib.sha256()
+    for path in paths:
+        with open(path, "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 def parse():
@@ -70,7 +75,59 @@ def parse():
     ap.add_argument("--graph", action="store_true",
                     help="replay the step from a CUDA graph (for small, launch-bound workloads)")
     ap.add_argument("--graph-inner", type=int, default=20, help="steps captured per graph")
+    ap.add_argument("--flush", choices=["auto", "on", "off"], default="auto",
+                    help="write a buffer of twice the L2 size before each timed step "
+                         "(auto: when a step moves less than 4x the L2 size)")
     return ap.parse_args()
+
+
+def kernel_launches(fn):
+    """Names, in launch order, of this library's CUDA kernels one call of fn
+    launches, as the profiler (CUPTI) records them; empty if it records none.
+    (Kernel records come only with CPU activity profiled too.)"""
+    import re
+    import torch
+    from torch.profiler import ProfilerActivity, profile
+    torch.cuda.synchronize()
+    for _ in range(3):  # the first session of a process records no kernels
+        with profile(activities=[ProfilerActivity.CPU, ProfilerActivity.CUDA]) as prof:
+            fn()
+            torch.cuda.synchronize()
+        evs = sorted((e for e in prof.events() if e.device_type.name == "CUDA"),
+                     key=lambda e: e.time_range.start)
+        out = []
+        for e in evs:
+            m = re.search(r"\bprcr::.*?\b(\w+_kernel)\b", e.name)
+            if m:
+                out.append(m.group(1))
+        if out:
+            return out
+    return []
+
+
+class L2Flush:
+    """Evicts L2 between timed steps by writing a buffer of twice its size."""
+
+    def __init__(self, dev, mode, nbytes):
+        import torch
+        self.l2 = int(getattr(torch.cuda.get_device_properties(dev), "L2_cache_size", 0)) or (129 << 20)
+        self.enabled = mode == "on" or (mode == "auto" and nbytes < 4 * self.l2)
+        self.buf = torch.empty(2 * self.l2, dtype=torch.uint8, device=dev) if self.enabled else None
+        self.i = 0
+
+    def __call__(self):
+        if self.enabled:
+            self.i += 1
+            self.buf.fill_(self.i & 0xFF)
+
+    def describe(self, nbytes):
+        if self.enabled:
+            return ("L2 flushed before each step (%d MB written); each step moves %.2f GB"
+                    % (2 * self.l2 >> 20, nbytes / 1e9))
+        if nbytes >= 4 * self.l2:
+            return "inputs larger than L2 (no flush): each step moves %.2f GB" % (nbytes / 1e9)
+        return ("warm: no flush between steps, %.2f GB per step against a %d MB L2"
+                % (nbytes / 1e9, self.l2 >> 20))
 
 
 def dist_env():
@@ -300,10 +357,19 @@ def run_gpu(args):
                      positions_slots_bit_exact=True, v_bit_exact=True)
 
     stream = torch.cuda.current_stream()
+    # what one public call launches: one fused kernel for small batches, or
+    # the plan kernel then the rebind + inject kernel (timed one by one)
+    launched = kernel_launches(rv.run)
+    split = launched == ["plan_kernel", "rebind_kernel"] or not launched
+    per_step = len(launched) if launched else 2
     for _ in range(args.warmup):
-        rv.run_plan()
-        rv.run_apply()
+        if split:
+            rv.run_plan()
+            rv.run_apply()
+        else:
+            rv.run()
     torch.cuda.synchronize()
+    flush = L2Flush(dev, "off" if args.graph else args.flush, nbytes)
 
     K = args.steps
     if args.graph:
@@ -344,16 +410,25 @@ def run_gpu(args):
         torch.cuda.synchronize()
         with Clocks(local) as clk:
             for e0, e1, e2 in ev:
+                flush()
                 e0.record(stream)
-                rv.run_plan()
-                e1.record(stream)
-                rv.run_apply()
+                if split:
+                    rv.run_plan()
+                    e1.record(stream)
+                    rv.run_apply()
+                else:
+                    rv.run()
+                    e1.record(stream)
                 e2.record(stream)
             torch.cuda.synchronize()
         barrier(world)
         step_ms = [e0.elapsed_time(e2) for e0, _, e2 in ev]
-        apply_ms = [e1.elapsed_time(e2) for _, e1, e2 in ev]
-        plan_ms = [e0.elapsed_time(e1) for e0, e1, _ in ev]
+        if split:
+            apply_ms = [e1.elapsed_time(e2) for _, e1, e2 in ev]
+            plan_ms = [e0.elapsed_time(e1) for e0, e1, _ in ev]
+        else:
+            apply_ms = step_ms
+            plan_ms = None
     total_s = sum(step_ms) / 1e3
     total_s = max_over_ranks(total_s, world, dev)
     value = nbytes * world * K / total_s / 1e9
@@ -374,13 +449,14 @@ def run_gpu(args):
     peak, peak_kind = measured_peaks()
     if apply_ms is not None:
         apply_avg_s = statistics.mean(apply_ms) / 1e3
-        kernel = "rebind_kernel"
+        kernel = "rebind_kernel" if split else "fused_kernel"
     else:  # graph replay: only whole steps are timed
         apply_avg_s = statistics.mean(step_ms) / 1e3
-        kernel = "plan_kernel + rebind_kernel (graph step)"
+        kernel = " + ".join(launched or ["plan_kernel", "rebind_kernel"]) + " (graph step)"
     achieved = nbytes / apply_avg_s / 1e9
-    src_sha = _sha(os.path.join(ROOT, "paper_2606_26631_gb300", "csrc", "prcr_rebind.cu"))
-    traffic = TRAFFIC.get((wl.name, src_sha))
+    src_sha = _sha(*(os.path.join(ROOT, "paper_2606_26631_gb300", "csrc", f)
+                     for f in ("prcr_rebind.cu", "prcr_device.cuh", "prcr_internal.h")))
+    traffic = TRAFFIC.get((wl.name, src_sha)) if split else None
     roof = dict(bound="hbm", achieved=achieved, peak=peak, unit="GB/s", frac=achieved / peak,
                 traffic=traffic, kernel=kernel, peak_kind=f"{peak_kind} copy (hbm_gbs)",
                 bytes_per_launch=nbytes, avg_launch_us=1e6 * apply_avg_s)
@@ -399,7 +475,7 @@ def run_gpu(args):
                         head_dim=wl.head_dim, sections=list(wl.sections), batch=wl.n_seqs,
                         tokens=batch.total_k, revisits=R, cache=f"{wl.cache}/{wl.block_size}",
                         L=wl.L, bytes_per_step=nbytes,
-                        l2="inputs larger than L2 (no flush): each step moves %.2f GB" % (nbytes / 1e9)),
+                        l2=flush.describe(nbytes)),
             pct_of_hbm_measured=100.0 * value / peak, pct_of_hbm_spec_8tbs=100.0 * value / SPEC_HBM_GBS,
             us_per_revisit=1e3 * ms_per_step / R,
             token_layers_per_s=batch.total_k * wl.n_layers * world * K / total_s,
@@ -409,14 +485,17 @@ def run_gpu(args):
             roofline=roof, cpu_baseline=cpu,
             e2e=dict(value=e2e_value, unit=UNIT, h2d_bytes_per_step=rv.h2d_bytes(),
                      d2h_bytes_per_step=rv.d2h_bytes(), steps=args.e2e_steps),
-            gpu_launches=2 * K, clocks=clk.summary(), parity=check)
+            gpu_launches=per_step * K, kernels_per_step=launched or None,
+            launches_counted_by="torch.profiler (CUPTI), one call" if launched
+            else "two entry points per step, one kernel each",
+            clocks=clk.summary(), parity=check)
         print(json.dumps(line), flush=True)
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
 
 
-def _timed(fn, steps, warmup, local):
+def _timed(fn, steps, warmup, local, flush):
     import torch
     stream = torch.cuda.current_stream()
     for _ in range(warmup):
@@ -426,12 +505,23 @@ def _timed(fn, steps, warmup, local):
           for _ in range(steps)]
     with Clocks(local) as clk:
         for e0, e1 in ev:
+            flush()
             e0.record(stream)
             fn()
             e1.record(stream)
         torch.cuda.synchronize()
     ms = [e0.elapsed_time(e1) for e0, e1 in ev]
     return ms, clk.summary()
+
+
+def _launch_keys(launched, expected, steps):
+    """gpu_launches from the kernels the profiler saw one step launch, else
+    from the entry points' own launch counts."""
+    if launched:
+        return dict(gpu_launches=len(launched) * steps, kernels_per_step=launched,
+                    launches_counted_by="torch.profiler (CUPTI), one step")
+    return dict(gpu_launches=expected * steps, kernels_per_step=None,
+                launches_counted_by="entry points' launch counts")
 
 
 def run_capture_path(args):
@@ -472,8 +562,10 @@ def run_capture_path(args):
     torch.cuda.synchronize()
     assert int(status.item()) == 0
     assert torch.equal(store_k.view(torch.int16), src.store_k.view(torch.int16))
-    ms, clk = _timed(step, args.steps, args.warmup, local)
     nbytes = B * M * nL * H * D * 2 * 6  # read k, v; write store k, v and cache k, v
+    launched = kernel_launches(step)
+    flush = L2Flush(dev, args.flush, nbytes)
+    ms, clk = _timed(step, args.steps, args.warmup, local, flush)
     t = sum(ms) / 1e3
     peak, kind = measured_peaks()
     value = nbytes * args.steps / t / 1e9
@@ -482,10 +574,11 @@ def run_capture_path(args):
         steps=args.steps, warmup=args.warmup, ms_per_step=1e3 * t / args.steps,
         higher_is_better=True, scaling="weak", vs_baseline=None, dtype="f32", io_dtype="bf16",
         data="synthetic", config=dict(workload=wl.name, batch=B, tokens_per_seq=M, n_layers=nL,
-                                      cache="paged/16", bytes_per_step=nbytes),
+                                      cache="paged/16", bytes_per_step=nbytes,
+                                      l2=flush.describe(nbytes)),
         roofline=dict(bound="hbm", achieved=value, peak=peak, unit="GB/s", frac=value / peak,
                       traffic=None, kernel="capture_kernel", peak_kind=f"{kind} copy (hbm_gbs)"),
-        gpu_launches=B * args.steps, clocks=clk)), flush=True)
+        **_launch_keys(launched, B, args.steps), clocks=clk)), flush=True)
 
 
 def run_decode_path(args):
@@ -519,9 +612,11 @@ def run_decode_path(args):
     step()
     torch.cuda.synchronize()
     assert int(status.item()) == 0
-    ms, clk = _timed(step, args.steps, args.warmup, local)
     slots = int(inp["seq_len"].sum())
     nbytes = slots * wl.n_layers * wl.n_kv_heads * wl.head_dim * 2 * 2
+    launched = kernel_launches(step)
+    flush = L2Flush(dev, args.flush, nbytes)
+    ms, clk = _timed(step, args.steps, args.warmup, local, flush)
     t = sum(ms) / 1e3
     peak, kind = measured_peaks()
     value = nbytes * args.steps / t / 1e9
@@ -531,11 +626,11 @@ def run_decode_path(args):
         higher_is_better=True, scaling="weak", vs_baseline=None, dtype="f32", io_dtype="bf16",
         data="synthetic", config=dict(workload=wl.name, batch=B, n_q_heads=Hq, max_len=max_len,
                                       slots=slots, cache="paged/16", bytes_per_step=nbytes,
-                                      workspace_bytes=nws),
+                                      workspace_bytes=nws, l2=flush.describe(nbytes)),
         roofline=dict(bound="hbm", achieved=value, peak=peak, unit="GB/s", frac=value / peak,
                       traffic=None, kernel="decode_kernel (+ merge)",
                       peak_kind=f"{kind} copy (hbm_gbs)"),
-        gpu_launches=(2 if nws else 1) * args.steps, clocks=clk)), flush=True)
+        **_launch_keys(launched, 2 if nws else 1, args.steps), clocks=clk)), flush=True)
 
 
 def run_select_path(args):
@@ -567,8 +662,10 @@ def run_select_path(args):
     def step():
         prcr.select_topk(cfg, sd, layer, q, batch.p_txt, k, idx, sro, rto, ws)
 
-    ms, clk = _timed(step, args.steps, args.warmup, local)
     nbytes = B * M * H * D * 2  # the layer's raw keys, read once
+    launched = kernel_launches(step)
+    flush = L2Flush(dev, args.flush, nbytes)
+    ms, clk = _timed(step, args.steps, args.warmup, local, flush)
     t = sum(ms) / 1e3
     peak, kind = measured_peaks()
     value = nbytes * args.steps / t / 1e9
@@ -578,11 +675,11 @@ def run_select_path(args):
         us_per_sequence=1e6 * t / args.steps / B, higher_is_better=True, scaling="weak",
         vs_baseline=None, dtype="f32", io_dtype="bf16", data="synthetic",
         config=dict(workload=wl.name, batch=B, tokens_per_seq=M, n_q_heads=Hq, k=k, layer=layer,
-                    bytes_per_step=nbytes),
+                    bytes_per_step=nbytes, l2=flush.describe(nbytes)),
         roofline=dict(bound="hbm", achieved=value, peak=peak, unit="GB/s", frac=value / peak,
-                      traffic=None, kernel="ads_logits_kernel + ads_select_kernel",
+                      traffic=None, kernel="ads_*_kernel (whole selection step)",
                       peak_kind=f"{kind} copy (hbm_gbs)"),
-        gpu_launches=2 * args.steps, clocks=clk)), flush=True)
+        **_launch_keys(launched, 5, args.steps), clocks=clk)), flush=True)
 
 
 def main():

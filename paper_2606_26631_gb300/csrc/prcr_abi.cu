@@ -155,7 +155,7 @@ PlanArgs make_plan_args(const prcr_store_desc* store, const prcr_cache_desc* cac
     return a;
 }
 
-enum KernelId { kRebind = 0, kCapture = 1 };
+enum KernelId { kRebind = 0, kCapture = 1, kFused = 2 };
 
 // Resident CTAs per SM of a kernel per (device, kernel, block, smem), cached.
 int blocks_per_sm(int dev, int block, size_t smem, int kernel = kRebind) {
@@ -168,8 +168,9 @@ int blocks_per_sm(int dev, int block, size_t smem, int kernel = kRebind) {
         if (it != cache.end()) return it->second;
     }
     int n = 0;
-    const cudaError_t e = kernel == kRebind ? rebind_blocks_per_sm(block, smem, &n)
-                                            : capture_blocks_per_sm(block, smem, &n);
+    const cudaError_t e = kernel == kRebind    ? rebind_blocks_per_sm(block, smem, &n)
+                          : kernel == kCapture ? capture_blocks_per_sm(block, smem, &n)
+                                               : fused_blocks_per_sm(block, smem, &n);
     if (e != cudaSuccess || n < 1) n = 1;
     std::lock_guard<std::mutex> g(mu);
     cache[key] = n;
@@ -219,7 +220,8 @@ int layers_per_cta(int64_t tiles, int n_layers, int64_t slots) {
 // Arguments and launch shape of the row-moving kernel (rebind or fused).
 int rebind_setup(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
                  const prcr_cache_desc* cache, const prcr_revisit_batch* b, const prcr_outputs* o,
-                 void* ws, RebindArgs& a, dim3& grid, int& block, size_t& smem) {
+                 void* ws, RebindArgs& a, dim3& grid, int& block, size_t& smem,
+                 KernelId kernel = kRebind) {
     a = RebindArgs{};
     a.store_k = static_cast<const uint16_t*>(store->k);
     a.store_v = static_cast<const uint16_t*>(store->v);
@@ -254,7 +256,7 @@ int rebind_setup(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return PRCR_ECUDA;
     const int64_t tiles = (b->total_k + T - 1) / T;
-    const int64_t slots = int64_t(sm_count(dev)) * blocks_per_sm(dev, block, smem);
+    const int64_t slots = int64_t(sm_count(dev)) * blocks_per_sm(dev, block, smem, kernel);
     const int G = layers_per_cta(tiles, cfg->n_layers, slots);
     const int64_t groups = (cfg->n_layers + G - 1) / G;
     a.layers_per_cta = G;
@@ -414,15 +416,23 @@ int prcr_rebind_inject(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
     const cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (batch->total_k > 0 && batch->total_k <= kFusedMaxTokens &&
         batch->n_revisits <= kFusedMaxRevisits && batch->n_seqs <= kFusedMaxSeqs) {
-        // a few small revisits: one kernel plans and moves them (no plan round trip)
+        // a few small revisits: one kernel plans and moves them (no plan round
+        // trip), when its grid runs as a single wave, so that every CTA's own
+        // planning happens at once instead of wave after wave
         FusedArgs fa;
-        fa.plan = make_plan_args(store, cache, batch, out, mode, L, flags, workspace);
         dim3 grid;
         int block = 0;
         size_t smem = 0;
-        rc = rebind_setup(cfg, store, cache, batch, out, workspace, fa.rebind, grid, block, smem);
+        rc = rebind_setup(cfg, store, cache, batch, out, workspace, fa.rebind, grid, block, smem,
+                          kFused);
         if (rc) return rc;
-        return launch_fused(fa, grid, block, smem, s) == cudaSuccess ? PRCR_OK : PRCR_ECUDA;
+        int dev = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess) return PRCR_ECUDA;
+        const int64_t resident = int64_t(sm_count(dev)) * blocks_per_sm(dev, block, smem, kFused);
+        if (int64_t(grid.x) * grid.y <= resident) {
+            fa.plan = make_plan_args(store, cache, batch, out, mode, L, flags, workspace);
+            return launch_fused(fa, grid, block, smem, s) == cudaSuccess ? PRCR_OK : PRCR_ECUDA;
+        }
     }
     rc = do_plan(store, cache, batch, out, mode, L, flags, workspace, s);
     if (rc) return rc;

@@ -170,6 +170,10 @@ __global__ void __launch_bounds__(512) fused_kernel(const __grid_constant__ Fuse
 
 }  // namespace
 
+cudaError_t fused_blocks_per_sm(int block, size_t smem, int* out) {
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, fused_kernel, block, smem);
+}
+
 cudaError_t launch_fused(const FusedArgs& a, dim3 grid, int block, size_t smem,
                          cudaStream_t stream) {
     fused_kernel<<<grid, block, smem, stream>>>(a);

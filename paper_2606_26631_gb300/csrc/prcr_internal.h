@@ -279,6 +279,7 @@ constexpr int kFusedMaxSeqs = 64;
 
 cudaError_t launch_fused(const FusedArgs& a, dim3 grid, int block, size_t smem,
                          cudaStream_t stream);
+cudaError_t fused_blocks_per_sm(int block, size_t smem, int* out);
 cudaError_t launch_plan(const PlanArgs& a, cudaStream_t stream);
 cudaError_t launch_rebind(const RebindArgs& a, dim3 grid, int block, size_t smem,
                           cudaStream_t stream);

@@ -8,6 +8,8 @@ there every position/slot/length is compared, K/V rows on sampled
 """
 import gc
 
+import re
+
 import numpy as np
 import pytest
 import torch
@@ -309,6 +311,23 @@ def test_graph_replay_matches(name):
     pu.full_check(batch, rv)
 
 
+def _kernel_names(fn):
+    """Names of this library's CUDA kernels that fn launches, as the profiler
+    (CUPTI) records them."""
+    from torch.profiler import ProfilerActivity, profile
+    for _ in range(3):  # the first session of a process records no kernels
+        with profile(activities=[ProfilerActivity.CPU, ProfilerActivity.CUDA]) as prof:
+            fn()
+            torch.cuda.synchronize()
+        names = set()
+        for e in prof.key_averages():
+            if e.device_type.name == "CUDA":
+                names.update(re.findall(r"\bprcr::.*?\b(\w+_kernel)\b", e.key))
+        if names:
+            return sorted(names)
+    return []
+
+
 SMALL = ["tiny", "qwen2vl-2b", "paper-8b-k32", "paper-8b-k128", "edge-d16", "edge-odd"]
 
 
@@ -327,8 +346,7 @@ def test_fused_path_matches_two_kernel_path(name, mode):
     assert batch.total_k <= 2048 and batch.n_revisits <= 64
     pristine_k = batch.cache_k.clone(); pristine_v = batch.cache_v.clone()
     fused = pu.make_revisit(batch, mode=mode)
-    fused.run()
-    torch.cuda.synchronize()
+    assert _kernel_names(fused.run) == ["fused_kernel"]
     fk, fv = batch.cache_k.clone(), batch.cache_v.clone()
     batch.cache_k.copy_(pristine_k); batch.cache_v.copy_(pristine_v)
     two = pu.make_revisit(batch, mode=mode)
@@ -341,6 +359,17 @@ def test_fused_path_matches_two_kernel_path(name, mode):
     assert torch.equal(fused.slot, two.slot)
     assert torch.equal(fused.cache_len_out, two.cache_len_out)
     assert torch.equal(fused.next_pos, two.next_pos)
+
+
+def test_large_batch_takes_two_kernels():
+    """A batch past the fused path's limits runs the plan kernel, then the
+    rebind + inject kernel."""
+    import parity_util as pu
+    batch = make_batch(get("qwen25vl-7b"), device=DEV)
+    assert batch.total_k > 2048
+    rv = pu.make_revisit(batch)
+    assert _kernel_names(rv.run) == ["plan_kernel", "rebind_kernel"]
+    assert rv.status_value() == 0
 
 
 def test_malformed_offsets_small_batch_write_nothing():
