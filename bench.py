@@ -67,6 +67,9 @@ def parse():
                          "decode: the first decode step over the active cache; select: the "
                          "attention-driven selection of the revisited set")
     ap.add_argument("--seqs", type=int, default=0, help="capture/decode: sequences (0 = workload's)")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="select: build the store with this many layers (0 = workload's); "
+                         "the selection reads the last one")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-samples", type=int, default=8,
@@ -647,6 +650,8 @@ def run_select_path(args):
     wl = get(args.workload)
     if args.seqs:
         wl = dataclasses.replace(wl, n_seqs=args.seqs)
+    if args.layers:
+        wl = dataclasses.replace(wl, n_layers=args.layers)
     batch = make_batch(wl, device=dev)
     B, M, H, D = wl.n_seqs, wl.n_tokens, wl.n_kv_heads, wl.head_dim
     Hq, k, layer = 4 * H, max(1, batch.total_k // B), wl.n_layers - 1

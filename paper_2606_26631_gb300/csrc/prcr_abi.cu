@@ -631,9 +631,10 @@ int prcr_select_topk(const prcr_rope_cfg* cfg, const prcr_store_desc* store, int
     {
         char* w = static_cast<char*>(workspace);
         const int64_t Bn = n_seqs, Hn = n_q_heads, M = store->n_tokens;
-        // one thread per (token, KV head) in a 256-thread CTA
-        int tile = 256 / H;
-        tile = tile < kSelectTokTile ? kSelectTokTile : (tile > 64 ? 64 : tile);
+        // token tiles of the logits kernel: 64 tokens (32 at head_dim 256, whose
+        // cos/sin rows are twice as long)
+        const int tile = cfg->head_dim > 128 ? 32 : 64;
+        a.n_seqs = n_seqs;
         a.tok_tile = tile;
         a.n_tiles = int32_t((M + tile - 1) / tile);
         const int64_t max_tiles = (M + kSelectTokTile - 1) / kSelectTokTile;
@@ -652,8 +653,11 @@ int prcr_select_topk(const prcr_rope_cfg* cfg, const prcr_store_desc* store, int
     a.rev_tok_off = rev_tok_off;
     a.seq_rev_off = seq_rev_off;
     copy_turn_freq(cfg, a.turn_freq);
-    return launch_select(a, n_seqs, static_cast<cudaStream_t>(stream)) == cudaSuccess ? PRCR_OK
-                                                                                     : PRCR_ECUDA;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return PRCR_ECUDA;
+    return launch_select(a, n_seqs, sm_count(dev), static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? PRCR_OK
+               : PRCR_ECUDA;
 }
 
 int64_t prcr_next_text_pos(int64_t p_txt, int64_t k_seq, int32_t mode) {

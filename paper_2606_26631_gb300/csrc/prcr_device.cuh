@@ -34,6 +34,24 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<const uint32_t*>(&v);
 }
 
+// Two floats as bf16 pairs: a head (round to nearest even) and the rounded
+// remainder, so that head + remainder keeps ~16 significant bits.
+__device__ __forceinline__ void split_bf16x2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+    hi = pack_bf16x2(x0, x1);
+    lo = pack_bf16x2(x0 - lo_f32(hi), x1 - hi_f32(hi));
+}
+
+// D += A B on tensor cores: mma.sync m16n8k16, bf16 operands, float32
+// accumulate (fragment layouts of the PTX ISA for this shape).
+__device__ __forceinline__ void mma_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                          uint32_t a3, uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+        "{%8,%9}, {%0,%1,%2,%3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
 // Rotate four bf16 pairs held as (first-half word x, second-half word y):
 // x' = x cos - y sin, y' = y cos + x sin, float32, bf16 round-to-nearest-even.
 __device__ __forceinline__ void rotate_word(uint32_t x, uint32_t y, float c0, float s0, float c1,

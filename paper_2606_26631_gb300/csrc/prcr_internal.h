@@ -251,7 +251,8 @@ struct SelectArgs {
     float* norm;                // workspace [B][n_q_heads][2] (max, 1 / (sum * n_q_heads))
     float* rel;                 // workspace [B][n_tokens] relevance
     float* qrot;                // workspace [B][n_q_heads][D] rotated, scaled queries
-    int32_t n_tiles;            // token tiles of the logits kernel
+    int32_t n_seqs;
+    int32_t n_tiles;            // token tiles of the logits kernel per sequence
     int32_t tok_tile;           // tokens per tile
     float* score_out;           // optional [B][n_tokens]
     int32_t* idx_out;           // [B][k]
@@ -260,7 +261,7 @@ struct SelectArgs {
     uint64_t turn_freq[kMaxPairs];  // pair i: round(inv_freq_i / (2 pi) * 2^64)
 };
 
-cudaError_t launch_select(const SelectArgs& a, int n_seqs, cudaStream_t stream);
+cudaError_t launch_select(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream);
 
 cudaError_t launch_decode(const DecodeArgs& a, int gp, dim3 grid, size_t smem,
                           cudaStream_t stream);

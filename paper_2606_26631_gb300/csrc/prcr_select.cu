@@ -10,32 +10,22 @@
 // written in ascending token order, one revisit per sequence, as the offsets
 // and indices prcr_rebind_inject takes.
 //
-// Kernel 0 rotates each sequence's trigger queries once. Kernel 1 (logits):
-// a CTA owns 256 / H (16..64) tokens of one sequence and all H KV heads, one
-// thread per (token, KV head); it copies the rotated queries (pre-scaled by
-// 1/sqrt(D)) into shared memory and computes each token's cos/sin once;
-// thread (token, KV head) rotates its raw key row on the fly and forms the logits of the
-// group's query heads, plus the tile's per-head softmax statistics (max, sum
-// of exp). Kernel 2 (norm) merges the tiles' statistics into each head's
-// normaliser; kernel 3 (relevance) averages every token's per-head softmax
-// weight; kernel 4 (select), one CTA per sequence, finds the K-th largest
-// relevance with a 4-pass 8-bit radix select on the float bits (relevance >=
-// 0, so bit order is value order) and compacts the selection in index order
-// with block-wide scans.
+// Kernel 0 rotates each sequence's trigger queries once (pre-scaled by
+// 1/sqrt(D)). Kernel 1 (logits, persistent) forms every (token, query head)
+// logit from the raw key rotated on the fly at the token's own coordinates,
+// and each token tile's per-head softmax statistics (max, sum of exp).
+// Kernel 2 (norm) merges the tiles' statistics into each head's normaliser;
+// kernel 3 (relevance) averages every token's per-head softmax weight;
+// kernel 4 (select), one CTA per sequence, finds the K-th largest relevance
+// by counting against thresholds two bits at a time on the float bits
+// (relevance >= 0, so bit order is value order) and compacts the selection
+// in index order with block-wide scans.
 #include <cmath>
 
-#include "prcr_internal.h"
+#include "prcr_device.cuh"
 
 namespace prcr {
 namespace {
-
-__device__ __forceinline__ int pair_axis(int i, int layout, int st, int sh, int sw) {
-    if (layout == PRCR_LAYOUT_SECTIONED) return i < st ? 0 : (i < st + sh ? 1 : 2);
-    const int r = i % 3;
-    if (r == 1 && i < 3 * sh) return 1;
-    if (r == 2 && i < 3 * sw) return 2;
-    return 0;
-}
 
 // The trigger queries of each sequence, rotated at (p, p, p) (pair i turns by
 // p * inv_freq_i for every head) and scaled by 1/sqrt(D), once per sequence.
@@ -57,132 +47,372 @@ __global__ void __launch_bounds__(256) ads_query_kernel(const __grid_constant__ 
     }
 }
 
-// NV: upper bound of the 16-byte vectors in half a head row (head_dim / 16).
-template <int NV>
-__global__ void __launch_bounds__(256) ads_logits_kernel(const __grid_constant__ SelectArgs a) {
-    extern __shared__ __align__(16) float sm[];
-    const int D = a.head_dim, P = D >> 1, Hq = a.n_q_heads, H = a.n_kv_heads;
-    const int T = a.tok_tile;
-    const int qs = D + 4;  // padded row strides (multiples of 4: float4 rows)
-    const int cs = P + 4;
-    float* q_s = sm;                 // [Hq][D + 4]
-    float* cos_s = q_s + Hq * qs;    // [T][P + 4]
-    float* sin_s = cos_s + T * cs;
-    float* lg_s = sin_s + T * cs;    // [Hq][T + 1] this tile's logits (padded rows)
-    const int b = blockIdx.y;
-    const int m0 = blockIdx.x * T;
+// Rotation of an integer coordinate: the turn fraction c * rate mod 1 in
+// 0.32 fixed point is bits 32..63 of the 64-bit product c * rate (rate in
+// 0.64 fixed point; the product's wrap mod 2^64 keeps those bits exact for
+// any int32 c), then one sin/cos evaluation on [-pi, pi).
+__device__ __forceinline__ void sincos_coord(int c, uint64_t turn_freq, float* s, float* co) {
+    const uint64_t prod = static_cast<uint64_t>(static_cast<int64_t>(c)) * turn_freq;
+    const int frac = static_cast<int>(static_cast<uint32_t>(prod >> 32));
+    __sincosf(float(frac) * 1.4629180792671596e-9f, s, co);  // 2 pi / 2^32
+}
 
-    // rotated queries of the sequence (ads_query_kernel) and the tile's coordinates
-    __shared__ int s_crd[3 * 64];
-    {
-        const float4* src = reinterpret_cast<const float4*>(a.qrot + int64_t(b) * Hq * D);
-        const int nv = Hq * D / 4;
-        // row of query head hq = kh * g + h is h * H + kh: the rows the 8 lanes of a
-        // quarter-warp read together (same h, consecutive kh) fall in distinct banks
-        const int g = Hq / H;
-#pragma unroll 4
-        for (int e = threadIdx.x; e < nv; e += blockDim.x) {
-            const int hq = (4 * e) / D, d = 4 * e - hq * D;
-            *reinterpret_cast<float4*>(q_s + ((hq % g) * H + hq / g) * qs + d) = src[e];
+// 16-byte chunk c of a shared row stored at c ^ bit 3 of c: the 8 lanes of a
+// quarter-warp that read chunks 2v (or 2v + 1), v = 0..7, hit 8 distinct
+// bank groups.
+__device__ __forceinline__ int swz(int c) { return c ^ ((c >> 3) & 1); }
+
+// Logits of every (token, query head). Persistent: CTA c takes a contiguous
+// run of the B * n_tiles token tiles (sequence-major), so it reloads the
+// rotated queries only when its run enters a new sequence. Per tile of T
+// tokens: the tile's cos/sin (one per token and pair) go to shared memory;
+// then each row (token, KV head) is taken by L lanes, lane v holding pairs
+// 8v..8v+7 (one 16-byte load from each half of the raw key row), which it
+// rotates and dots with the group's query heads in packed float2 FMAs; the
+// lanes' partial sums are reduced by shuffles. The loads of a lane's next two
+// rows are in flight during the current row's arithmetic. The tile's logits are staged
+// in shared memory, reduced to per-head (max, sum of exp) and written out
+// coalesced.
+// L lanes per row (a power of two >= head_dim / 16); G = the GQA group size g
+// for g = 1, 2 and 4, else 8 (heads h >= g skipped).
+template <int L, int G>
+__global__ void __launch_bounds__(256, 3) ads_logits_kernel(const __grid_constant__ SelectArgs a) {
+    extern __shared__ __align__(16) float sm[];
+    const int D = a.head_dim, P = D >> 1, Hq = a.n_q_heads, H = a.n_kv_heads, g = Hq / H;
+    const int NV = P >> 3, M = a.n_tokens, T = a.tok_tile;
+    const int qrow = D / 4 + 1;  // chunks per row; odd, so adjacent rows fall in other banks
+    const int crow = P / 4 + 1;
+    float4* q_s = reinterpret_cast<float4*>(sm);  // row h * H + kh holds query head kh * g + h
+    float4* c_s = q_s + Hq * qrow;                // [T] cos rows
+    float4* s_s = c_s + T * crow;                 // [T] sin rows
+    float* lg_s = reinterpret_cast<float*>(s_s + T * crow);  // [Hq][T + 1]
+    int* crd_s = reinterpret_cast<int*>(lg_s + Hq * (T + 1));  // [T][3]
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int v = tid & (L - 1), grp = tid / L;
+    constexpr int RS = 256 / L;  // rows per pass
+    const bool act = v < NV;
+    const int t0_r = grp / H, kh0_r = grp - t0_r * H;  // a lane's first row in a tile
+    const int dt_r = RS / H, dkh_r = RS - dt_r * H;     // its step between rows
+    const int dt_e = 256 / P, di_e = 256 - dt_e * P;    // cos/sin loop step (t, i)
+    const int64_t total = int64_t(a.n_seqs) * a.n_tiles;
+    const int64_t t_beg = total * blockIdx.x / gridDim.x, t_end = total * (blockIdx.x + 1) / gridDim.x;
+    int cur_b = -1;
+
+    for (int64_t tile = t_beg; tile < t_end; ++tile) {
+        const int b = int(tile / a.n_tiles), j = int(tile % a.n_tiles);
+        const int m0 = j * T, nt = min(T, M - m0);
+        if (b != cur_b) {
+            const float4* src = reinterpret_cast<const float4*>(a.qrot + int64_t(b) * Hq * D);
+            const int nch = D / 4;
+            for (int e = tid; e < Hq * nch; e += blockDim.x) {
+                const int hq = e / nch, c = e - hq * nch;
+                q_s[((hq % g) * H + hq / g) * qrow + swz(c)] = src[e];
+            }
+            cur_b = b;
         }
         const int32_t* crd = a.coords + int64_t(b) * a.coord_seq_stride + 3 * int64_t(m0);
-        const int nc = 3 * min(T, a.n_tokens - m0);
-        for (int e = threadIdx.x; e < nc; e += blockDim.x) s_crd[e] = crd[e];
-    }
-    __syncthreads();
-    for (int e = threadIdx.x; e < T * P; e += blockDim.x) {
-        const int t = e / P, i = e - (e / P) * P;
-        const int m = m0 + t;
-        float sn = 0.0f, cn = 1.0f;
-        if (m < a.n_tokens) {
+        for (int e = tid; e < 3 * nt; e += blockDim.x) crd_s[e] = crd[e];
+        __syncthreads();
+        float* cf = reinterpret_cast<float*>(c_s);
+        float* sf = reinterpret_cast<float*>(s_s);
+        for (int e = tid, t = tid / P, i = tid - (tid / P) * P; e < nt * P;
+             e += 256, t += dt_e, i += di_e) {
+            if (i >= P) {
+                i -= P;
+                ++t;
+            }
             const int ax = pair_axis(i, a.layout, a.sec_t, a.sec_h, a.sec_w);
-            sincos_turns(double(s_crd[3 * t + ax]), a.turn_freq[i], &sn, &cn);
+            float sn, cn;
+            sincos_coord(crd_s[3 * t + ax], a.turn_freq[i], &sn, &cn);
+            const int o = (t * crow + swz(i >> 2)) * 4 + (i & 3);
+            cf[o] = cn;
+            sf[o] = sn;
         }
-        cos_s[t * cs + i] = cn;
-        sin_s[t * cs + i] = sn;
-    }
-    __syncthreads();
+        __syncthreads();
 
-    const int g = Hq / H;
-    for (int e = threadIdx.x; e < T * H; e += blockDim.x) {
-        const int t = e / H, kh = e - (e / H) * H;
-        const int m = m0 + t;
-        if (m >= a.n_tokens) continue;
-        const uint16_t* kr = a.store_k + int64_t(b) * a.store_seq_stride +
-                             int64_t(a.layer) * a.store_layer_stride +
-                             int64_t(m) * a.store_token_stride + int64_t(kh) * D;
-        const float4* c4 = reinterpret_cast<const float4*>(cos_s + t * cs);
-        const float4* s4 = reinterpret_cast<const float4*>(sin_s + t * cs);
-        float acc[8];
-#pragma unroll
-        for (int h = 0; h < 8; ++h) acc[h] = 0.0f;
-        // the whole row is requested before any of it is used: one load latency
-        uint4 klo[NV], khi[NV];
-#pragma unroll
-        for (int v = 0; v < NV; ++v) {
-            if (8 * v < P) {
-                klo[v] = __ldg(reinterpret_cast<const uint4*>(kr + 8 * v));
-                khi[v] = __ldg(reinterpret_cast<const uint4*>(kr + 8 * v + P));
-            }
+        const uint16_t* kbase = a.store_k + int64_t(b) * a.store_seq_stride +
+                                int64_t(a.layer) * a.store_layer_stride + 8 * v;
+        const int rows = nt * H;
+        // row r = t * H + kh; a lane's rows advance by RS = dt_r * H + dkh_r.
+        // Rows r + RS and r + 2 RS are in flight while row r is computed.
+        int t = t0_r, kh = kh0_r;        // the row computed
+        int tn = t + dt_r, khn = kh + dkh_r;  // the row two ahead, after the step below
+        if (khn >= H) {
+            khn -= H;
+            ++tn;
         }
-#pragma unroll
-        for (int v = 0; v < NV; ++v) {
-            if (8 * v >= P) break;
-            const int i0 = 8 * v;
-            const uint4 lo = klo[v];
-            const uint4 hi = khi[v];
-            const float4 ca = c4[i0 / 4], cb = c4[i0 / 4 + 1];
-            const float4 sa = s4[i0 / 4], sb = s4[i0 / 4 + 1];
-            const uint32_t lw[4] = {lo.x, lo.y, lo.z, lo.w};
-            const uint32_t hw[4] = {hi.x, hi.y, hi.z, hi.w};
-            const float cc[8] = {ca.x, ca.y, ca.z, ca.w, cb.x, cb.y, cb.z, cb.w};
-            const float ss[8] = {sa.x, sa.y, sa.z, sa.w, sb.x, sb.y, sb.z, sb.w};
-            float kx[8], ky[8];
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const uint32_t wl = lw[j >> 1], wh = hw[j >> 1];
-                const float x = __uint_as_float((j & 1) ? (wl & 0xffff0000u) : (wl << 16));
-                const float y = __uint_as_float((j & 1) ? (wh & 0xffff0000u) : (wh << 16));
-                kx[j] = fmaf(x, cc[j], -y * ss[j]);
-                ky[j] = fmaf(y, cc[j], x * ss[j]);
+        uint4 lo_1 = make_uint4(0, 0, 0, 0), hi_1 = lo_1, lo_2 = lo_1, hi_2 = lo_1;
+        if (grp < rows && act) {
+            const uint16_t* kr = kbase + int64_t(m0 + t) * a.store_token_stride + kh * D;
+            lo_1 = ld_stream(kr);
+            hi_1 = ld_stream(kr + P);
+        }
+        if (grp + RS < rows && act) {
+            const uint16_t* kr = kbase + int64_t(m0 + tn) * a.store_token_stride + khn * D;
+            lo_2 = ld_stream(kr);
+            hi_2 = ld_stream(kr + P);
+        }
+        for (int r = grp; r - grp < rows; r += RS) {
+            const uint4 lo = lo_1, hi = hi_1;
+            lo_1 = lo_2;
+            hi_1 = hi_2;
+            tn += dt_r;
+            khn += dkh_r;
+            if (khn >= H) {
+                khn -= H;
+                ++tn;
             }
+            if (r + 2 * RS < rows && act) {
+                const uint16_t* kr = kbase + int64_t(m0 + tn) * a.store_token_stride + khn * D;
+                lo_2 = ld_stream(kr);
+                hi_2 = ld_stream(kr + P);
+            }
+            float acc[G];
 #pragma unroll
-            for (int h = 0; h < 8; ++h) {
-                if (h < g) {
-                    const float4* qh = reinterpret_cast<const float4*>(q_s + (h * H + kh) * qs);
-                    const float4 qa = qh[i0 / 4], qb2 = qh[i0 / 4 + 1];
-                    const float4 qc = qh[(i0 + P) / 4], qd = qh[(i0 + P) / 4 + 1];
-                    float r = acc[h];
-                    r = fmaf(qa.x, kx[0], r); r = fmaf(qa.y, kx[1], r);
-                    r = fmaf(qa.z, kx[2], r); r = fmaf(qa.w, kx[3], r);
-                    r = fmaf(qb2.x, kx[4], r); r = fmaf(qb2.y, kx[5], r);
-                    r = fmaf(qb2.z, kx[6], r); r = fmaf(qb2.w, kx[7], r);
-                    r = fmaf(qc.x, ky[0], r); r = fmaf(qc.y, ky[1], r);
-                    r = fmaf(qc.z, ky[2], r); r = fmaf(qc.w, ky[3], r);
-                    r = fmaf(qd.x, ky[4], r); r = fmaf(qd.y, ky[5], r);
-                    r = fmaf(qd.z, ky[6], r); r = fmaf(qd.w, ky[7], r);
-                    acc[h] = r;
+            for (int h = 0; h < G; ++h) acc[h] = 0.0f;
+            if (r < rows && act) {
+                const float4* cr = c_s + t * crow;
+                const float4* sr = s_s + t * crow;
+                const float4 ca = cr[swz(2 * v)], cb = cr[swz(2 * v + 1)];
+                const float4 sa = sr[swz(2 * v)], sb = sr[swz(2 * v + 1)];
+                const uint32_t lw[4] = {lo.x, lo.y, lo.z, lo.w};
+                const uint32_t hw[4] = {hi.x, hi.y, hi.z, hi.w};
+                const float2 c2[4] = {make_float2(ca.x, ca.y), make_float2(ca.z, ca.w),
+                                      make_float2(cb.x, cb.y), make_float2(cb.z, cb.w)};
+                const float2 s2[4] = {make_float2(sa.x, sa.y), make_float2(sa.z, sa.w),
+                                      make_float2(sb.x, sb.y), make_float2(sb.z, sb.w)};
+                float2 kx[4], ky[4];
+#pragma unroll
+                for (int w = 0; w < 4; ++w) {
+                    const float2 x = make_float2(__uint_as_float(lw[w] << 16),
+                                                 __uint_as_float(lw[w] & 0xffff0000u));
+                    const float2 y = make_float2(__uint_as_float(hw[w] << 16),
+                                                 __uint_as_float(hw[w] & 0xffff0000u));
+                    const float2 ys = __fmul2_rn(y, s2[w]);
+                    const float2 xs = __fmul2_rn(x, s2[w]);
+                    kx[w] = __ffma2_rn(x, c2[w], make_float2(-ys.x, -ys.y));
+                    ky[w] = __ffma2_rn(y, c2[w], xs);
+                }
+#pragma unroll
+                for (int h = 0; h < G; ++h) {
+                    if (G != 8 || h < g) {
+                        const float4* qr = q_s + (h * H + kh) * qrow;
+                        const float4 qa = qr[swz(2 * v)], qb = qr[swz(2 * v + 1)];
+                        const float4 qc = qr[swz(P / 4 + 2 * v)], qd = qr[swz(P / 4 + 2 * v + 1)];
+                        float2 s2a = __fmul2_rn(make_float2(qa.x, qa.y), kx[0]);
+                        s2a = __ffma2_rn(make_float2(qa.z, qa.w), kx[1], s2a);
+                        s2a = __ffma2_rn(make_float2(qb.x, qb.y), kx[2], s2a);
+                        s2a = __ffma2_rn(make_float2(qb.z, qb.w), kx[3], s2a);
+                        s2a = __ffma2_rn(make_float2(qc.x, qc.y), ky[0], s2a);
+                        s2a = __ffma2_rn(make_float2(qc.z, qc.w), ky[1], s2a);
+                        s2a = __ffma2_rn(make_float2(qd.x, qd.y), ky[2], s2a);
+                        s2a = __ffma2_rn(make_float2(qd.z, qd.w), ky[3], s2a);
+                        acc[h] = s2a.x + s2a.y;
+                    }
                 }
             }
-        }
 #pragma unroll
-        for (int h = 0; h < 8; ++h)
-            if (h < g) {
-                a.logits[(int64_t(b) * Hq + kh * g + h) * a.n_tokens + m] = acc[h];
-                lg_s[(kh * g + h) * (T + 1) + t] = acc[h];
+            for (int o = L / 2; o; o >>= 1) {
+#pragma unroll
+                for (int h = 0; h < G; ++h) acc[h] += __shfl_xor_sync(0xffffffffu, acc[h], o);
             }
+            if (r < rows && v == 0) {
+#pragma unroll
+                for (int h = 0; h < G; ++h)
+                    if (G != 8 || h < g) lg_s[(kh * g + h) * (T + 1) + t] = acc[h];
+            }
+            t += dt_r;
+            kh += dkh_r;
+            if (kh >= H) {
+                kh -= H;
+                ++t;
+            }
+        }
+        __syncthreads();
+
+        // per query head: the tile's (max, sum of exp), and its logits written out coalesced
+        for (int hq = warp; hq < Hq; hq += blockDim.x >> 5) {
+            const float* row = lg_s + hq * (T + 1);
+            float mx = -INFINITY;
+            for (int t = lane; t < nt; t += 32) mx = fmaxf(mx, row[t]);
+#pragma unroll
+            for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            float z = 0.0f;
+            float* dst = a.logits + (int64_t(b) * Hq + hq) * M + m0;
+            for (int t = lane; t < nt; t += 32) {
+                z += expf(row[t] - mx);
+                dst[t] = row[t];
+            }
+#pragma unroll
+            for (int o = 16; o; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
+            if (lane == 0) {
+                float* ts = a.tile_stats + ((int64_t(b) * Hq + hq) * a.n_tiles + j) * 2;
+                ts[0] = mx;
+                ts[1] = z;
+            }
+        }
+        // the next tile rewrites the coordinates first, then (after a barrier)
+        // the cos/sin rows and logits this tile's warps may still be reading
     }
-    __syncthreads();
-    // this tile's softmax statistics per query head: max and sum of exp
-    const int nt = min(T, a.n_tokens - m0);
-    for (int hq = threadIdx.x; hq < Hq; hq += blockDim.x) {
-        float mx = -INFINITY;
-        for (int t = 0; t < nt; ++t) mx = fmaxf(mx, lg_s[hq * (T + 1) + t]);
-        float sm2 = 0.0f;
-        for (int t = 0; t < nt; ++t) sm2 += expf(lg_s[hq * (T + 1) + t] - mx);
-        float* ts = a.tile_stats + ((int64_t(b) * Hq + hq) * a.n_tiles + blockIdx.x) * 2;
-        ts[0] = mx;
-        ts[1] = sm2;
+}
+
+// D += A B on tensor cores: mma.sync m16n8k8 with tf32 operands (the upper
+// 19 bits of each float32 register), float32 accumulate.
+__device__ __forceinline__ void mma_1688_tf32(float (&c)[4], uint32_t a0, uint32_t a2, uint32_t b0,
+                                              uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+        "{%8,%9}, {%0,%1,%2,%3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
+}
+
+// A float32 as tf32 head (round to nearest, ties away) and float32 remainder
+// (exact); the remainder enters the MMA truncated to tf32, so head +
+// remainder carries ~21 significant bits.
+__device__ __forceinline__ void split_tf32(float x, uint32_t& hi, uint32_t& lo) {
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(hi) : "f"(x));
+    lo = __float_as_uint(x - __uint_as_float(hi));
+}
+
+// Tensor-core logits (head_dim 64 and 128). Persistent over token tiles like
+// the kernel above; a tile is 64 tokens, one octet of 8 per warp, and a warp
+// takes its octet through all KV heads:
+//   S (16 rows = the group's query heads, rows >= g zero; 8 tokens)
+//     = Q (16 x D) K_rot^T (D x 8), D / 8 k-steps of mma.sync m16n8k8 (tf32).
+// The dot product does not depend on the order of the dimensions, so k-step j
+// of lane group t (= lane & 3) takes pair t * P/4 + j: k-slot t holds its
+// first-half dimension and k-slot t + 4 its rotate-half partner. A lane then
+// owns P/4 whole pairs of its token (= lane >> 2), loads them as two
+// contiguous runs and rotates them itself with its own cos/sin, computed once
+// per octet and reused for every KV head. Queries and rotated keys are split
+// into tf32 head + remainder and three products are summed (head x head,
+// head x remainder, remainder x head; float32 accumulate), which keeps the
+// logits at float32-level accuracy over float32's range. The accumulator of
+// lane (g, t) holds head g at tokens 2t, 2t+1 of the octet.
+template <int D>
+__global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_constant__ SelectArgs a) {
+    constexpr int P = D / 2, PL = P / 4, T = 64;
+    constexpr int NW = PL / 8;  // 16-byte loads per half row per lane
+    extern __shared__ __align__(16) float sm[];
+    const int Hq = a.n_q_heads, H = a.n_kv_heads, g = Hq / H, M = a.n_tokens;
+    uint4* qa_s = reinterpret_cast<uint4*>(sm);                // [H][PL][32]: (a0 hi, a0 lo, a2 hi, a2 lo)
+    float* lg_s = reinterpret_cast<float*>(qa_s + H * PL * 32);  // [Hq][T + 1]
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int gid = lane >> 2, tq = lane & 3;
+    const int64_t total = int64_t(a.n_seqs) * a.n_tiles;
+    const int64_t t_beg = total * blockIdx.x / gridDim.x, t_end = total * (blockIdx.x + 1) / gridDim.x;
+    // axis of each of this lane's pairs, two bits each
+    uint32_t axes = 0u;
+#pragma unroll
+    for (int p = 0; p < PL; ++p)
+        axes |= uint32_t(pair_axis(tq * PL + p, a.layout, a.sec_t, a.sec_h, a.sec_w)) << (2 * p);
+    int cur_b = -1;
+
+    for (int64_t tile = t_beg; tile < t_end; ++tile) {
+        const int b = int(tile / a.n_tiles), j = int(tile % a.n_tiles);
+        const int m0 = j * T, nt = min(T, M - m0);
+        if (b != cur_b) {
+            // the sequence's rotated queries as A fragments, split once
+            const float* qs = a.qrot + int64_t(b) * Hq * D;
+            for (int e = tid; e < H * PL * 32; e += blockDim.x) {
+                const int kh = e / (PL * 32), ks = (e / 32) % PL, ln = e & 31;
+                const int h = ln >> 2, tt = ln & 3;
+                uint4 f = make_uint4(0u, 0u, 0u, 0u);
+                if (h < g) {
+                    const float* qr = qs + (kh * g + h) * D + tt * PL + ks;
+                    split_tf32(qr[0], f.x, f.y);
+                    split_tf32(qr[P], f.z, f.w);
+                }
+                qa_s[e] = f;
+            }
+            cur_b = b;
+        }
+        __syncthreads();
+
+        // this warp's octet: the lane's token and its cos/sin for pairs tq * PL ..
+        const int to = 8 * warp + gid;  // token within the tile
+        const bool live = to < nt;
+        const int m = m0 + (live ? to : 0);
+        float cs[PL], sn[PL];
+        {
+            const int32_t* crd = a.coords + int64_t(b) * a.coord_seq_stride + 3 * int64_t(m);
+            const int c0 = crd[0], c1 = crd[1], c2 = crd[2];
+#pragma unroll
+            for (int p = 0; p < PL; ++p) {
+                const uint32_t ax = (axes >> (2 * p)) & 3u;
+                sincos_coord(ax == 0 ? c0 : (ax == 1 ? c1 : c2), a.turn_freq[tq * PL + p], &sn[p], &cs[p]);
+            }
+        }
+        const uint16_t* krow = a.store_k + int64_t(b) * a.store_seq_stride +
+                               int64_t(a.layer) * a.store_layer_stride +
+                               int64_t(m) * a.store_token_stride + tq * PL;
+        uint4 xn[NW], yn[NW];
+#pragma unroll
+        for (int u = 0; u < NW; ++u) {
+            xn[u] = live ? ld_stream(krow + 8 * u) : make_uint4(0u, 0u, 0u, 0u);
+            yn[u] = live ? ld_stream(krow + P + 8 * u) : make_uint4(0u, 0u, 0u, 0u);
+        }
+        for (int kh = 0; kh < H; ++kh) {
+            uint32_t xw[4 * NW], yw[4 * NW];
+#pragma unroll
+            for (int u = 0; u < NW; ++u) {
+                xw[4 * u] = xn[u].x; xw[4 * u + 1] = xn[u].y; xw[4 * u + 2] = xn[u].z; xw[4 * u + 3] = xn[u].w;
+                yw[4 * u] = yn[u].x; yw[4 * u + 1] = yn[u].y; yw[4 * u + 2] = yn[u].z; yw[4 * u + 3] = yn[u].w;
+            }
+            if (kh + 1 < H) {  // the next head's pairs, in flight during this head's MMAs
+#pragma unroll
+                for (int u = 0; u < NW; ++u) {
+                    xn[u] = live ? ld_stream(krow + (kh + 1) * D + 8 * u) : make_uint4(0u, 0u, 0u, 0u);
+                    yn[u] = live ? ld_stream(krow + (kh + 1) * D + P + 8 * u) : make_uint4(0u, 0u, 0u, 0u);
+                }
+            }
+            float c[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+            const uint4* qa = qa_s + kh * PL * 32 + lane;
+#pragma unroll
+            for (int ks = 0; ks < PL; ++ks) {
+                // pair ks of this lane: element ks of each half
+                const float x = (ks & 1) ? hi_f32(xw[ks >> 1]) : lo_f32(xw[ks >> 1]);
+                const float y = (ks & 1) ? hi_f32(yw[ks >> 1]) : lo_f32(yw[ks >> 1]);
+                const float kx = fmaf(x, cs[ks], -y * sn[ks]);
+                const float ky = fmaf(y, cs[ks], x * sn[ks]);
+                uint32_t bxh, bxl, byh, byl;
+                split_tf32(kx, bxh, bxl);
+                split_tf32(ky, byh, byl);
+                const uint4 f = qa[ks * 32];
+                mma_1688_tf32(c, f.x, f.z, bxh, byh);
+                mma_1688_tf32(c, f.y, f.w, bxh, byh);
+                mma_1688_tf32(c, f.x, f.z, bxl, byl);
+            }
+            if (gid < g) {  // (rows are T + 1 floats apart: 4-byte stores)
+                float* dst = lg_s + (kh * g + gid) * (T + 1) + 8 * warp + 2 * tq;
+                dst[0] = c[0];
+                dst[1] = c[1];
+            }
+        }
+        __syncthreads();
+
+        for (int hq = warp; hq < Hq; hq += blockDim.x >> 5) {
+            const float* row = lg_s + hq * (T + 1);
+            float mx = -INFINITY;
+            for (int t = lane; t < nt; t += 32) mx = fmaxf(mx, row[t]);
+#pragma unroll
+            for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            float z = 0.0f;
+            float* dst = a.logits + (int64_t(b) * Hq + hq) * M + m0;
+            for (int t = lane; t < nt; t += 32) {
+                z += expf(row[t] - mx);
+                dst[t] = row[t];
+            }
+#pragma unroll
+            for (int o = 16; o; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
+            if (lane == 0) {
+                float* ts = a.tile_stats + ((int64_t(b) * Hq + hq) * a.n_tiles + j) * 2;
+                ts[0] = mx;
+                ts[1] = z;
+            }
+        }
     }
 }
 
@@ -258,64 +488,79 @@ __device__ __forceinline__ int block_scan(int v, int* s_warp, int* out_excl) {
     return total;
 }
 
+// PER: relevances per thread (a thread keeps its PER consecutive tokens in
+// registers; 1024 * PER >= n_tokens).
+template <int PER>
 __global__ void __launch_bounds__(1024) ads_select_kernel(const __grid_constant__ SelectArgs a) {
-    extern __shared__ __align__(16) float rel[];  // [n_tokens]
     __shared__ int s_warp[32];
-    __shared__ unsigned int s_hist[256];
-    __shared__ unsigned int s_prefix, s_kleft;
+    __shared__ unsigned int s_cnt[3 * 32];
     const int b = blockIdx.x;
     const int M = a.n_tokens;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int beg = threadIdx.x * PER;
 
-    // relevance of this sequence's tokens (from the relevance kernel)
+    // this thread's relevances (from the relevance kernel); tokens past the
+    // end read as 0 and are excluded wherever 0 could count
+    unsigned int key[PER];
     const float* rs = a.rel + int64_t(b) * M;
-    for (int m = threadIdx.x; m < M; m += blockDim.x) rel[m] = rs[m];
-    if (threadIdx.x == 0) {
-        s_prefix = 0u;
-        s_kleft = unsigned(a.k);
+#pragma unroll
+    for (int i = 0; i < PER; ++i) key[i] = beg + i < M ? __float_as_uint(rs[beg + i]) : 0u;
+
+    // 1. the K-th largest relevance, two bits per round from the top: of the
+    // candidates X | d << bit (d = 1, 2, 3) keep the largest that at least K
+    // keys reach (relevance >= 0, so float bits order as values; every
+    // candidate is >= 1, so the padding never counts). Counting against
+    // thresholds needs no histogram, hence no atomics on the few bins that
+    // relevances sharing their high bits would all fall into.
+    const unsigned int K = unsigned(a.k);
+    unsigned int X = 0u;
+    for (int bit = 30; bit >= 0; bit -= 2) {
+        const unsigned int x1 = X | (1u << bit), x2 = X | (2u << bit), x3 = X | (3u << bit);
+        unsigned int c1 = 0u, c2 = 0u, c3 = 0u;
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            c1 += key[i] >= x1;
+            c2 += key[i] >= x2;
+            c3 += key[i] >= x3;
+        }
+        c1 = __reduce_add_sync(0xffffffffu, c1);
+        c2 = __reduce_add_sync(0xffffffffu, c2);
+        c3 = __reduce_add_sync(0xffffffffu, c3);
+        if (lane == 0) {
+            s_cnt[warp] = c1;
+            s_cnt[32 + warp] = c2;
+            s_cnt[64 + warp] = c3;
+        }
+        __syncthreads();
+        const unsigned int t1 = __reduce_add_sync(0xffffffffu, s_cnt[lane]);
+        const unsigned int t2 = __reduce_add_sync(0xffffffffu, s_cnt[32 + lane]);
+        const unsigned int t3 = __reduce_add_sync(0xffffffffu, s_cnt[64 + lane]);
+        X = t3 >= K ? x3 : (t2 >= K ? x2 : (t1 >= K ? x1 : X));
+        __syncthreads();
     }
+    // keys strictly above X: all taken; of the keys equal to X, the first ones
+    unsigned int above = 0u, n_eq = 0u;
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+        above += key[i] > X;
+        n_eq += beg + i < M && key[i] == X;
+    }
+    above = __reduce_add_sync(0xffffffffu, above);
+    if (lane == 0) s_cnt[warp] = above;
     __syncthreads();
+    const int need_eq = int(K - __reduce_add_sync(0xffffffffu, s_cnt[lane]));
 
-    // 1. radix select of the K-th largest relevance (bits of a float >= 0)
-    for (int shift = 24; shift >= 0; shift -= 8) {
-        for (int i = threadIdx.x; i < 256; i += blockDim.x) s_hist[i] = 0u;
-        __syncthreads();
-        const unsigned int prefix = s_prefix;
-        const unsigned int hi_mask = shift == 24 ? 0u : (0xffffffffu << (shift + 8));
-        for (int m = threadIdx.x; m < M; m += blockDim.x) {
-            const unsigned int key = __float_as_uint(rel[m]);
-            if ((key & hi_mask) == prefix) atomicAdd(&s_hist[(key >> shift) & 255u], 1u);
-        }
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            unsigned int left = s_kleft, acc = 0u;
-            int bin = 255;
-            for (; bin > 0; --bin) {
-                if (acc + s_hist[bin] >= left) break;
-                acc += s_hist[bin];
-            }
-            s_kleft = left - acc;
-            s_prefix = prefix | (unsigned(bin) << shift);
-        }
-        __syncthreads();
-    }
-    const unsigned int thr = s_prefix;   // the K-th largest key
-    const int need_eq = int(s_kleft);    // how many keys equal to thr are taken
-
-    // 2. ordered compaction: all keys > thr, then the first need_eq keys == thr
-    const int per = (M + blockDim.x - 1) / blockDim.x;
-    const int beg = threadIdx.x * per;
-    const int end = min(M, beg + per);
-    int n_eq = 0;
-    for (int m = beg; m < end; ++m) n_eq += __float_as_uint(rel[m]) == thr;
+    // 2. ordered compaction: all keys > X, then the first need_eq keys == X
     int eq_before = 0;
-    block_scan(n_eq, s_warp, &eq_before);
+    block_scan(int(n_eq), s_warp, &eq_before);
     int n_sel = 0;
     {
         int e = eq_before;
-        for (int m = beg; m < end; ++m) {
-            const unsigned int key = __float_as_uint(rel[m]);
-            if (key > thr) ++n_sel;
-            else if (key == thr) { if (e < need_eq) ++n_sel; ++e; }
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            const bool eq = beg + i < M && key[i] == X;
+            n_sel += key[i] > X || (eq && e < need_eq);
+            e += eq;
         }
     }
     int sel_before = 0;
@@ -323,11 +568,11 @@ __global__ void __launch_bounds__(1024) ads_select_kernel(const __grid_constant_
     int32_t* out = a.idx_out + int64_t(b) * a.k;
     {
         int e = eq_before, o = sel_before;
-        for (int m = beg; m < end; ++m) {
-            const unsigned int key = __float_as_uint(rel[m]);
-            bool take = key > thr;
-            if (key == thr) { take = e < need_eq; ++e; }
-            if (take) out[o++] = m;
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            const bool eq = beg + i < M && key[i] == X;
+            if (key[i] > X || (eq && e < need_eq)) out[o++] = beg + i;
+            e += eq;
         }
     }
     if (threadIdx.x == 0) {
@@ -342,35 +587,77 @@ __global__ void __launch_bounds__(1024) ads_select_kernel(const __grid_constant_
 
 }  // namespace
 
-cudaError_t launch_select(const SelectArgs& a, int n_seqs, cudaStream_t stream) {
-    const int D = a.head_dim, P = D / 2;
-    const size_t smem1 = (size_t(a.n_q_heads) * (D + 4) + 2 * size_t(a.tok_tile) * (P + 4) +
-                          size_t(a.n_q_heads) * (a.tok_tile + 1)) * sizeof(float);
-    const dim3 g1(a.n_tiles, n_seqs, 1);
+size_t select_logits_smem(const SelectArgs& a) {
+    const int D = a.head_dim, P = D / 2, T = a.tok_tile;
+    return size_t(a.n_q_heads) * (D / 4 + 1) * 16 + 2 * size_t(T) * (P / 4 + 1) * 16 +
+           size_t(a.n_q_heads) * (T + 1) * 4 + size_t(T) * 3 * 4;
+}
+
+template <int L, int G>
+cudaError_t launch_logits_g(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream) {
+    const size_t smem = select_logits_smem(a);
+    cudaError_t e = cudaFuncSetAttribute(ads_logits_kernel<L, G>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ads_logits_kernel<L, G>, 256, smem);
+    if (e != cudaSuccess) return e;
+    const int64_t tiles = int64_t(n_seqs) * a.n_tiles;
+    const int64_t resident = int64_t(sms) * (per_sm > 0 ? per_sm : 1);
+    const unsigned grid = unsigned(tiles < resident ? tiles : resident);
+    ads_logits_kernel<L, G><<<grid, 256, smem, stream>>>(a);
+    return cudaGetLastError();
+}
+
+template <int L>
+cudaError_t launch_logits(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream) {
+    const int g = a.n_q_heads / a.n_kv_heads;
+    if (g == 1) return launch_logits_g<L, 1>(a, n_seqs, sms, stream);
+    if (g == 2) return launch_logits_g<L, 2>(a, n_seqs, sms, stream);
+    if (g == 4) return launch_logits_g<L, 4>(a, n_seqs, sms, stream);
+    return launch_logits_g<L, 8>(a, n_seqs, sms, stream);
+}
+
+template <int D>
+cudaError_t launch_logits_mma(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream) {
+    const size_t smem = size_t(a.n_kv_heads) * (D / 8) * 32 * 16 +
+                        size_t(a.n_q_heads) * (a.tok_tile + 1) * 4;
+    cudaError_t e = cudaFuncSetAttribute(ads_logits_mma_kernel<D>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ads_logits_mma_kernel<D>, 256, smem);
+    if (e != cudaSuccess) return e;
+    const int64_t tiles = int64_t(n_seqs) * a.n_tiles;
+    const int64_t resident = int64_t(sms) * (per_sm > 0 ? per_sm : 1);
+    ads_logits_mma_kernel<D><<<unsigned(tiles < resident ? tiles : resident), 256, smem, stream>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_select(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream) {
     ads_query_kernel<<<n_seqs, 256, 0, stream>>>(a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    if (D <= 64) {
-        e = cudaFuncSetAttribute(ads_logits_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem1));
-        if (e == cudaSuccess) ads_logits_kernel<4><<<g1, 256, smem1, stream>>>(a);
-    } else if (D <= 128) {
-        e = cudaFuncSetAttribute(ads_logits_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem1));
-        if (e == cudaSuccess) ads_logits_kernel<8><<<g1, 256, smem1, stream>>>(a);
+    if (a.head_dim == 128 && a.tok_tile == 64) {
+        e = launch_logits_mma<128>(a, n_seqs, sms, stream);
+    } else if (a.head_dim == 64 && a.tok_tile == 64) {
+        e = launch_logits_mma<64>(a, n_seqs, sms, stream);
     } else {
-        e = cudaFuncSetAttribute(ads_logits_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem1));
-        if (e == cudaSuccess) ads_logits_kernel<16><<<g1, 256, smem1, stream>>>(a);
+        const int L = a.head_dim <= 64 ? 4 : (a.head_dim <= 128 ? 8 : 16);
+        e = L == 4 ? launch_logits<4>(a, n_seqs, sms, stream)
+                   : (L == 8 ? launch_logits<8>(a, n_seqs, sms, stream)
+                             : launch_logits<16>(a, n_seqs, sms, stream));
     }
     if (e != cudaSuccess) return e;
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
     ads_norm_kernel<<<dim3(a.n_q_heads, n_seqs, 1), 256, 0, stream>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     ads_relevance_kernel<<<dim3((a.n_tokens + 255) / 256, n_seqs, 1), 256, 0, stream>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    const size_t smem2 = size_t(a.n_tokens) * sizeof(float);
-    e = cudaFuncSetAttribute(ads_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             int(smem2));
-    if (e != cudaSuccess) return e;
-    ads_select_kernel<<<n_seqs, 1024, smem2, stream>>>(a);
+    const int M = a.n_tokens;
+    if (M <= 4096) ads_select_kernel<4><<<n_seqs, 1024, 0, stream>>>(a);
+    else if (M <= 8192) ads_select_kernel<8><<<n_seqs, 1024, 0, stream>>>(a);
+    else if (M <= 16384) ads_select_kernel<16><<<n_seqs, 1024, 0, stream>>>(a);
+    else ads_select_kernel<32><<<n_seqs, 1024, 0, stream>>>(a);
     return cudaGetLastError();
 }
 

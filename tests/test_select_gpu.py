@@ -14,7 +14,7 @@ import pytest
 import torch
 
 from oracle import prcr_oracle as O
-from workloads import get, make_batch
+from workloads import Workload, get, make_batch
 
 pytestmark = pytest.mark.gpu
 
@@ -42,10 +42,24 @@ def _topk_by(values, k):
     return np.sort(order[:k])
 
 
+# odd shapes: head_dim 48 (3 of 4 lanes per row active), 3 KV heads with a
+# GQA group of 3, two grids per sequence; head_dim 256 with a group of 2;
+# token counts that leave a ragged last tile
+SHAPES = {
+    "sel-odd": Workload(name="sel-odd", n_layers=2, n_kv_heads=3, head_dim=48, sections=(8, 8, 8),
+                        n_seqs=3, grids=((3, 5, 5), (1, 4, 4)), selection="random",
+                        cache="contiguous", cur_pos=("uniform", 100, 4000), extra=(0, 3, 0, 37)),
+    "sel-d256": Workload(name="sel-d256", n_layers=1, n_kv_heads=2, head_dim=256,
+                         sections=(40, 44, 44), n_seqs=2, grids=((2, 10, 13),), selection="random",
+                         cache="contiguous", cur_pos=("uniform", 500, 900), extra=(1, 2, 1, 40)),
+}
+
+
 @pytest.mark.parametrize("name,Hq,k,layer", [("qwen25vl-7b", 28, 64, 5), ("qwen3vl-8b", 32, 300, 35),
-                                             ("tiny", 2, 16, 1)])
+                                             ("tiny", 2, 16, 1), ("qwen2vl-2b", 4, 100, 20),
+                                             ("sel-odd", 9, 20, 1), ("sel-d256", 4, 30, 0)])
 def test_select_parity(name, Hq, k, layer):
-    wl = get(name)
+    wl = SHAPES.get(name) or get(name)
     batch = make_batch(wl, device=DEV)
     B, M, D = wl.n_seqs, wl.n_tokens, wl.head_dim
     g = torch.Generator(device=DEV)
