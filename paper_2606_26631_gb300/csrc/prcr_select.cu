@@ -288,9 +288,9 @@ __device__ __forceinline__ void split_tf32(float x, uint32_t& hi, uint32_t& lo) 
 // contiguous runs and rotates them itself with its own cos/sin, computed once
 // per octet and reused for every KV head. Queries and rotated keys are split
 // into tf32 head + remainder and three products are summed (head x head,
-// head x remainder, remainder x head; float32 accumulate), which keeps the
-// logits at float32-level accuracy over float32's range. The accumulator of
-// lane (g, t) holds head g at tokens 2t, 2t+1 of the octet.
+// head x remainder, remainder x head; float32 accumulate): each product
+// keeps ~19 significant bits (float32-level logits) over float32's range.
+// The accumulator of lane (g, t) holds head g at tokens 2t, 2t+1 of the octet.
 template <int D>
 __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_constant__ SelectArgs a) {
     constexpr int P = D / 2, PL = P / 4, T = 64;
@@ -377,9 +377,12 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
                 const float y = (ks & 1) ? hi_f32(yw[ks >> 1]) : lo_f32(yw[ks >> 1]);
                 const float kx = fmaf(x, cs[ks], -y * sn[ks]);
                 const float ky = fmaf(y, cs[ks], x * sn[ks]);
-                uint32_t bxh, bxl, byh, byl;
-                split_tf32(kx, bxh, bxl);
-                split_tf32(ky, byh, byl);
+                // keys: tf32 head by truncation (one bit operation), exact
+                // float32 remainder < 2^-10 |k|, truncated in turn by the MMA
+                const uint32_t bxh = __float_as_uint(kx) & 0xffffe000u;
+                const uint32_t byh = __float_as_uint(ky) & 0xffffe000u;
+                const uint32_t bxl = __float_as_uint(kx - __uint_as_float(bxh));
+                const uint32_t byl = __float_as_uint(ky - __uint_as_float(byh));
                 const uint4 f = qa[ks * 32];
                 mma_1688_tf32(c, f.x, f.z, bxh, byh);
                 mma_1688_tf32(c, f.y, f.w, bxh, byh);
