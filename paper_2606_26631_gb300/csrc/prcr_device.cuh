@@ -19,6 +19,10 @@ __device__ __forceinline__ uint4 ld_stream(const uint16_t* p) {
     return r;
 }
 
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
 __device__ __forceinline__ void st_row(uint16_t* p, const uint4& v) {
     asm volatile("st.global.v4.u32 [%0], {%1, %2, %3, %4};"
                  :

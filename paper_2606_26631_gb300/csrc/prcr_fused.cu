@@ -27,6 +27,20 @@ __global__ void __launch_bounds__(512) fused_kernel(const __grid_constant__ Fuse
     __shared__ int s_bad;
     const bool lead = blockIdx.x == 0 && blockIdx.y == 0;
 
+    // 0. this thread's token index and the per-sequence inputs are requested
+    // before the offsets are checked, so that their latencies overlap
+    const int T = rb.tok_per_cta;
+    const int64_t tok0 = int64_t(blockIdx.x) * T;
+    const int lanes = rb.lanes;
+    const int my_t = threadIdx.x / lanes;
+    const int64_t my_j = tok0 + my_t;
+    const bool my_tok = my_t < T && my_j < a.total_k;
+    const int my_m = my_tok ? a.idx[my_j] : -1;
+    if (threadIdx.x < a.n_seqs) {
+        prefetch_l2(a.cache_len_in + threadIdx.x);
+        prefetch_l2(a.p_txt + threadIdx.x);
+    }
+
     // 1. the offsets: monotone, spanning [0, total_k) and [0, n_revisits)
     if (threadIdx.x == 0) s_bad = 0;
     __syncthreads();
@@ -48,6 +62,37 @@ __global__ void __launch_bounds__(512) fused_kernel(const __grid_constant__ Fuse
         if (lead && threadIdx.x == 0) atomicOr(a.status, PRCR_ST_CSR);
         return;
     }
+    // 1b. with the offsets checked (and in L1): the token's revisit and
+    // sequence, then its coordinates and its first layer's rows are
+    // prefetched while the revisit ranges are reduced
+    if (my_tok && my_m >= 0 && my_m < a.n_tokens) {
+        int r0 = 0, r1 = a.n_revisits;  // last revisit starting at or before my_j
+        while (r1 - r0 > 1) {
+            const int mid = (r0 + r1) >> 1;
+            if (a.rev_tok_off[mid] <= my_j) r0 = mid; else r1 = mid;
+        }
+        int s0 = 0, s1 = a.n_seqs;  // last sequence whose first revisit is at or before r0
+        while (s1 - s0 > 1) {
+            const int mid = (s0 + s1) >> 1;
+            if (a.seq_rev_off[mid] <= r0) s0 = mid; else s1 = mid;
+        }
+        const int lane = threadIdx.x - my_t * lanes;
+        if (lane == 0) prefetch_l2(a.coords + int64_t(s0) * a.coord_seq_stride + 3 * int64_t(my_m));
+        if (lane == 1 && a.cache_kind == PRCR_CACHE_PAGED) {
+            // the block-table entry of the token's slot (as token_plan finds it)
+            const int64_t slot = int64_t(a.cache_len_in[s0]) + (my_j - a.rev_tok_off[a.seq_rev_off[s0]]);
+            if (slot >= 0 && slot < int64_t(a.bt_stride) * a.block_size)
+                prefetch_l2(a.block_table + int64_t(s0) * a.bt_stride + slot / a.block_size);
+        }
+        const int vph = rb.head_dim >> 4;
+        const int64_t row = int64_t(s0) * a.store_seq_stride + int64_t(my_m) * a.store_token_stride +
+                            int64_t(blockIdx.y) * rb.layers_per_cta * rb.store_layer_stride +
+                            int64_t(lane / vph) * rb.head_dim + (lane % vph) * 8;
+        prefetch_l2(rb.store_k + row);
+        prefetch_l2(rb.store_k + row + (rb.head_dim >> 1));
+        prefetch_l2(rb.store_v + row);
+        prefetch_l2(rb.store_v + row + (rb.head_dim >> 1));
+    }
     uint32_t err = 0;
     if (lead) {
         for (int b = threadIdx.x; b < a.n_seqs; b += blockDim.x) {
@@ -61,8 +106,6 @@ __global__ void __launch_bounds__(512) fused_kernel(const __grid_constant__ Fuse
     }
 
     // 2. plan of this CTA's tokens [tok0, tok1)
-    const int T = rb.tok_per_cta;
-    const int64_t tok0 = int64_t(blockIdx.x) * T;
     const int64_t tok1 = min(tok0 + T, a.total_k);
     int ra = 0, hi = a.n_revisits;  // last revisit starting at or before tok0
     while (hi - ra > 1) {
@@ -142,7 +185,6 @@ __global__ void __launch_bounds__(512) fused_kernel(const __grid_constant__ Fuse
     }
     __syncthreads();
 
-    const int lanes = rb.lanes;
     const int t = threadIdx.x / lanes;
     const int lane = threadIdx.x - t * lanes;
     if (t >= T || tok0 + t >= tok1) return;
