@@ -21,7 +21,7 @@
 
 #include <cuda_bf16.h>
 
-#include "prcr_internal.h"
+#include "prcr_device.cuh"
 
 namespace prcr {
 namespace {
@@ -29,8 +29,6 @@ namespace {
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kDecodeThreads = 128;
 
-__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
 
 // EPL consecutive bf16 of a row as EPL / 2 packed words.
 template <int EPL>
@@ -176,8 +174,8 @@ __global__ void __launch_bounds__(kDecodeThreads, 3) decode_kernel(const __grid_
                     float d = 0.0f;
 #pragma unroll
                     for (int w = 0; w < EPL / 2; ++w) {
-                        d = fmaf(qf[h][2 * w], bf16_lo(kw[si][w]), d);
-                        d = fmaf(qf[h][2 * w + 1], bf16_hi(kw[si][w]), d);
+                        d = fmaf(qf[h][2 * w], lo_f32(kw[si][w]), d);
+                        d = fmaf(qf[h][2 * w + 1], hi_f32(kw[si][w]), d);
                     }
                     val[h * S + si] = d;
                 }
@@ -230,8 +228,8 @@ __global__ void __launch_bounds__(kDecodeThreads, 3) decode_kernel(const __grid_
                     const float pw = __shfl_sync(kFull, pl, h * S + si);
 #pragma unroll
                     for (int w = 0; w < EPL / 2; ++w) {
-                        acc[h][2 * w] = fmaf(pw, bf16_lo(vw[si][w]), acc[h][2 * w]);
-                        acc[h][2 * w + 1] = fmaf(pw, bf16_hi(vw[si][w]), acc[h][2 * w + 1]);
+                        acc[h][2 * w] = fmaf(pw, lo_f32(vw[si][w]), acc[h][2 * w]);
+                        acc[h][2 * w + 1] = fmaf(pw, hi_f32(vw[si][w]), acc[h][2 * w + 1]);
                     }
                 }
         }
@@ -279,26 +277,6 @@ __global__ void __launch_bounds__(kDecodeThreads, 3) decode_kernel(const __grid_
 // float32 probabilities are each split into a bf16 head and a bf16 remainder
 // (two MMAs each): products stay exact and the result keeps ~16 bits per
 // operand, float32-accumulated. K and V are bf16 already and enter exactly.
-__device__ __forceinline__ void mma_bf16(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
-                                         uint32_t a3, uint32_t b0, uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-        "{%8,%9}, {%0,%1,%2,%3};"
-        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-
-__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
-    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<const uint32_t*>(&v);
-}
-
-// (head, remainder) bf16 pairs of two floats
-__device__ __forceinline__ void split2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
-    hi = pack2(x0, x1);
-    lo = pack2(x0 - bf16_lo(hi), x1 - bf16_hi(hi));
-}
-
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
                  "r"(src_bytes)
@@ -368,8 +346,8 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
             for (int j = 0; j < KS; ++j) {
                 const float x0 = hv ? qr[4 * j] : 0.0f, x1 = hv ? qr[4 * j + 1] : 0.0f;
                 const float x2 = hv ? qr[4 * j + 2] : 0.0f, x3 = hv ? qr[4 * j + 3] : 0.0f;
-                split2(x0, x1, qh[j][0], ql[j][0]);
-                split2(x2, x3, qh[j][1], ql[j][1]);
+                split_bf16x2(x0, x1, qh[j][0], ql[j][0]);
+                split_bf16x2(x2, x3, qh[j][1], ql[j][1]);
             }
         }
         float o[KS][4];
@@ -440,8 +418,8 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
                     const uint4& w = kn[nt][j >> 1];
                     const uint32_t b0 = (j & 1) ? w.z : w.x;
                     const uint32_t b1 = (j & 1) ? w.w : w.y;
-                    mma_bf16(sc[nt], qh[j][0], 0u, qh[j][1], 0u, b0, b1);
-                    mma_bf16(sc[nt], ql[j][0], 0u, ql[j][1], 0u, b0, b1);
+                    mma_16816(sc[nt], qh[j][0], 0u, qh[j][1], 0u, b0, b1);
+                    mma_16816(sc[nt], ql[j][0], 0u, ql[j][1], 0u, b0, b1);
                 }
             }
             // the next tile's K and V are in flight during the softmax and P V
@@ -478,8 +456,8 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
                 o[mt][0] *= a0; o[mt][1] *= a1; o[mt][2] *= a0; o[mt][3] *= a1;
             }
             uint32_t pb0h, pb0l, pb1h, pb1l;
-            split2(v[0], v[1], pb0h, pb0l);
-            split2(v[2], v[3], pb1h, pb1l);
+            split_bf16x2(v[0], v[1], pb0h, pb0l);
+            split_bf16x2(v[2], v[3], pb1h, pb1l);
 
             // O^T += V^T P^T
             if (more) asm volatile("cp.async.wait_group 1;" ::: "memory");
@@ -494,8 +472,8 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
                 asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
                              : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
                              : "r"(addr));
-                mma_bf16(o[mt], r0, r1, r2, r3, pb0h, pb1h);
-                mma_bf16(o[mt], r0, r1, r2, r3, pb0l, pb1l);
+                mma_16816(o[mt], r0, r1, r2, r3, pb0h, pb1h);
+                mma_16816(o[mt], r0, r1, r2, r3, pb0l, pb1l);
             }
             __syncwarp();
         }
