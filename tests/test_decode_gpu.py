@@ -151,3 +151,40 @@ def test_decode_sees_only_relative_positions():
         outs.append(out.cpu().numpy())
     vmax = float(torch.abs(batch.store_v.float()).max())
     assert np.abs(outs[0] - outs[1]).max() / vmax <= 2e-3
+
+
+def _layer_rows(inp, b, l, n):
+    """[n, H, D] value arrays of slots 0..n-1 of sequence b at layer l (paged)."""
+    s = torch.arange(n, device=inp["cache_k"].device)
+    bs = inp["cache_k"].shape[2]
+    blk = inp["block_table"][b][s // bs].long()
+    off = s % bs
+    return _f64(inp["cache_k"][l, blk, off]), _f64(inp["cache_v"][l, blk, off])
+
+
+@pytest.mark.slow
+def test_decode_full_size_sampled():
+    """The decode configuration bench.py times (qwen3vl-8b shape: 16 sequences
+    of up to 8192 slots, 36 layers, 8 KV heads, 32 query heads, paged, the same
+    seed, so the same chunk split and merge launch); sampled (sequence, layer)
+    pairs, every query head, against the oracle."""
+    import paper_2606_26631_gb300 as prcr
+    wl = get("qwen3vl-8b")
+    B, nL, H, D = wl.n_seqs, wl.n_layers, wl.n_kv_heads, wl.head_dim
+    Hq, max_len = 4 * H, 8192
+    inp = make_decode_inputs(B, nL, H, Hq, D, max_len, True, device=DEV, seed=1)
+    cfg = prcr.rope_cfg(nL, H, D, wl.sections, wl.theta)
+    cd = prcr.cache_paged(inp["cache_k"], inp["cache_v"], inp["block_table"])
+    out, st = _run_decode(cfg, cd, inp["q"], inp["q_pos"], inp["seq_len"], max_len)
+    assert st == 0
+    got = out.cpu().numpy()
+    qv = _f64(inp["q"])
+    for b in (0, B // 2, B - 1):
+        n = int(inp["seq_len"][b])
+        for l in (0, nL // 2, nL - 1):
+            K, V = _layer_rows(inp, b, l, n)
+            ref = O.decode_attention(qv[b, l], int(inp["q_pos"][b]), K, V, D, wl.sections, wl.theta)
+            err = np.abs(got[b, l] - ref).max() / np.abs(V).max()
+            assert err <= 1e-4, (b, l, n, err)
+    del inp
+    torch.cuda.empty_cache()

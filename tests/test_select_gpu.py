@@ -131,3 +131,33 @@ def test_select_feeds_rebind_inject():
     assert torch.equal(rv.next_pos, batch.p_txt + 1)
     written = int((ck.view(torch.int16) != -1).sum().item())
     assert written == B * k * wl.n_layers * wl.n_kv_heads * wl.head_dim
+
+
+@pytest.mark.slow
+def test_select_full_size_sampled():
+    """The selection configuration bench.py times on the stress shape (32
+    sequences x 16,384 tokens, 32 query heads, k = 4096, last layer); sampled
+    sequences checked like test_select_parity."""
+    wl = get("stress")
+    batch = make_batch(wl, device=DEV)
+    B, M, H, D = wl.n_seqs, wl.n_tokens, wl.n_kv_heads, wl.head_dim
+    Hq, k, layer = 4 * H, batch.total_k // B, wl.n_layers - 1
+    q = torch.randn((B, Hq, D), device=DEV, generator=torch.Generator(device=DEV).manual_seed(3)
+                    ).to(torch.bfloat16)
+    idx, sro, rto, score = _select(batch, layer, Hq, k, q, batch.p_txt)
+    assert np.array_equal(sro, np.arange(B + 1))
+    assert np.array_equal(rto, k * np.arange(B + 1))
+    qv = O.bf16_bits_to_f64(q.view(torch.int16).cpu().numpy())
+    coords = batch.coords.cpu().numpy()
+    for b in (0, B // 2, B - 1):
+        k_raw = batch.store_k[b, layer].view(torch.int16).cpu().numpy()
+        ref = O.ads_relevance(qv[b], int(batch.p_txt[b]), k_raw, coords[b], D, wl.sections, wl.theta)
+        assert (np.abs(score[b] - ref) / ref).max() <= 1e-4
+        sel = idx[b]
+        assert np.array_equal(sel, _topk_by(score[b].astype(np.float64), k))
+        tol = 2 * np.abs(score[b] - ref).max() + 1e-12
+        chosen = np.zeros(M, dtype=bool)
+        chosen[sel] = True
+        assert ref[chosen].min() >= ref[~chosen].max() - tol
+    del batch
+    torch.cuda.empty_cache()
