@@ -125,3 +125,53 @@ def test_prefill_capture_capacity_error():
     for c in (ck, cv):
         n = int((c.view(torch.int16) == CANARY_BITS).sum().item())
         assert n == c.numel() - fit * 2 * 128
+
+
+@pytest.mark.slow
+def test_prefill_capture_full_size_sampled():
+    """The capture configuration bench.py times (qwen3vl-8b: 16 sequences x
+    8192 tokens x 36 layers, one call per sequence over all layers into a
+    shuffled paged cache from slot 0); store bit-exact everywhere, cache rows
+    on sampled sequences, tokens and layers against the oracle."""
+    import paper_2606_26631_gb300 as prcr
+    import parity_util as pu
+    wl = get("qwen3vl-8b")
+    src = make_batch(wl, device=DEV)
+    B, nL, M, H, D = wl.n_seqs, wl.n_layers, wl.n_tokens, wl.n_kv_heads, wl.head_dim
+    store_k = torch.empty_like(src.store_k)
+    store_v = torch.empty_like(src.store_v)
+    coords = torch.empty_like(src.coords)
+    bs = 16
+    nblk = (M + bs - 1) // bs
+    perm = torch.randperm(B * nblk, device=DEV, generator=torch.Generator(device=DEV).manual_seed(2))
+    bt = perm.view(B, nblk).to(torch.int32).contiguous()
+    ck = torch.empty((nL, B * nblk, bs, H, D), dtype=torch.bfloat16, device=DEV)
+    cv = torch.empty_like(ck)
+    cfg = prcr.rope_cfg(nL, H, D, wl.sections, wl.theta)
+    sd = prcr.store_desc(store_k, store_v, coords)
+    cd = prcr.cache_paged(ck, cv, bt)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    for b in range(B):
+        prcr.prefill_capture(cfg, sd, cd, b, 0, 0, 0, src.store_k[b], src.store_v[b], src.coords[b],
+                             status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    assert torch.equal(store_k.view(torch.int16), src.store_k.view(torch.int16))
+    assert torch.equal(store_v.view(torch.int16), src.store_v.view(torch.int16))
+    assert torch.equal(coords, src.coords)
+    rng = np.random.default_rng(9)
+    layers = [0, nL // 2, nL - 1]
+    for b in (0, B // 2, B - 1):
+        toks = np.sort(rng.choice(M, size=512, replace=False))
+        t_dev = torch.as_tensor(toks, device=DEV)
+        k_raw = pu.bits(src.store_k[b][:, t_dev].transpose(0, 1)[:, layers])  # [n, L, H, D]
+        v_raw = pu.bits(src.store_v[b][:, t_dev].transpose(0, 1)[:, layers])
+        crd = src.coords[b].cpu().numpy()[toks]
+        _, _, k_want, v_want = O.prefill_capture(k_raw, v_raw, crd, D, wl.sections, wl.theta)
+        k_got = pu.bits(_rows(ck, bt, b, toks, layers, True))
+        v_got = pu.bits(_rows(cv, bt, b, toks, layers, True))
+        assert np.array_equal(v_got, v_want)
+        e = pu.k_error(k_got, k_want, k_raw)
+        assert e["max_err"] <= pu.K_TOL, e
+    del src, store_k, store_v, ck, cv
+    torch.cuda.empty_cache()
