@@ -645,8 +645,6 @@ int prcr_select_topk(const prcr_rope_cfg* cfg, const prcr_store_desc* store, int
         a.norm = reinterpret_cast<float*>(w);
         w += align256(size_t(8 * Bn * Hn));
         a.rel = reinterpret_cast<float*>(w);
-        w += align256(size_t(4 * Bn * M));
-        a.qrot = reinterpret_cast<float*>(w);
     }
     a.score_out = score_out;
     a.idx_out = idx_out;

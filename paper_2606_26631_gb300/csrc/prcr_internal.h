@@ -222,8 +222,7 @@ constexpr int kSelectTokTile = 16;   // smallest tile of the logits kernel (size
 inline size_t select_workspace_bytes(int64_t B, int64_t Hq, int64_t M) {
     const int64_t tiles = (M + kSelectTokTile - 1) / kSelectTokTile;
     return align256(size_t(4 * B * Hq * M)) + align256(size_t(8 * B * Hq * tiles)) +
-           align256(size_t(8 * B * Hq)) + align256(size_t(4 * B * M)) +
-           align256(size_t(4 * B * Hq) * kMaxPairs * 2);
+           align256(size_t(8 * B * Hq)) + align256(size_t(4 * B * M));
 }
 
 struct SelectArgs {
@@ -250,7 +249,6 @@ struct SelectArgs {
     float* tile_stats;          // workspace [B][n_q_heads][n_tiles][2] (max, sum of exp)
     float* norm;                // workspace [B][n_q_heads][2] (max, 1 / (sum * n_q_heads))
     float* rel;                 // workspace [B][n_tokens] relevance
-    float* qrot;                // workspace [B][n_q_heads][D] rotated, scaled queries
     int32_t n_seqs;
     int32_t n_tiles;            // token tiles of the logits kernel per sequence
     int32_t tok_tile;           // tokens per tile

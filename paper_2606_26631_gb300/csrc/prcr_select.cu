@@ -10,16 +10,20 @@
 // written in ascending token order, one revisit per sequence, as the offsets
 // and indices prcr_rebind_inject takes.
 //
-// Kernel 0 rotates each sequence's trigger queries once (pre-scaled by
-// 1/sqrt(D)). Kernel 1 (logits, persistent) forms every (token, query head)
-// logit from the raw key rotated on the fly at the token's own coordinates,
-// and each token tile's per-head softmax statistics (max, sum of exp).
-// Kernel 2 (norm) merges the tiles' statistics into each head's normaliser;
-// kernel 3 (relevance) averages every token's per-head softmax weight;
-// kernel 4 (select), one CTA per sequence, finds the K-th largest relevance
-// by counting against thresholds two bits at a time on the float bits
-// (relevance >= 0, so bit order is value order) and compacts the selection
-// in index order with block-wide scans.
+// A rotation preserves dot products and composes by adding angles, so
+// RoPE(q, (p, p, p)) . RoPE(k, c) = q . R(c - p) k: pair i of the raw key is
+// turned by theta_i (c_axis(i) - p) and dotted with the raw query, and the
+// 1/sqrt(D) scale is applied to the dot product. The raw bf16 query is then
+// exact in any operand format, and nothing is computed per query.
+// Kernel 1 (logits, persistent) forms every (token, query head) logit that
+// way from the raw key rotated on the fly, and each token tile's per-head
+// softmax statistics (max, sum of exp). Kernel 2 (norm) merges the tiles'
+// statistics into each head's normaliser; kernel 3 (relevance) averages
+// every token's per-head softmax weight; kernel 4 (select), one CTA per
+// sequence, finds the K-th largest relevance by counting against thresholds
+// two bits at a time on the float bits (relevance >= 0, so bit order is
+// value order) and compacts the selection in index order with block-wide
+// scans.
 #include <cmath>
 
 #include "prcr_device.cuh"
@@ -27,32 +31,12 @@
 namespace prcr {
 namespace {
 
-// The trigger queries of each sequence, rotated at (p, p, p) (pair i turns by
-// p * inv_freq_i for every head) and scaled by 1/sqrt(D), once per sequence.
-__global__ void __launch_bounds__(256) ads_query_kernel(const __grid_constant__ SelectArgs a) {
-    __shared__ float s_c[kMaxPairs], s_s[kMaxPairs];
-    const int b = blockIdx.x;
-    const int D = a.head_dim, P = D >> 1, Hq = a.n_q_heads;
-    const int64_t p = a.q_pos[b];
-    for (int i = threadIdx.x; i < P; i += blockDim.x) sincos_turns(double(p), a.turn_freq[i], &s_s[i], &s_c[i]);
-    __syncthreads();
-    const uint16_t* qb = a.q + int64_t(b) * Hq * D;
-    float* qo = a.qrot + int64_t(b) * Hq * D;
-    for (int e = threadIdx.x; e < Hq * P; e += blockDim.x) {
-        const int hq = e / P, i = e - (e / P) * P;
-        const float x = __uint_as_float(uint32_t(qb[hq * D + i]) << 16);
-        const float y = __uint_as_float(uint32_t(qb[hq * D + i + P]) << 16);
-        qo[hq * D + i] = fmaf(x, s_c[i], -y * s_s[i]) * a.scale;
-        qo[hq * D + i + P] = fmaf(y, s_c[i], x * s_s[i]) * a.scale;
-    }
-}
-
-// Rotation of an integer coordinate: the turn fraction c * rate mod 1 in
-// 0.32 fixed point is bits 32..63 of the 64-bit product c * rate (rate in
+// Rotation of an integer position offset: the turn fraction c * rate mod 1
+// in 0.32 fixed point is bits 32..63 of the 64-bit product c * rate (rate in
 // 0.64 fixed point; the product's wrap mod 2^64 keeps those bits exact for
-// any int32 c), then one sin/cos evaluation on [-pi, pi).
-__device__ __forceinline__ void sincos_coord(int c, uint64_t turn_freq, float* s, float* co) {
-    const uint64_t prod = static_cast<uint64_t>(static_cast<int64_t>(c)) * turn_freq;
+// any int64 c), then one sin/cos evaluation on [-pi, pi).
+__device__ __forceinline__ void sincos_coord(int64_t c, uint64_t turn_freq, float* s, float* co) {
+    const uint64_t prod = static_cast<uint64_t>(c) * turn_freq;
     const int frac = static_cast<int>(static_cast<uint32_t>(prod >> 32));
     __sincosf(float(frac) * 1.4629180792671596e-9f, s, co);  // 2 pi / 2^32
 }
@@ -102,15 +86,18 @@ __global__ void __launch_bounds__(256, 3) ads_logits_kernel(const __grid_constan
     for (int64_t tile = t_beg; tile < t_end; ++tile) {
         const int b = int(tile / a.n_tiles), j = int(tile % a.n_tiles);
         const int m0 = j * T, nt = min(T, M - m0);
-        if (b != cur_b) {
-            const float4* src = reinterpret_cast<const float4*>(a.qrot + int64_t(b) * Hq * D);
+        if (b != cur_b) {  // the sequence's raw queries as float32 (4-byte loads)
+            const uint32_t* src = reinterpret_cast<const uint32_t*>(a.q + int64_t(b) * Hq * D);
             const int nch = D / 4;
             for (int e = tid; e < Hq * nch; e += blockDim.x) {
                 const int hq = e / nch, c = e - hq * nch;
-                q_s[((hq % g) * H + hq / g) * qrow + swz(c)] = src[e];
+                const uint32_t w0 = src[2 * e], w1 = src[2 * e + 1];
+                q_s[((hq % g) * H + hq / g) * qrow + swz(c)] =
+                    make_float4(lo_f32(w0), hi_f32(w0), lo_f32(w1), hi_f32(w1));
             }
             cur_b = b;
         }
+        const int64_t p = a.q_pos[b];
         const int32_t* crd = a.coords + int64_t(b) * a.coord_seq_stride + 3 * int64_t(m0);
         for (int e = tid; e < 3 * nt; e += blockDim.x) crd_s[e] = crd[e];
         __syncthreads();
@@ -124,7 +111,7 @@ __global__ void __launch_bounds__(256, 3) ads_logits_kernel(const __grid_constan
             }
             const int ax = pair_axis(i, a.layout, a.sec_t, a.sec_h, a.sec_w);
             float sn, cn;
-            sincos_coord(crd_s[3 * t + ax], a.turn_freq[i], &sn, &cn);
+            sincos_coord(crd_s[3 * t + ax] - p, a.turn_freq[i], &sn, &cn);
             const int o = (t * crow + swz(i >> 2)) * 4 + (i & 3);
             cf[o] = cn;
             sf[o] = sn;
@@ -208,7 +195,7 @@ __global__ void __launch_bounds__(256, 3) ads_logits_kernel(const __grid_constan
                         s2a = __ffma2_rn(make_float2(qc.z, qc.w), ky[1], s2a);
                         s2a = __ffma2_rn(make_float2(qd.x, qd.y), ky[2], s2a);
                         s2a = __ffma2_rn(make_float2(qd.z, qd.w), ky[3], s2a);
-                        acc[h] = s2a.x + s2a.y;
+                        acc[h] = (s2a.x + s2a.y) * a.scale;
                     }
                 }
             }
@@ -268,28 +255,22 @@ __device__ __forceinline__ void mma_1688_tf32(float (&c)[4], uint32_t a0, uint32
         : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
 }
 
-// A float32 as tf32 head (round to nearest, ties away) and float32 remainder
-// (exact); the remainder enters the MMA truncated to tf32, so head +
-// remainder carries ~21 significant bits.
-__device__ __forceinline__ void split_tf32(float x, uint32_t& hi, uint32_t& lo) {
-    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(hi) : "f"(x));
-    lo = __float_as_uint(x - __uint_as_float(hi));
-}
-
 // Tensor-core logits (head_dim 64 and 128). Persistent over token tiles like
 // the kernel above; a tile is 64 tokens, one octet of 8 per warp, and a warp
 // takes its octet through all KV heads:
 //   S (16 rows = the group's query heads, rows >= g zero; 8 tokens)
-//     = Q (16 x D) K_rot^T (D x 8), D / 8 k-steps of mma.sync m16n8k8 (tf32).
+//     = Q (16 x D) K_rot^T (D x 8), D / 8 k-steps of mma.sync m16n8k8 (tf32),
+//   K_rot the keys turned by the offsets of their coordinates from p.
 // The dot product does not depend on the order of the dimensions, so k-step j
 // of lane group t (= lane & 3) takes pair t * P/4 + j: k-slot t holds its
 // first-half dimension and k-slot t + 4 its rotate-half partner. A lane then
 // owns P/4 whole pairs of its token (= lane >> 2), loads them as two
 // contiguous runs and rotates them itself with its own cos/sin, computed once
-// per octet and reused for every KV head. Queries and rotated keys are split
-// into tf32 head + remainder and three products are summed (head x head,
-// head x remainder, remainder x head; float32 accumulate): each product
-// keeps ~19 significant bits (float32-level logits) over float32's range.
+// per octet and reused for every KV head. The raw bf16 queries are exact
+// tf32 operands; each rotated key is split into a tf32 head (truncation) and
+// its float32 remainder (< 2^-10 of the value, itself truncated by the MMA),
+// and both products are summed (float32 accumulate): each keeps ~20
+// significant bits (float32-level logits) over float32's range.
 // The accumulator of lane (g, t) holds head g at tokens 2t, 2t+1 of the octet.
 template <int D>
 __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_constant__ SelectArgs a) {
@@ -297,7 +278,7 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
     constexpr int NW = PL / 8;  // 16-byte loads per half row per lane
     extern __shared__ __align__(16) float sm[];
     const int Hq = a.n_q_heads, H = a.n_kv_heads, g = Hq / H, M = a.n_tokens;
-    uint4* qa_s = reinterpret_cast<uint4*>(sm);                // [H][PL][32]: (a0 hi, a0 lo, a2 hi, a2 lo)
+    uint2* qa_s = reinterpret_cast<uint2*>(sm);                // [H][PL][32]: (a0, a2), raw queries
     float* lg_s = reinterpret_cast<float*>(qa_s + H * PL * 32);  // [Hq][T + 1]
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int gid = lane >> 2, tq = lane & 3;
@@ -314,16 +295,17 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
         const int b = int(tile / a.n_tiles), j = int(tile % a.n_tiles);
         const int m0 = j * T, nt = min(T, M - m0);
         if (b != cur_b) {
-            // the sequence's rotated queries as A fragments, split once
-            const float* qs = a.qrot + int64_t(b) * Hq * D;
+            // the sequence's raw queries as A fragments (a bf16 value is an
+            // exact tf32 operand)
+            const uint16_t* qs = a.q + int64_t(b) * Hq * D;
             for (int e = tid; e < H * PL * 32; e += blockDim.x) {
                 const int kh = e / (PL * 32), ks = (e / 32) % PL, ln = e & 31;
                 const int h = ln >> 2, tt = ln & 3;
-                uint4 f = make_uint4(0u, 0u, 0u, 0u);
+                uint2 f = make_uint2(0u, 0u);
                 if (h < g) {
-                    const float* qr = qs + (kh * g + h) * D + tt * PL + ks;
-                    split_tf32(qr[0], f.x, f.y);
-                    split_tf32(qr[P], f.z, f.w);
+                    const uint16_t* qr = qs + (kh * g + h) * D + tt * PL + ks;
+                    f.x = uint32_t(qr[0]) << 16;
+                    f.y = uint32_t(qr[P]) << 16;
                 }
                 qa_s[e] = f;
             }
@@ -337,8 +319,10 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
         const int m = m0 + (live ? to : 0);
         float cs[PL], sn[PL];
         {
+            // angles at the offsets from the trigger position
             const int32_t* crd = a.coords + int64_t(b) * a.coord_seq_stride + 3 * int64_t(m);
-            const int c0 = crd[0], c1 = crd[1], c2 = crd[2];
+            const int64_t p = a.q_pos[b];
+            const int64_t c0 = crd[0] - p, c1 = crd[1] - p, c2 = crd[2] - p;
 #pragma unroll
             for (int p = 0; p < PL; ++p) {
                 const uint32_t ax = (axes >> (2 * p)) & 3u;
@@ -369,7 +353,7 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
                 }
             }
             float c[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-            const uint4* qa = qa_s + kh * PL * 32 + lane;
+            const uint2* qa = qa_s + kh * PL * 32 + lane;
 #pragma unroll
             for (int ks = 0; ks < PL; ++ks) {
                 // pair ks of this lane: element ks of each half
@@ -383,15 +367,14 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
                 const uint32_t byh = __float_as_uint(ky) & 0xffffe000u;
                 const uint32_t bxl = __float_as_uint(kx - __uint_as_float(bxh));
                 const uint32_t byl = __float_as_uint(ky - __uint_as_float(byh));
-                const uint4 f = qa[ks * 32];
-                mma_1688_tf32(c, f.x, f.z, bxh, byh);
-                mma_1688_tf32(c, f.y, f.w, bxh, byh);
-                mma_1688_tf32(c, f.x, f.z, bxl, byl);
+                const uint2 f = qa[ks * 32];
+                mma_1688_tf32(c, f.x, f.y, bxh, byh);
+                mma_1688_tf32(c, f.x, f.y, bxl, byl);
             }
             if (gid < g) {  // (rows are T + 1 floats apart: 4-byte stores)
                 float* dst = lg_s + (kh * g + gid) * (T + 1) + 8 * warp + 2 * tq;
-                dst[0] = c[0];
-                dst[1] = c[1];
+                dst[0] = c[0] * a.scale;
+                dst[1] = c[1] * a.scale;
             }
         }
         __syncthreads();
@@ -623,7 +606,7 @@ cudaError_t launch_logits(const SelectArgs& a, int n_seqs, int sms, cudaStream_t
 
 template <int D>
 cudaError_t launch_logits_mma(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream) {
-    const size_t smem = size_t(a.n_kv_heads) * (D / 8) * 32 * 16 +
+    const size_t smem = size_t(a.n_kv_heads) * (D / 8) * 32 * 8 +
                         size_t(a.n_q_heads) * (a.tok_tile + 1) * 4;
     cudaError_t e = cudaFuncSetAttribute(ads_logits_mma_kernel<D>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
@@ -638,9 +621,7 @@ cudaError_t launch_logits_mma(const SelectArgs& a, int n_seqs, int sms, cudaStre
 }
 
 cudaError_t launch_select(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream) {
-    ads_query_kernel<<<n_seqs, 256, 0, stream>>>(a);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    cudaError_t e;
     if (a.head_dim == 128 && a.tok_tile == 64) {
         e = launch_logits_mma<128>(a, n_seqs, sms, stream);
     } else if (a.head_dim == 64 && a.tok_tile == 64) {
