@@ -543,6 +543,7 @@ int prcr_decode_attention(const prcr_rope_cfg* cfg, const prcr_cache_desc* cache
     DecodeArgs a = {};
     decode_split(int64_t(n_seqs) * cfg->n_layers, max_len, sm_count(dev),
                  int64_t(n_q_heads) * cfg->head_dim, &a.splits, &a.chunk);
+    if (n_seqs > 65535 || cfg->n_layers > 65535) return PRCR_EINVAL;  // grid z and y
     if (a.splits > 1) {
         const size_t need = size_t(n_seqs) * cfg->n_layers * n_q_heads * a.splits *
                             (cfg->head_dim + 2) * sizeof(float);
