@@ -276,7 +276,8 @@ def cpu_baseline(wl, n_layers: int, n_samples: int = 1, device="cpu"):
         total_t += oracle_step(batch)
         total_b += batch.algorithmic_bytes()
         del batch
-    return dict(value=total_b / total_t / 1e9, unit=UNIT, cores=1, kind="oracle",
+    return dict(value=total_b / total_t / 1e9, unit=UNIT, cores=1, host_cores=os.cpu_count(),
+                kind="oracle",
                 sample=(f"{n_samples} sequence(s) drawn like '{wl.name}' (seeds 0..{n_samples - 1}), "
                         f"all selected tokens x {n_layers} of {wl.n_layers} layers x "
                         f"{wl.n_kv_heads} KV heads, one sequence per oracle call "
@@ -308,8 +309,8 @@ def run_reference(args):
                 scaling="weak", vs_baseline=None, dtype="f64", data="synthetic",
                 config=dict(workload=wl.name, sample_per_step=describe_sample(wl, batch)),
                 impl="reference",
-                cpu_baseline=dict(kind="oracle", cores=1, value=value, unit=UNIT,
-                                  sample=describe_sample(wl, batch)),
+                cpu_baseline=dict(kind="oracle", cores=1, host_cores=os.cpu_count(), value=value,
+                                  unit=UNIT, sample=describe_sample(wl, batch)),
                 e2e=dict(value=value, unit=UNIT, h2d_bytes_per_step=0, d2h_bytes_per_step=0),
                 gpu_launches=0)
     print(json.dumps(line), flush=True)
