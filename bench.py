@@ -62,10 +62,12 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["prcr", "reference"], default="prcr")
     ap.add_argument("--workload", default="stress")
-    ap.add_argument("--path", choices=["revisit", "capture", "decode", "select"], default="revisit",
+    ap.add_argument("--path", choices=["revisit", "capture", "decode", "select", "pipeline"],
+                    default="revisit",
                     help="revisit: the rebind+inject step (default); capture: prefill capture; "
                          "decode: the first decode step over the active cache; select: the "
-                         "attention-driven selection of the revisited set")
+                         "attention-driven selection of the revisited set; pipeline: select, "
+                         "rebind+inject and the first decode step of one revisit, end to end")
     ap.add_argument("--seqs", type=int, default=0, help="capture/decode: sequences (0 = workload's)")
     ap.add_argument("--layers", type=int, default=0,
                     help="select: build the store with this many layers (0 = workload's); "
@@ -688,6 +690,95 @@ def run_select_path(args):
         **_launch_keys(launched, 5, args.steps), clocks=clk)), flush=True)
 
 
+def run_pipeline_path(args):
+    """One revisit end to end on the device, as a decoder would run it: the
+    revisited set chosen by attention at the last layer (k = the fewest tokens
+    a sequence of the workload revisits), its raw rows rebound and appended to the active
+    cache (whose context rows are data), and the first decode step over the
+    grown cache at the next text position."""
+    import torch
+    _, _, local = dist_env()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    from paper_2606_26631_gb300 import _build
+    if not _build.up_to_date():
+        _build.build()
+    import paper_2606_26631_gb300 as prcr
+    from workloads import get, make_batch
+    wl = get(args.workload)
+    batch = make_batch(wl, device=dev, context="random")
+    B, nL, M, H, D = wl.n_seqs, wl.n_layers, wl.n_tokens, wl.n_kv_heads, wl.head_dim
+    # k: the fewest tokens any sequence of the workload revisits, so that the
+    # appended span stays inside the cache rows the workload provides
+    sro_h, rto_h = batch.seq_rev_off.cpu().numpy(), batch.rev_tok_off.cpu().numpy()
+    Hq, k = 4 * H, max(1, int(min(rto_h[sro_h[b + 1]] - rto_h[sro_h[b]] for b in range(B))))
+    gen = torch.Generator(device=dev).manual_seed(5)
+    q_sel = torch.randn((B, Hq, D), device=dev, generator=gen).to(torch.bfloat16)
+    q_dec = torch.randn((B, nL, Hq, D), device=dev, generator=gen).to(torch.bfloat16)
+    cfg = prcr.rope_cfg(nL, H, D, wl.sections, wl.theta)
+    sd = prcr.store_desc(batch.store_k, batch.store_v, batch.coords)
+    idx = torch.empty(B * k, dtype=torch.int32, device=dev)
+    sro = torch.empty(B + 1, dtype=torch.int32, device=dev)
+    rto = torch.empty(B + 1, dtype=torch.int32, device=dev)
+    ws_sel = torch.empty(prcr.select_workspace_size(B, Hq, M), dtype=torch.uint8, device=dev)
+    rv = prcr.Revisit(cfg, batch.store_k, batch.store_v, batch.coords, batch.cache_k, batch.cache_v,
+                      batch.block_table, sro, rto, idx, batch.p_txt, batch.cache_len_in)
+    max_len = int(batch.cache_len_in.max().item()) + k
+    out = torch.empty(q_dec.shape, dtype=torch.float32, device=dev)
+    dstat = torch.zeros(1, dtype=torch.int32, device=dev)
+    nws = prcr.decode_workspace_size(cfg, B, Hq, max_len)
+    ws_dec = torch.empty(max(nws, 16), dtype=torch.uint8, device=dev)
+
+    def select():
+        prcr.select_topk(cfg, sd, nL - 1, q_sel, batch.p_txt, k, idx, sro, rto, ws_sel)
+
+    def decode():
+        prcr.decode_attention(cfg, rv.cache, q_dec, rv.next_pos, rv.cache_len_out, max_len, out,
+                              dstat, ws_dec)
+
+    def step():
+        select()
+        rv.run()
+        decode()
+
+    step()
+    torch.cuda.synchronize()
+    if rv.status_value() != 0 or int(dstat.item()) != 0:
+        raise RuntimeError(f"device status {rv.status_value():#x} / {int(dstat.item()):#x}")
+    launched = kernel_launches(step)
+    nbytes = batch.algorithmic_bytes()
+    flush = L2Flush(dev, args.flush, nbytes)
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    with Clocks(local) as clk:
+        for e in ev:
+            flush()
+            e[0].record(stream)
+            select()
+            e[1].record(stream)
+            rv.run()
+            e[2].record(stream)
+            decode()
+            e[3].record(stream)
+        torch.cuda.synchronize()
+    part = [[e[i].elapsed_time(e[i + 1]) * 1e3 for e in ev] for i in range(3)]
+    total = [e[0].elapsed_time(e[3]) * 1e3 for e in ev]
+    print(json.dumps(dict(
+        metric="revisit pipeline us per step (select + rebind/inject + first decode)",
+        value=statistics.mean(total), unit="us", n_gpus=1, steps=args.steps, warmup=args.warmup,
+        ms_per_step=statistics.mean(total) / 1e3, higher_is_better=False, scaling="weak",
+        vs_baseline=None, dtype="f32", io_dtype="bf16", data="synthetic",
+        config=dict(workload=wl.name, batch=B, tokens_per_seq=M, k=k, n_q_heads=Hq, n_layers=nL,
+                    context_slots=int(batch.cache_len_in.max().item()), rebind_bytes=nbytes,
+                    l2=flush.describe(nbytes)),
+        us_select=statistics.mean(part[0]), us_rebind_inject=statistics.mean(part[1]),
+        us_decode=statistics.mean(part[2]), us_per_revisit=statistics.mean(total) / B,
+        **_launch_keys(launched, 7, args.steps), clocks=clk.summary())), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -698,6 +789,8 @@ def main():
         run_decode_path(args)
     elif args.path == "select":
         run_select_path(args)
+    elif args.path == "pipeline":
+        run_pipeline_path(args)
     else:
         run_gpu(args)
 

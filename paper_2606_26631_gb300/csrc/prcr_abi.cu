@@ -362,10 +362,13 @@ void decode_split(int64_t base_ctas, int64_t max_len, int sms, int64_t q_elems, 
     if (want < 1) want = 1;
     int64_t c = (max_len + want - 1) / want;
     c = (c + 31) / 32 * 32;
-    // below ~768 slots a chunk's prologue and its share of the merge outweigh
-    // the better balance (measured: 512 -> 768 slots took the qwen25vl-7b
-    // shape from 5032 to 5394 GB/s; 1184 -> 768 changed qwen3vl-8b by < 1 %)
-    if (c < 768) c = 768;
+    // Below ~768 slots a chunk's prologue and its share of the merge outweigh
+    // the better balance when there is work for a few waves anyway (measured:
+    // 512 -> 768 slots took the qwen25vl-7b shape from 5032 to 5394 GB/s;
+    // 1184 -> 768 changed qwen3vl-8b by < 1 %). A small batch (one sequence
+    // of ~1k slots) needs the parallelism instead: chunks of 64 slots.
+    const int64_t floor_c = base_ctas * ((max_len + 767) / 768) >= int64_t(sms) * 6 ? 768 : 64;
+    if (c < floor_c) c = floor_c;
     if (c > kDecodeMaxChunk) c = kDecodeMaxChunk;
     const int64_t cap = (int64_t(kDecodeSmem) - q_elems * int64_t(sizeof(float))) / 8 / 32 * 32;
     if (c > cap) c = cap;
