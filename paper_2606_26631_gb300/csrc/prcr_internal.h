@@ -252,6 +252,7 @@ struct SelectArgs {
     int32_t n_seqs;
     int32_t n_tiles;            // token tiles of the logits kernel per sequence
     int32_t tok_tile;           // tokens per tile
+    int32_t kh_per_item;        // tensor-core logits: KV heads per work item
     float* score_out;           // optional [B][n_tokens]
     int32_t* idx_out;           // [B][k]
     int32_t* rev_tok_off;       // [B + 1]

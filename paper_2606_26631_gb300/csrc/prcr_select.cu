@@ -272,34 +272,41 @@ __device__ __forceinline__ void mma_1688_tf32(float (&c)[4], uint32_t a0, uint32
 // and both products are summed (float32 accumulate): each keeps ~20
 // significant bits (float32-level logits) over float32's range.
 // The accumulator of lane (g, t) holds head g at tokens 2t, 2t+1 of the octet.
-template <int D>
+// SPLIT: work items cover a group of KV heads (small batches); else every
+// item covers all of them.
+template <int D, bool SPLIT>
 __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_constant__ SelectArgs a) {
     constexpr int P = D / 2, PL = P / 4, T = 64;
     constexpr int NW = PL / 8;  // 16-byte loads per half row per lane
     extern __shared__ __align__(16) float sm[];
     const int Hq = a.n_q_heads, H = a.n_kv_heads, g = Hq / H, M = a.n_tokens;
-    uint2* qa_s = reinterpret_cast<uint2*>(sm);                // [H][PL][32]: (a0, a2), raw queries
-    float* lg_s = reinterpret_cast<float*>(qa_s + H * PL * 32);  // [Hq][T + 1]
+    // a work item is (sequence, group of KPI KV heads, token tile), tiles fastest
+    const int KPI = SPLIT ? a.kh_per_item : H, n_khg = SPLIT ? (H + KPI - 1) / KPI : 1;
+    uint2* qa_s = reinterpret_cast<uint2*>(sm);                  // [KPI][PL][32]: (a0, a2), raw queries
+    float* lg_s = reinterpret_cast<float*>(qa_s + KPI * PL * 32);  // [Hq][T + 1]
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int gid = lane >> 2, tq = lane & 3;
-    const int64_t total = int64_t(a.n_seqs) * a.n_tiles;
+    const int64_t total = int64_t(a.n_seqs) * n_khg * a.n_tiles;
     const int64_t t_beg = total * blockIdx.x / gridDim.x, t_end = total * (blockIdx.x + 1) / gridDim.x;
     // axis of each of this lane's pairs, two bits each
     uint32_t axes = 0u;
 #pragma unroll
     for (int p = 0; p < PL; ++p)
         axes |= uint32_t(pair_axis(tq * PL + p, a.layout, a.sec_t, a.sec_h, a.sec_w)) << (2 * p);
-    int cur_b = -1;
+    int64_t cur_bg = -1;
 
-    for (int64_t tile = t_beg; tile < t_end; ++tile) {
-        const int b = int(tile / a.n_tiles), j = int(tile % a.n_tiles);
+    for (int64_t item = t_beg; item < t_end; ++item) {
+        const int64_t bg = item / a.n_tiles;  // (sequence, KV-head group)
+        const int b = SPLIT ? int(bg / n_khg) : int(bg), j = int(item - bg * a.n_tiles);
+        const int kh_a = SPLIT ? int(bg - int64_t(b) * n_khg) * KPI : 0;
+        const int kh_b = SPLIT ? min(H, kh_a + KPI) : H;
         const int m0 = j * T, nt = min(T, M - m0);
-        if (b != cur_b) {
-            // the sequence's raw queries as A fragments (a bf16 value is an
-            // exact tf32 operand)
+        if (bg != cur_bg) {
+            // the group's raw queries as A fragments (a bf16 value is an exact
+            // tf32 operand)
             const uint16_t* qs = a.q + int64_t(b) * Hq * D;
-            for (int e = tid; e < H * PL * 32; e += blockDim.x) {
-                const int kh = e / (PL * 32), ks = (e / 32) % PL, ln = e & 31;
+            for (int e = tid; e < (kh_b - kh_a) * PL * 32; e += blockDim.x) {
+                const int kh = kh_a + e / (PL * 32), ks = (e / 32) % PL, ln = e & 31;
                 const int h = ln >> 2, tt = ln & 3;
                 uint2 f = make_uint2(0u, 0u);
                 if (h < g) {
@@ -309,7 +316,7 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
                 }
                 qa_s[e] = f;
             }
-            cur_b = b;
+            cur_bg = bg;
         }
         __syncthreads();
 
@@ -335,17 +342,17 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
         uint4 xn[NW], yn[NW];
 #pragma unroll
         for (int u = 0; u < NW; ++u) {
-            xn[u] = live ? ld_stream(krow + 8 * u) : make_uint4(0u, 0u, 0u, 0u);
-            yn[u] = live ? ld_stream(krow + P + 8 * u) : make_uint4(0u, 0u, 0u, 0u);
+            xn[u] = live ? ld_stream(krow + kh_a * D + 8 * u) : make_uint4(0u, 0u, 0u, 0u);
+            yn[u] = live ? ld_stream(krow + kh_a * D + P + 8 * u) : make_uint4(0u, 0u, 0u, 0u);
         }
-        for (int kh = 0; kh < H; ++kh) {
+        for (int kh = kh_a; kh < kh_b; ++kh) {
             uint32_t xw[4 * NW], yw[4 * NW];
 #pragma unroll
             for (int u = 0; u < NW; ++u) {
                 xw[4 * u] = xn[u].x; xw[4 * u + 1] = xn[u].y; xw[4 * u + 2] = xn[u].z; xw[4 * u + 3] = xn[u].w;
                 yw[4 * u] = yn[u].x; yw[4 * u + 1] = yn[u].y; yw[4 * u + 2] = yn[u].z; yw[4 * u + 3] = yn[u].w;
             }
-            if (kh + 1 < H) {  // the next head's pairs, in flight during this head's MMAs
+            if (kh + 1 < kh_b) {  // the next head's pairs, in flight during this head's MMAs
 #pragma unroll
                 for (int u = 0; u < NW; ++u) {
                     xn[u] = live ? ld_stream(krow + (kh + 1) * D + 8 * u) : make_uint4(0u, 0u, 0u, 0u);
@@ -353,7 +360,7 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
                 }
             }
             float c[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-            const uint2* qa = qa_s + kh * PL * 32 + lane;
+            const uint2* qa = qa_s + (kh - kh_a) * PL * 32 + lane;
 #pragma unroll
             for (int ks = 0; ks < PL; ++ks) {
                 // pair ks of this lane: element ks of each half
@@ -379,7 +386,7 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
         }
         __syncthreads();
 
-        for (int hq = warp; hq < Hq; hq += blockDim.x >> 5) {
+        for (int hq = kh_a * g + warp; hq < kh_b * g; hq += blockDim.x >> 5) {
             const float* row = lg_s + hq * (T + 1);
             float mx = -INFINITY;
             for (int t = lane; t < nt; t += 32) mx = fmaxf(mx, row[t]);
@@ -442,7 +449,15 @@ __global__ void __launch_bounds__(256) ads_relevance_kernel(const __grid_constan
     if (m >= M) return;
     const float* lg = a.logits + int64_t(b) * Hq * M + m;
     float r = 0.0f;
-    for (int h = 0; h < Hq; ++h) r = fmaf(expf(lg[int64_t(h) * M] - s_n[2 * h]), s_n[2 * h + 1], r);
+    int h = 0;
+    for (; h + 8 <= Hq; h += 8) {  // eight heads' logits requested together
+        float x[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) x[u] = lg[int64_t(h + u) * M];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) r = fmaf(expf(x[u] - s_n[2 * (h + u)]), s_n[2 * (h + u) + 1], r);
+    }
+    for (; h < Hq; ++h) r = fmaf(expf(lg[int64_t(h) * M] - s_n[2 * h]), s_n[2 * h + 1], r);
     a.rel[int64_t(b) * M + m] = r;
     if (a.score_out) a.score_out[int64_t(b) * M + m] = r;
 }
@@ -608,15 +623,29 @@ template <int D>
 cudaError_t launch_logits_mma(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream) {
     const size_t smem = size_t(a.n_kv_heads) * (D / 8) * 32 * 8 +
                         size_t(a.n_q_heads) * (a.tok_tile + 1) * 4;
-    cudaError_t e = cudaFuncSetAttribute(ads_logits_mma_kernel<D>,
+    cudaError_t e = cudaFuncSetAttribute(ads_logits_mma_kernel<D, false>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(ads_logits_mma_kernel<D, true>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     if (e != cudaSuccess) return e;
     int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ads_logits_mma_kernel<D>, 256, smem);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ads_logits_mma_kernel<D, false>, 256,
+                                                      smem);
     if (e != cudaSuccess) return e;
-    const int64_t tiles = int64_t(n_seqs) * a.n_tiles;
     const int64_t resident = int64_t(sms) * (per_sm > 0 ? per_sm : 1);
-    ads_logits_mma_kernel<D><<<unsigned(tiles < resident ? tiles : resident), 256, smem, stream>>>(a);
+    // Few tiles (a small batch): split the KV heads over work items until
+    // there are two per resident CTA, so that short chains run side by side.
+    SelectArgs b = a;
+    const int H = a.n_kv_heads;
+    b.kh_per_item = H;
+    while (b.kh_per_item > 1 &&
+           int64_t(n_seqs) * a.n_tiles * ((H + b.kh_per_item - 1) / b.kh_per_item) < 2 * resident)
+        b.kh_per_item = (b.kh_per_item + 1) / 2;
+    const int64_t items = int64_t(n_seqs) * a.n_tiles * ((H + b.kh_per_item - 1) / b.kh_per_item);
+    const unsigned grid = unsigned(items < resident ? items : resident);
+    if (b.kh_per_item < H) ads_logits_mma_kernel<D, true><<<grid, 256, smem, stream>>>(b);
+    else ads_logits_mma_kernel<D, false><<<grid, 256, smem, stream>>>(b);
     return cudaGetLastError();
 }
 
