@@ -283,7 +283,9 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int sr
                  : "memory");
 }
 
-template <int D>
+// HG: the CTAs of a (sequence, layer, chunk) split its KV heads, one per warp
+// (small batches: more, shorter CTAs); else one CTA takes all of them.
+template <int D, bool HG>
 __global__ void __launch_bounds__(kDecodeThreads, 3)
     decode_mma_kernel(const __grid_constant__ DecodeArgs a) {
     constexpr int KS = D / 16;     // k-steps of QK, m-tiles of PV
@@ -297,7 +299,14 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     uint16_t* vbuf = reinterpret_cast<uint16_t*>(smem_raw + size_t(Hq) * D * sizeof(float));
     const int b = blockIdx.z;
     const int l = blockIdx.y;
-    const int split = blockIdx.x;
+    constexpr int NWARP = kDecodeThreads / 32;
+    int split = blockIdx.x, kh0 = 0, kh1 = a.n_kv_heads;
+    if constexpr (HG) {
+        const int n_hg = (a.n_kv_heads + NWARP - 1) / NWARP;
+        split = int(blockIdx.x) / n_hg;
+        kh0 = (int(blockIdx.x) - split * n_hg) * NWARP;
+        kh1 = min(a.n_kv_heads, kh0 + NWARP);
+    }
     uint32_t err = 0;
 
     int64_t len = a.seq_len[b];
@@ -315,7 +324,9 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     }
     __syncthreads();
     const uint16_t* qb = a.q + (int64_t(b) * a.n_layers + l) * Hq * D;
-    for (int e = threadIdx.x; e < Hq * P; e += blockDim.x) {
+    // the query heads of this CTA's KV heads
+    const int e_beg = HG ? kh0 * a.group * P : 0, e_end = HG ? kh1 * a.group * P : Hq * P;
+    for (int e = e_beg + threadIdx.x; e < e_end; e += blockDim.x) {
         const int hq = e / P;
         const int i = e - hq * P;
         const float sn = s_sin[i], cs = s_cos[i];
@@ -336,7 +347,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     uint16_t* wv = vbuf + size_t(warp) * 2 * 16 * PITCH;
     const uint32_t wv_s = uint32_t(__cvta_generic_to_shared(wv));
 
-    for (int kh = warp; kh < a.n_kv_heads; kh += nwarps) {
+    for (int kh = kh0 + warp; kh < kh1; kh += nwarps) {
         // Q A-fragments (rows = heads of the group; rows >= g and 8..15 are zero)
         uint32_t qh[KS][2], ql[KS][2];
         {
@@ -514,23 +525,68 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     if (err) atomicOr(a.status, err);
 }
 
-// Merge the chunks of one (sequence, layer, query head): thread d owns one dimension.
+// Merge the chunks of one (sequence, layer, query head). The chunks' maxima
+// and sums are reduced by the whole CTA, their weights exp(m_s - M) staged in
+// shared memory 256 at a time, and thread d accumulates dimension d over the
+// chunks with eight partial rows requested at once.
 __global__ void __launch_bounds__(256) decode_merge_kernel(const __grid_constant__ DecodeArgs a) {
-    const int D = a.head_dim;
+    __shared__ float s_red[8];
+    __shared__ float s_w[256];
+    const int D = a.head_dim, S = a.splits, R = D + 2;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
     const int64_t o_idx = blockIdx.x;
-    const float* part = a.partial + o_idx * a.splits * (D + 2);
+    const float* part = a.partial + o_idx * S * R;
     float M = -INFINITY;
-    for (int s = 0; s < a.splits; ++s) M = fmaxf(M, part[s * (D + 2) + D]);
-    for (int d = threadIdx.x; d < D; d += blockDim.x) {
-        float num = 0.0f, den = 0.0f;
-        for (int s = 0; s < a.splits; ++s) {
-            const float ms = part[s * (D + 2) + D];
-            if (ms == -INFINITY) continue;
-            const float w = expf(ms - M);
-            num = fmaf(w, part[s * (D + 2) + d], num);
-            den = fmaf(w, part[s * (D + 2) + D + 1], den);
+    for (int sp = threadIdx.x; sp < S; sp += blockDim.x) M = fmaxf(M, part[int64_t(sp) * R + D]);
+#pragma unroll
+    for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    if (lane == 0) s_red[warp] = M;
+    __syncthreads();
+    M = s_red[0];
+    for (int w = 1; w < nw; ++w) M = fmaxf(M, s_red[w]);
+    __syncthreads();
+    float den = 0.0f;
+    for (int sp = threadIdx.x; sp < S; sp += blockDim.x) {
+        const float ms = part[int64_t(sp) * R + D];
+        if (ms != -INFINITY) den = fmaf(expf(ms - M), part[int64_t(sp) * R + D + 1], den);
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) den += __shfl_xor_sync(0xffffffffu, den, o);
+    if (lane == 0) s_red[warp] = den;
+    __syncthreads();
+    den = 0.0f;
+    for (int w = 0; w < nw; ++w) den += s_red[w];
+    float num[2] = {0.0f, 0.0f};  // dimensions threadIdx.x and threadIdx.x + blockDim.x (D <= 2 x 256)
+    for (int s0 = 0; s0 < S; s0 += 256) {
+        const int n = min(256, S - s0);
+        __syncthreads();
+        for (int q = threadIdx.x; q < n; q += blockDim.x) {
+            const float ms = part[int64_t(s0 + q) * R + D];
+            s_w[q] = ms == -INFINITY ? 0.0f : expf(ms - M);
         }
-        a.out[o_idx * D + d] = den > 0.0f ? num / den : 0.0f;
+        __syncthreads();
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const int d = threadIdx.x + k * blockDim.x;
+            if (d >= D) break;
+            const float* col = part + int64_t(s0) * R + d;
+            float acc = num[k];
+            int q = 0;
+            for (; q + 8 <= n; q += 8) {
+                float x[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) x[u] = col[int64_t(q + u) * R];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) acc = fmaf(s_w[q + u], x[u], acc);
+            }
+            for (; q < n; ++q) acc = fmaf(s_w[q], col[int64_t(q) * R], acc);
+            num[k] = acc;
+        }
+    }
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const int d = threadIdx.x + k * blockDim.x;
+        if (d < D) a.out[o_idx * D + d] = den > 0.0f ? num[k] / den : 0.0f;
     }
 }
 
@@ -553,12 +609,23 @@ cudaError_t launch_decode(const DecodeArgs& a, int gp, dim3 grid, size_t smem,
         // tensor-core kernel: rotated queries + two staged V tiles per warp
         const size_t sm = size_t(a.n_q_heads) * a.head_dim * sizeof(float) +
                           size_t(kDecodeThreads / 32) * 2 * 16 * (a.head_dim + 8) * sizeof(uint16_t);
+        // a batch that fills under ~2 waves of resident CTAs splits its KV
+        // heads over more CTAs (a shorter chain per CTA)
+        const int n_hg = (a.n_kv_heads + kDecodeThreads / 32 - 1) / (kDecodeThreads / 32);
+        int dev = 0, sms = 148;
+        if (cudaGetDevice(&dev) == cudaSuccess)
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        const bool hg = n_hg > 1 && int64_t(grid.x) * grid.y * grid.z < int64_t(sms) * 6;
+        dim3 g2 = grid;
+        if (hg) g2.x *= unsigned(n_hg);
         if (a.head_dim == 64) {
-            e = cudaFuncSetAttribute(decode_mma_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
-            if (e == cudaSuccess) decode_mma_kernel<64><<<grid, kDecodeThreads, sm, stream>>>(a);
+            auto k = hg ? decode_mma_kernel<64, true> : decode_mma_kernel<64, false>;
+            e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
+            if (e == cudaSuccess) k<<<g2, kDecodeThreads, sm, stream>>>(a);
         } else {
-            e = cudaFuncSetAttribute(decode_mma_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
-            if (e == cudaSuccess) decode_mma_kernel<128><<<grid, kDecodeThreads, sm, stream>>>(a);
+            auto k = hg ? decode_mma_kernel<128, true> : decode_mma_kernel<128, false>;
+            e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
+            if (e == cudaSuccess) k<<<g2, kDecodeThreads, sm, stream>>>(a);
         }
         if (e == cudaSuccess) e = cudaGetLastError();
     } else {
