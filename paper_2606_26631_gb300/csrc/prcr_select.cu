@@ -490,7 +490,7 @@ __device__ __forceinline__ int block_scan(int v, int* s_warp, int* out_excl) {
 }
 
 // PER: relevances per thread (a thread keeps its PER consecutive tokens in
-// registers; 1024 * PER >= n_tokens).
+// registers; blockDim.x * PER >= n_tokens, blockDim.x a multiple of 32).
 template <int PER>
 __global__ void __launch_bounds__(1024) ads_select_kernel(const __grid_constant__ SelectArgs a) {
     __shared__ int s_warp[32];
@@ -499,6 +499,7 @@ __global__ void __launch_bounds__(1024) ads_select_kernel(const __grid_constant_
     const int M = a.n_tokens;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int beg = threadIdx.x * PER;
+    const int nwarp = blockDim.x >> 5;  // a multiple of 32 threads, <= 1024
 
     // this thread's relevances (from the relevance kernel); tokens past the
     // end read as 0 and are excluded wherever 0 could count
@@ -533,9 +534,10 @@ __global__ void __launch_bounds__(1024) ads_select_kernel(const __grid_constant_
             s_cnt[64 + warp] = c3;
         }
         __syncthreads();
-        const unsigned int t1 = __reduce_add_sync(0xffffffffu, s_cnt[lane]);
-        const unsigned int t2 = __reduce_add_sync(0xffffffffu, s_cnt[32 + lane]);
-        const unsigned int t3 = __reduce_add_sync(0xffffffffu, s_cnt[64 + lane]);
+        const bool wl = lane < nwarp;  // this lane reads warp `lane`'s counts
+        const unsigned int t1 = __reduce_add_sync(0xffffffffu, wl ? s_cnt[lane] : 0u);
+        const unsigned int t2 = __reduce_add_sync(0xffffffffu, wl ? s_cnt[32 + lane] : 0u);
+        const unsigned int t3 = __reduce_add_sync(0xffffffffu, wl ? s_cnt[64 + lane] : 0u);
         X = t3 >= K ? x3 : (t2 >= K ? x2 : (t1 >= K ? x1 : X));
         __syncthreads();
     }
@@ -549,7 +551,7 @@ __global__ void __launch_bounds__(1024) ads_select_kernel(const __grid_constant_
     above = __reduce_add_sync(0xffffffffu, above);
     if (lane == 0) s_cnt[warp] = above;
     __syncthreads();
-    const int need_eq = int(K - __reduce_add_sync(0xffffffffu, s_cnt[lane]));
+    const int need_eq = int(K - __reduce_add_sync(0xffffffffu, lane < nwarp ? s_cnt[lane] : 0u));
 
     // 2. ordered compaction: all keys > X, then the first need_eq keys == X
     int eq_before = 0;
@@ -667,10 +669,12 @@ cudaError_t launch_select(const SelectArgs& a, int n_seqs, int sms, cudaStream_t
     ads_relevance_kernel<<<dim3((a.n_tokens + 255) / 256, n_seqs, 1), 256, 0, stream>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     const int M = a.n_tokens;
-    if (M <= 4096) ads_select_kernel<4><<<n_seqs, 1024, 0, stream>>>(a);
-    else if (M <= 8192) ads_select_kernel<8><<<n_seqs, 1024, 0, stream>>>(a);
-    else if (M <= 16384) ads_select_kernel<16><<<n_seqs, 1024, 0, stream>>>(a);
-    else ads_select_kernel<32><<<n_seqs, 1024, 0, stream>>>(a);
+    // just enough warps for PER tokens per thread: fewer warps, cheaper rounds
+    auto threads = [M](int per) { return int(((M + per - 1) / per + 31) / 32 * 32); };
+    if (M <= 4096) ads_select_kernel<4><<<n_seqs, threads(4), 0, stream>>>(a);
+    else if (M <= 8192) ads_select_kernel<8><<<n_seqs, threads(8), 0, stream>>>(a);
+    else if (M <= 16384) ads_select_kernel<16><<<n_seqs, threads(16), 0, stream>>>(a);
+    else ads_select_kernel<32><<<n_seqs, threads(32), 0, stream>>>(a);
     return cudaGetLastError();
 }
 
