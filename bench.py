@@ -752,20 +752,45 @@ def run_pipeline_path(args):
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
-    with Clocks(local) as clk:
-        for e in ev:
-            flush()
-            e[0].record(stream)
-            select()
-            e[1].record(stream)
-            rv.run()
-            e[2].record(stream)
-            decode()
-            e[3].record(stream)
+    if args.graph:
+        # the three stages as one CUDA graph (no launch gaps), one replay per step
+        g = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            step()
+        stream.wait_stream(side)
         torch.cuda.synchronize()
-    part = [[e[i].elapsed_time(e[i + 1]) * 1e3 for e in ev] for i in range(3)]
-    total = [e[0].elapsed_time(e[3]) * 1e3 for e in ev]
+        with torch.cuda.graph(g):
+            step()
+        for _ in range(3):
+            g.replay()
+        torch.cuda.synchronize()
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+        with Clocks(local) as clk:
+            for e in ev:
+                flush()
+                e[0].record(stream)
+                g.replay()
+                e[1].record(stream)
+            torch.cuda.synchronize()
+        total = [e[0].elapsed_time(e[1]) * 1e3 for e in ev]
+        part = [[float("nan")] for _ in range(3)]
+    else:
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+        with Clocks(local) as clk:
+            for e in ev:
+                flush()
+                e[0].record(stream)
+                select()
+                e[1].record(stream)
+                rv.run()
+                e[2].record(stream)
+                decode()
+                e[3].record(stream)
+            torch.cuda.synchronize()
+        part = [[e[i].elapsed_time(e[i + 1]) * 1e3 for e in ev] for i in range(3)]
+        total = [e[0].elapsed_time(e[3]) * 1e3 for e in ev]
     print(json.dumps(dict(
         metric="revisit pipeline us per step (select + rebind/inject + first decode)",
         value=statistics.mean(total), unit="us", n_gpus=1, steps=args.steps, warmup=args.warmup,
@@ -774,6 +799,8 @@ def run_pipeline_path(args):
         config=dict(workload=wl.name, batch=B, tokens_per_seq=M, k=k, n_q_heads=Hq, n_layers=nL,
                     context_slots=int(batch.cache_len_in.max().item()), rebind_bytes=nbytes,
                     l2=flush.describe(nbytes)),
+        timing="one CUDA graph per step (stages not timed separately)" if args.graph
+        else "stream launches, events around each stage",
         us_select=statistics.mean(part[0]), us_rebind_inject=statistics.mean(part[1]),
         us_decode=statistics.mean(part[2]), us_per_revisit=statistics.mean(total) / B,
         **_launch_keys(launched, 7, args.steps), clocks=clk.summary())), flush=True)
