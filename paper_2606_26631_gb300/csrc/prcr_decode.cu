@@ -309,6 +309,27 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     }
     uint32_t err = 0;
 
+    // Requests that do not depend on the sequence length go out first: this
+    // CTA's query rows, and (contiguous caches) its first tile's K and V rows,
+    // are prefetched to L2 while the length and position load.
+    {
+        const char* qrow = reinterpret_cast<const char*>(
+            a.q + ((int64_t(b) * a.n_layers + l) * Hq + kh0 * a.group) * D);
+        const int qbytes = (kh1 - kh0) * a.group * D * 2;
+        for (int o = threadIdx.x * 128; o < qbytes; o += blockDim.x * 128) prefetch_l2(qrow + o);
+        if (a.cache_kind == PRCR_CACHE_CONTIGUOUS) {
+            const int64_t s = int64_t(split) * a.chunk + (threadIdx.x & 15);
+            const int kh = kh0 + ((threadIdx.x >> 4) & 3);
+            if (s < a.capacity && kh < kh1) {
+                const int64_t row = int64_t(b) * a.seq_stride + s * a.slot_stride +
+                                    int64_t(l) * a.layer_stride + int64_t(kh) * D;
+                const uint16_t* base = (threadIdx.x & 64) ? a.cache_v : a.cache_k;
+#pragma unroll
+                for (int c = 0; c < D * 2; c += 128) prefetch_l2(base + row + c / 2);
+            }
+        }
+    }
+
     int64_t len = a.seq_len[b];
     if (len < 0 || len > a.capacity) {
         err |= PRCR_ST_CAPACITY;
