@@ -276,7 +276,8 @@ PRCR_API int prcr_prefill_capture(const prcr_rope_cfg* cfg, const prcr_store_des
  *            seq_len is a host bound used for the split of the sequence axis
  *   out:     device float32 [n_seqs][n_layers][n_q_heads][D]
  * Limits: D in {64, 128, 256}; n_q_heads a multiple of n_kv_heads, at most 8
- * query heads per KV head and n_q_heads * D <= PRCR_DECODE_MAX_Q_ELEMS.
+ * query heads per KV head and n_q_heads * D <= PRCR_DECODE_MAX_Q_ELEMS;
+ * n_seqs and n_layers at most 65535 (launch grid limits).
  * workspace: device, >= prcr_decode_workspace_size(...) bytes (0 when the
  * sequence axis is not split), 16-byte aligned. A seq_len beyond the
  * capacity sets PRCR_ST_CAPACITY (clamped); an unmapped block in range sets
