@@ -161,3 +161,35 @@ def test_select_full_size_sampled():
         assert ref[chosen].min() >= ref[~chosen].max() - tol
     del batch
     torch.cuda.empty_cache()
+
+
+def test_select_interleaved_layout():
+    """The interleaved M-RoPE band layout (pair i to h when i % 3 == 1, to w
+    when i % 3 == 2, within their sections) on both logits kernels: head_dim
+    128 (tensor cores) and 48 (CUDA cores)."""
+    import paper_2606_26631_gb300 as prcr
+    for wl, Hq, k, layer in ((get("qwen2vl-2b"), 8, 100, 9), (SHAPES["sel-odd"], 9, 20, 1)):
+        batch = make_batch(wl, device=DEV)
+        B, M, D = wl.n_seqs, wl.n_tokens, wl.head_dim
+        cfg = prcr.rope_cfg(wl.n_layers, wl.n_kv_heads, D, wl.sections, wl.theta,
+                            O.LAYOUT_INTERLEAVED)
+        sd = prcr.store_desc(batch.store_k, batch.store_v, batch.coords)
+        q = (3.0 * torch.randn((B, Hq, D), device=DEV,
+                               generator=torch.Generator(device=DEV).manual_seed(8))).to(torch.bfloat16)
+        idx = torch.empty(B * k, dtype=torch.int32, device=DEV)
+        sro = torch.empty(B + 1, dtype=torch.int32, device=DEV)
+        rto = torch.empty(B + 1, dtype=torch.int32, device=DEV)
+        score = torch.empty((B, M), dtype=torch.float32, device=DEV)
+        ws = torch.empty(prcr.select_workspace_size(B, Hq, M), dtype=torch.uint8, device=DEV)
+        prcr.select_topk(cfg, sd, layer, q, batch.p_txt, k, idx, sro, rto, ws, score)
+        torch.cuda.synchronize()
+        qv = O.bf16_bits_to_f64(q.view(torch.int16).cpu().numpy())
+        coords = batch.coords.cpu().numpy()
+        sc = score.cpu().numpy()
+        sel = idx.view(B, k).cpu().numpy()
+        for b in range(B):
+            k_raw = batch.store_k[b, layer].view(torch.int16).cpu().numpy()
+            ref = O.ads_relevance(qv[b], int(batch.p_txt[b]), k_raw, coords[b], D, wl.sections,
+                                  wl.theta, O.LAYOUT_INTERLEAVED)
+            assert (np.abs(sc[b] - ref) / ref).max() <= 1e-4, wl.name
+            assert np.array_equal(sel[b], _topk_by(sc[b].astype(np.float64), k))
