@@ -175,3 +175,34 @@ def test_prefill_capture_full_size_sampled():
         assert e["max_err"] <= pu.K_TOL, e
     del src, store_k, store_v, ck, cv
     torch.cuda.empty_cache()
+
+
+def test_prefill_capture_interleaved_layout():
+    """The cache keys rotated with the interleaved M-RoPE band layout."""
+    import paper_2606_26631_gb300 as prcr
+    import parity_util as pu
+    wl = get("qwen2vl-2b")
+    src = make_batch(wl, device=DEV)
+    nL, M, H, D = wl.n_layers, wl.n_tokens, wl.n_kv_heads, wl.head_dim
+    rng = np.random.default_rng(6)
+    ck, cv, bt = _cache(wl, 1, [7], M, False, rng)
+    store_k = torch.empty_like(src.store_k)
+    store_v = torch.empty_like(src.store_v)
+    coords = torch.empty_like(src.coords)
+    cfg = prcr.rope_cfg(nL, H, D, wl.sections, wl.theta, O.LAYOUT_INTERLEAVED)
+    sd = prcr.store_desc(store_k, store_v, coords)
+    cd = prcr.cache_contiguous(ck, cv)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    prcr.prefill_capture(cfg, sd, cd, 0, 0, 0, 7, src.store_k[0], src.store_v[0], src.coords[0],
+                         status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    layers = [0, nL // 2, nL - 1]
+    k_raw = pu.bits(src.store_k[0].transpose(0, 1)[:, layers])
+    v_raw = pu.bits(src.store_v[0].transpose(0, 1)[:, layers])
+    _, _, k_want, v_want = O.prefill_capture(k_raw, v_raw, src.coords[0].cpu().numpy(), D,
+                                             wl.sections, wl.theta, O.LAYOUT_INTERLEAVED)
+    slots = np.arange(M) + 7
+    assert np.array_equal(pu.bits(_rows(cv, bt, 0, slots, layers, False)), v_want)
+    e = pu.k_error(pu.bits(_rows(ck, bt, 0, slots, layers, False)), k_want, k_raw)
+    assert e["max_err"] <= pu.K_TOL, e
