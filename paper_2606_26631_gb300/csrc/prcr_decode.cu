@@ -28,6 +28,17 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kDecodeThreads = 128;
+// slots of its chunk a CTA of the head-split (small batch) variant requests
+// into L2 before its tile loop: 4 KV heads x 64 slots x 512 B = 128 KB
+constexpr int kDecodeHgPrefetch = 64;
+
+// The merge kernel is launched as a programmatic dependent of the decode
+// kernel: every decode CTA allows it at entry, so that the merge's CTAs are
+// launched once the last decode CTA is resident and only wait (below) for the
+// decode grid to complete and its partials to be visible.
+__device__ __forceinline__ void allow_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
 
 
 // EPL consecutive bf16 of a row as EPL / 2 packed words.
@@ -57,6 +68,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3) decode_kernel(const __grid_
     const int l = blockIdx.y;
     const int split = blockIdx.x;
     uint32_t err = 0;
+    allow_dependents();
 
     int64_t len = a.seq_len[b];
     if (len < 0 || len > a.capacity) {
@@ -308,6 +320,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
         kh1 = min(a.n_kv_heads, kh0 + NWARP);
     }
     uint32_t err = 0;
+    allow_dependents();
 
     // Requests that do not depend on the sequence length go out first: this
     // CTA's query rows, and (contiguous caches) its first tile's K and V rows,
@@ -337,24 +350,79 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     }
     const int64_t s_begin = int64_t(split) * a.chunk;
     const int64_t s_end = min(len, s_begin + a.chunk);
+    if constexpr (HG) {
+        // A small batch gives each warp a few tiles only, and a chain of a
+        // few DRAM round trips per warp is most of the CTA's life: the chunk's
+        // rows (its first kDecodeHgPrefetch slots) are all requested into L2
+        // now, so that the tile loop waits on L2. Slot s's KV heads kh0..kh1
+        // are one contiguous span of its K (and of its V) row.
+        const int64_t s_lo = a.cache_kind == PRCR_CACHE_CONTIGUOUS ? s_begin + 16 : s_begin;
+        const int64_t s_hi = min(s_end, s_begin + kDecodeHgPrefetch);
+        const int span = (kh1 - kh0) * D * 2;  // bytes
+        for (int64_t s = s_lo + threadIdx.x; s < s_hi; s += blockDim.x) {
+            int64_t row;
+            if (a.cache_kind == PRCR_CACHE_CONTIGUOUS) {
+                row = int64_t(b) * a.seq_stride + s * a.slot_stride;
+            } else {
+                const int64_t lb = s / a.block_size;
+                const int32_t blk = a.block_table[int64_t(b) * a.bt_stride + lb];
+                if (blk < 0 || blk >= a.n_blocks) continue;  // reported by the tile loop
+                row = int64_t(blk) * a.block_stride + (s - lb * a.block_size) * a.slot_stride;
+            }
+            const int64_t off = row + int64_t(l) * a.layer_stride + int64_t(kh0) * D;
+            const char* kp = reinterpret_cast<const char*>(a.cache_k + off);
+            const char* vp = reinterpret_cast<const char*>(a.cache_v + off);
+            for (int o = 0; o < span; o += 128) {
+                prefetch_l2(kp + o);
+                prefetch_l2(vp + o);
+            }
+        }
+    }
 
-    __shared__ float s_cos[kMaxPairs], s_sin[kMaxPairs];
+    __shared__ __align__(16) float s_cos[kMaxPairs];
+    __shared__ __align__(16) float s_sin[kMaxPairs];
     const int64_t p = a.q_pos[b];
     for (int i = threadIdx.x; i < P; i += blockDim.x) {
         sincos_turns(double(p), a.turn_freq[i], &s_sin[i], &s_cos[i]);
     }
     __syncthreads();
     const uint16_t* qb = a.q + (int64_t(b) * a.n_layers + l) * Hq * D;
-    // the query heads of this CTA's KV heads
+    // the query heads of this CTA's KV heads, eight rotation pairs per thread
+    // (two 16-byte loads when the query rows are 16-byte aligned)
     const int e_beg = HG ? kh0 * a.group * P : 0, e_end = HG ? kh1 * a.group * P : Hq * P;
-    for (int e = e_beg + threadIdx.x; e < e_end; e += blockDim.x) {
+    const bool q16 = (reinterpret_cast<uintptr_t>(a.q) & 15) == 0;
+    for (int e = e_beg + 8 * threadIdx.x; e < e_end; e += 8 * blockDim.x) {
         const int hq = e / P;
-        const int i = e - hq * P;
-        const float sn = s_sin[i], cs = s_cos[i];
-        const float x = __uint_as_float(uint32_t(qb[hq * D + i]) << 16);
-        const float y = __uint_as_float(uint32_t(qb[hq * D + i + P]) << 16);
-        q_s[hq * D + i] = fmaf(x, cs, -y * sn) * a.scale;
-        q_s[hq * D + i + P] = fmaf(y, cs, x * sn) * a.scale;
+        const int i = e - hq * P;  // a multiple of 8: P is 32 or 64
+        const uint16_t* qx = qb + hq * D + i;
+        uint32_t wx[4], wy[4];
+        if (q16) {
+            const uint4 x4 = __ldg(reinterpret_cast<const uint4*>(qx));
+            const uint4 y4 = __ldg(reinterpret_cast<const uint4*>(qx + P));
+            wx[0] = x4.x; wx[1] = x4.y; wx[2] = x4.z; wx[3] = x4.w;
+            wy[0] = y4.x; wy[1] = y4.y; wy[2] = y4.z; wy[3] = y4.w;
+        } else {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                wx[u] = uint32_t(qx[2 * u]) | (uint32_t(qx[2 * u + 1]) << 16);
+                wy[u] = uint32_t(qx[P + 2 * u]) | (uint32_t(qx[P + 2 * u + 1]) << 16);
+            }
+        }
+        float rx[8], ry[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const float x = __uint_as_float((u & 1) ? (wx[u >> 1] & 0xffff0000u) : (wx[u >> 1] << 16));
+            const float y = __uint_as_float((u & 1) ? (wy[u >> 1] & 0xffff0000u) : (wy[u >> 1] << 16));
+            const float sn = s_sin[i + u], cs = s_cos[i + u];
+            rx[u] = fmaf(x, cs, -y * sn) * a.scale;
+            ry[u] = fmaf(y, cs, x * sn) * a.scale;
+        }
+        float4* ox = reinterpret_cast<float4*>(q_s + hq * D + i);
+        float4* oy = reinterpret_cast<float4*>(q_s + hq * D + i + P);
+        ox[0] = make_float4(rx[0], rx[1], rx[2], rx[3]);
+        ox[1] = make_float4(rx[4], rx[5], rx[6], rx[7]);
+        oy[0] = make_float4(ry[0], ry[1], ry[2], ry[3]);
+        oy[1] = make_float4(ry[4], ry[5], ry[6], ry[7]);
     }
     __syncthreads();
 
@@ -554,6 +622,7 @@ __global__ void __launch_bounds__(256) decode_merge_kernel(const __grid_constant
     __shared__ float s_red[8];
     __shared__ float s_w[256];
     const int D = a.head_dim, S = a.splits, R = D + 2;
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // the decode grid's partials
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
     const int64_t o_idx = blockIdx.x;
     const float* part = a.partial + o_idx * S * R;
@@ -655,9 +724,16 @@ cudaError_t launch_decode(const DecodeArgs& a, int gp, dim3 grid, size_t smem,
         e = gp <= 4 ? launch_gp<4>(a, grid, smem, stream) : launch_gp<8>(a, grid, smem, stream);
     }
     if (e != cudaSuccess || a.splits == 1) return e;
-    const unsigned n = unsigned(int64_t(grid.z) * a.n_layers * a.n_q_heads);
-    decode_merge_kernel<<<n, a.head_dim < 256 ? a.head_dim : 256, 0, stream>>>(a);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(int64_t(grid.z) * a.n_layers * a.n_q_heads), 1, 1);
+    cfg.blockDim = dim3(a.head_dim < 256 ? a.head_dim : 256, 1, 1);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, decode_merge_kernel, a);
 }
 
 }  // namespace prcr

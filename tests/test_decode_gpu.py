@@ -56,6 +56,10 @@ CASES = [  # (B, layers, H, Hq, D, max_len, paged)
     (2, 2, 2, 14, 64, 700, False),
     (2, 2, 4, 4, 256, 1200, True),
     (5, 1, 4, 28, 128, 9000, True),
+    # one sequence of the Table 3 shape (small batch: KV heads split over
+    # CTAs, chunk rows requested into L2 ahead of the tile loop)
+    (1, 36, 8, 32, 128, 933, False),
+    (2, 2, 8, 16, 64, 500, True),
 ]
 
 
@@ -80,6 +84,25 @@ def test_decode_parity(case):
             ref = O.decode_attention(qv[b, l], int(inp["q_pos"][b]), K[:, l], V[:, l], D, sec, 1e6)
             err = np.abs(got[b, l] - ref).max() / np.abs(V[:, l]).max()
             assert err <= 1e-4, (b, l, err)
+
+
+def test_decode_unaligned_query():
+    """Query rows only 4-byte aligned (the ABI's minimum) take the scalar
+    loads of the rotation: the output is bit-identical to the aligned call."""
+    import paper_2606_26631_gb300 as prcr
+    B, nL, H, Hq, D, max_len = 1, 4, 8, 32, 128, 933
+    inp = make_decode_inputs(B, nL, H, Hq, D, max_len, False, device=DEV, seed=3)
+    cfg = prcr.rope_cfg(nL, H, D, (16, 24, 24), 1e6)
+    cd = prcr.cache_contiguous(inp["cache_k"], inp["cache_v"])
+    q = inp["q"]
+    buf = torch.empty(q.numel() + 2, dtype=torch.bfloat16, device=DEV)
+    q_odd = buf[2:].view(q.shape)
+    q_odd.copy_(q)
+    assert q_odd.data_ptr() % 16 == 4
+    ref, st0 = _run_decode(cfg, cd, q, inp["q_pos"], inp["seq_len"], max_len)
+    got, st1 = _run_decode(cfg, cd, q_odd, inp["q_pos"], inp["seq_len"], max_len)
+    assert st0 == 0 and st1 == 0
+    assert torch.equal(ref, got)
 
 
 def test_inject_then_decode():
