@@ -22,6 +22,7 @@
 #include <cuda_bf16.h>
 
 #include "prcr_device.cuh"
+#include "prcr_pdl.cuh"
 
 namespace prcr {
 namespace {
@@ -31,14 +32,6 @@ constexpr int kDecodeThreads = 128;
 // slots of its chunk a CTA of the head-split (small batch) variant requests
 // into L2 before its tile loop: 4 KV heads x 64 slots x 512 B = 128 KB
 constexpr int kDecodeHgPrefetch = 64;
-
-// The merge kernel is launched as a programmatic dependent of the decode
-// kernel: every decode CTA allows it at entry, so that the merge's CTAs are
-// launched once the last decode CTA is resident and only wait (below) for the
-// decode grid to complete and its partials to be visible.
-__device__ __forceinline__ void allow_dependents() {
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
 
 
 // EPL consecutive bf16 of a row as EPL / 2 packed words.
@@ -68,7 +61,8 @@ __global__ void __launch_bounds__(kDecodeThreads, 3) decode_kernel(const __grid_
     const int l = blockIdx.y;
     const int split = blockIdx.x;
     uint32_t err = 0;
-    allow_dependents();
+    pdl_allow();
+    pdl_wait();
 
     int64_t len = a.seq_len[b];
     if (len < 0 || len > a.capacity) {
@@ -320,7 +314,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
         kh1 = min(a.n_kv_heads, kh0 + NWARP);
     }
     uint32_t err = 0;
-    allow_dependents();
+    pdl_allow();
 
     // Requests that do not depend on the sequence length go out first: this
     // CTA's query rows, and (contiguous caches) its first tile's K and V rows,
@@ -343,6 +337,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
         }
     }
 
+    pdl_wait();
     int64_t len = a.seq_len[b];
     if (len < 0 || len > a.capacity) {
         err |= PRCR_ST_CAPACITY;
@@ -622,7 +617,8 @@ __global__ void __launch_bounds__(256) decode_merge_kernel(const __grid_constant
     __shared__ float s_red[8];
     __shared__ float s_w[256];
     const int D = a.head_dim, S = a.splits, R = D + 2;
-    asm volatile("griddepcontrol.wait;" ::: "memory");  // the decode grid's partials
+    pdl_allow();
+    pdl_wait();  // the decode grid's partials
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
     const int64_t o_idx = blockIdx.x;
     const float* part = a.partial + o_idx * S * R;
@@ -682,12 +678,12 @@ __global__ void __launch_bounds__(256) decode_merge_kernel(const __grid_constant
 
 template <int GP>
 cudaError_t launch_gp(const DecodeArgs& a, dim3 grid, size_t smem, cudaStream_t stream) {
+    const dim3 block(kDecodeThreads);
     switch (a.head_dim) {
-        case 64: decode_kernel<GP, 2><<<grid, kDecodeThreads, smem, stream>>>(a); break;
-        case 128: decode_kernel<GP, 4><<<grid, kDecodeThreads, smem, stream>>>(a); break;
-        default: decode_kernel<GP, 8><<<grid, kDecodeThreads, smem, stream>>>(a); break;
+        case 64: return launch_pdl(decode_kernel<GP, 2>, grid, block, smem, stream, a);
+        case 128: return launch_pdl(decode_kernel<GP, 4>, grid, block, smem, stream, a);
+        default: return launch_pdl(decode_kernel<GP, 8>, grid, block, smem, stream, a);
     }
-    return cudaGetLastError();
 }
 
 }  // namespace
@@ -711,29 +707,20 @@ cudaError_t launch_decode(const DecodeArgs& a, int gp, dim3 grid, size_t smem,
         if (a.head_dim == 64) {
             auto k = hg ? decode_mma_kernel<64, true> : decode_mma_kernel<64, false>;
             e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
-            if (e == cudaSuccess) k<<<g2, kDecodeThreads, sm, stream>>>(a);
+            if (e == cudaSuccess) e = launch_pdl(k, g2, dim3(kDecodeThreads), sm, stream, a);
         } else {
             auto k = hg ? decode_mma_kernel<128, true> : decode_mma_kernel<128, false>;
             e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
-            if (e == cudaSuccess) k<<<g2, kDecodeThreads, sm, stream>>>(a);
+            if (e == cudaSuccess) e = launch_pdl(k, g2, dim3(kDecodeThreads), sm, stream, a);
         }
-        if (e == cudaSuccess) e = cudaGetLastError();
     } else {
         // groups of 1, 2 and 4 query heads run as 4 (padded) heads x 8 slots per
         // warp iteration, groups of 5..8 as 8 heads x 4 slots
         e = gp <= 4 ? launch_gp<4>(a, grid, smem, stream) : launch_gp<8>(a, grid, smem, stream);
     }
     if (e != cudaSuccess || a.splits == 1) return e;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(unsigned(int64_t(grid.z) * a.n_layers * a.n_q_heads), 1, 1);
-    cfg.blockDim = dim3(a.head_dim < 256 ? a.head_dim : 256, 1, 1);
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, decode_merge_kernel, a);
+    return launch_pdl(decode_merge_kernel, dim3(unsigned(int64_t(grid.z) * a.n_layers * a.n_q_heads)),
+                      dim3(a.head_dim < 256 ? a.head_dim : 256), 0, stream, a);
 }
 
 }  // namespace prcr

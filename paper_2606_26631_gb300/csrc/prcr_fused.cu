@@ -11,6 +11,7 @@
 // arithmetic as the plan kernel (token_plan); then it streams the rows as the
 // rebind kernel does.
 #include "prcr_device.cuh"
+#include "prcr_pdl.cuh"
 
 namespace prcr {
 namespace {
@@ -27,19 +28,22 @@ __global__ void __launch_bounds__(512) fused_kernel(const __grid_constant__ Fuse
     __shared__ int s_bad;
     const bool lead = blockIdx.x == 0 && blockIdx.y == 0;
 
-    // 0. this thread's token index and the per-sequence inputs are requested
-    // before the offsets are checked, so that their latencies overlap
+    // 0. the per-sequence inputs are prefetched while the grid this one
+    // depends on finishes; this thread's token index is requested before the
+    // offsets are checked, so that their latencies overlap
+    pdl_allow();
     const int T = rb.tok_per_cta;
     const int64_t tok0 = int64_t(blockIdx.x) * T;
     const int lanes = rb.lanes;
     const int my_t = threadIdx.x / lanes;
     const int64_t my_j = tok0 + my_t;
     const bool my_tok = my_t < T && my_j < a.total_k;
-    const int my_m = my_tok ? a.idx[my_j] : -1;
     if (threadIdx.x < a.n_seqs) {
         prefetch_l2(a.cache_len_in + threadIdx.x);
         prefetch_l2(a.p_txt + threadIdx.x);
     }
+    pdl_wait();
+    const int my_m = my_tok ? a.idx[my_j] : -1;
 
     // 1. the offsets: monotone, spanning [0, total_k) and [0, n_revisits)
     if (threadIdx.x == 0) s_bad = 0;
@@ -218,8 +222,7 @@ cudaError_t fused_blocks_per_sm(int block, size_t smem, int* out) {
 
 cudaError_t launch_fused(const FusedArgs& a, dim3 grid, int block, size_t smem,
                          cudaStream_t stream) {
-    fused_kernel<<<grid, block, smem, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(fused_kernel, grid, dim3(block), smem, stream, a);
 }
 
 }  // namespace prcr

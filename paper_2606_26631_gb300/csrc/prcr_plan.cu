@@ -18,6 +18,7 @@
 #include <cmath>
 
 #include "prcr_device.cuh"
+#include "prcr_pdl.cuh"
 
 namespace prcr {
 namespace {
@@ -141,7 +142,8 @@ __device__ void plan_revisit(const PlanArgs& a, int r, int* s_part, double (*s_t
 __global__ void __launch_bounds__(kPlanThreads) plan_kernel(const __grid_constant__ PlanArgs a) {
     // The rebind grid may start launching now; it waits for this grid to
     // finish (griddepcontrol.wait) before it reads the plan.
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    pdl_allow();
+    pdl_wait();
     __shared__ int s_part[33 * 6];
     __shared__ double s_tab[3][kPosTable];
     uint32_t err = 0;
@@ -183,8 +185,7 @@ cudaError_t launch_plan(const PlanArgs& a, cudaStream_t stream) {
     const int seq_ctas = (a.n_seqs + kPlanThreads - 1) / kPlanThreads;
     int grid = a.n_revisits > seq_ctas ? a.n_revisits : seq_ctas;
     if (grid < 1) grid = 1;
-    plan_kernel<<<grid, kPlanThreads, 0, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(plan_kernel, dim3(unsigned(grid)), dim3(kPlanThreads), 0, stream, a);
 }
 
 }  // namespace prcr

@@ -27,6 +27,7 @@
 #include <cmath>
 
 #include "prcr_device.cuh"
+#include "prcr_pdl.cuh"
 
 namespace prcr {
 namespace {
@@ -61,6 +62,8 @@ __device__ __forceinline__ int swz(int c) { return c ^ ((c >> 3) & 1); }
 // for g = 1, 2 and 4, else 8 (heads h >= g skipped).
 template <int L, int G>
 __global__ void __launch_bounds__(256, 3) ads_logits_kernel(const __grid_constant__ SelectArgs a) {
+    pdl_allow();
+    pdl_wait();
     extern __shared__ __align__(16) float sm[];
     const int D = a.head_dim, P = D >> 1, Hq = a.n_q_heads, H = a.n_kv_heads, g = Hq / H;
     const int NV = P >> 3, M = a.n_tokens, T = a.tok_tile;
@@ -276,6 +279,8 @@ __device__ __forceinline__ void mma_1688_tf32(float (&c)[4], uint32_t a0, uint32
 // item covers all of them.
 template <int D, bool SPLIT>
 __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_constant__ SelectArgs a) {
+    pdl_allow();
+    pdl_wait();
     constexpr int P = D / 2, PL = P / 4, T = 64;
     constexpr int NW = PL / 8;  // 16-byte loads per half row per lane
     extern __shared__ __align__(16) float sm[];
@@ -411,6 +416,8 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
 
 // Softmax normaliser of each (sequence, query head) from the tiles' statistics.
 __global__ void __launch_bounds__(256) ads_norm_kernel(const __grid_constant__ SelectArgs a) {
+    pdl_allow();
+    pdl_wait();
     __shared__ float s_m[8], s_z[8];
     const int hq = blockIdx.x, b = blockIdx.y;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
@@ -440,6 +447,8 @@ __global__ void __launch_bounds__(256) ads_norm_kernel(const __grid_constant__ S
 
 // Relevance of every token: mean over the query heads of its softmax weight.
 __global__ void __launch_bounds__(256) ads_relevance_kernel(const __grid_constant__ SelectArgs a) {
+    pdl_allow();
+    pdl_wait();
     __shared__ float s_n[2 * kSelectMaxQHeads];
     const int b = blockIdx.y;
     const int Hq = a.n_q_heads, M = a.n_tokens;
@@ -493,6 +502,8 @@ __device__ __forceinline__ int block_scan(int v, int* s_warp, int* out_excl) {
 // registers; blockDim.x * PER >= n_tokens, blockDim.x a multiple of 32).
 template <int PER>
 __global__ void __launch_bounds__(1024) ads_select_kernel(const __grid_constant__ SelectArgs a) {
+    pdl_allow();
+    pdl_wait();
     __shared__ int s_warp[32];
     __shared__ unsigned int s_cnt[3 * 32];
     const int b = blockIdx.x;
@@ -608,8 +619,7 @@ cudaError_t launch_logits_g(const SelectArgs& a, int n_seqs, int sms, cudaStream
     const int64_t tiles = int64_t(n_seqs) * a.n_tiles;
     const int64_t resident = int64_t(sms) * (per_sm > 0 ? per_sm : 1);
     const unsigned grid = unsigned(tiles < resident ? tiles : resident);
-    ads_logits_kernel<L, G><<<grid, 256, smem, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(ads_logits_kernel<L, G>, dim3(grid), dim3(256), smem, stream, a);
 }
 
 template <int L>
@@ -646,9 +656,9 @@ cudaError_t launch_logits_mma(const SelectArgs& a, int n_seqs, int sms, cudaStre
         b.kh_per_item = (b.kh_per_item + 1) / 2;
     const int64_t items = int64_t(n_seqs) * a.n_tiles * ((H + b.kh_per_item - 1) / b.kh_per_item);
     const unsigned grid = unsigned(items < resident ? items : resident);
-    if (b.kh_per_item < H) ads_logits_mma_kernel<D, true><<<grid, 256, smem, stream>>>(b);
-    else ads_logits_mma_kernel<D, false><<<grid, 256, smem, stream>>>(b);
-    return cudaGetLastError();
+    return b.kh_per_item < H
+               ? launch_pdl(ads_logits_mma_kernel<D, true>, dim3(grid), dim3(256), smem, stream, b)
+               : launch_pdl(ads_logits_mma_kernel<D, false>, dim3(grid), dim3(256), smem, stream, b);
 }
 
 cudaError_t launch_select(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream) {
@@ -664,18 +674,19 @@ cudaError_t launch_select(const SelectArgs& a, int n_seqs, int sms, cudaStream_t
                              : launch_logits<16>(a, n_seqs, sms, stream));
     }
     if (e != cudaSuccess) return e;
-    ads_norm_kernel<<<dim3(a.n_q_heads, n_seqs, 1), 256, 0, stream>>>(a);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    ads_relevance_kernel<<<dim3((a.n_tokens + 255) / 256, n_seqs, 1), 256, 0, stream>>>(a);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    e = launch_pdl(ads_norm_kernel, dim3(a.n_q_heads, n_seqs, 1), dim3(256), 0, stream, a);
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(ads_relevance_kernel, dim3((a.n_tokens + 255) / 256, n_seqs, 1), dim3(256), 0,
+                   stream, a);
+    if (e != cudaSuccess) return e;
     const int M = a.n_tokens;
     // just enough warps for PER tokens per thread: fewer warps, cheaper rounds
     auto threads = [M](int per) { return int(((M + per - 1) / per + 31) / 32 * 32); };
-    if (M <= 4096) ads_select_kernel<4><<<n_seqs, threads(4), 0, stream>>>(a);
-    else if (M <= 8192) ads_select_kernel<8><<<n_seqs, threads(8), 0, stream>>>(a);
-    else if (M <= 16384) ads_select_kernel<16><<<n_seqs, threads(16), 0, stream>>>(a);
-    else ads_select_kernel<32><<<n_seqs, threads(32), 0, stream>>>(a);
-    return cudaGetLastError();
+    const dim3 grid(unsigned(n_seqs), 1, 1);
+    if (M <= 4096) return launch_pdl(ads_select_kernel<4>, grid, dim3(threads(4)), 0, stream, a);
+    if (M <= 8192) return launch_pdl(ads_select_kernel<8>, grid, dim3(threads(8)), 0, stream, a);
+    if (M <= 16384) return launch_pdl(ads_select_kernel<16>, grid, dim3(threads(16)), 0, stream, a);
+    return launch_pdl(ads_select_kernel<32>, grid, dim3(threads(32)), 0, stream, a);
 }
 
 }  // namespace prcr
