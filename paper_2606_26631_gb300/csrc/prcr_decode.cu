@@ -532,11 +532,13 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
             mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 1));
             mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 2));
             const float m_new = fmaxf(m_run, mx);
-            const float alpha = m_new == -INFINITY ? 1.0f : expf(m_run - m_new);
+            // arguments are <= 0: __expf's error (a few ulp) is far inside
+            // the float32 accumulation's
+            const float alpha = m_new == -INFINITY ? 1.0f : __expf(m_run - m_new);
             float ps = 0.0f;
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
-                v[i] = v[i] == -INFINITY ? 0.0f : expf(v[i] - m_new);
+                v[i] = v[i] == -INFINITY ? 0.0f : __expf(v[i] - m_new);
                 ps += v[i];
             }
             ps += __shfl_xor_sync(kFull, ps, 1);
