@@ -52,12 +52,17 @@ SHAPES = {
     "sel-d256": Workload(name="sel-d256", n_layers=1, n_kv_heads=2, head_dim=256,
                          sections=(40, 44, 44), n_seqs=2, grids=((2, 10, 13),), selection="random",
                          cache="contiguous", cur_pos=("uniform", 500, 900), extra=(1, 2, 1, 40)),
+    # 1500 tokens over 24 tiles of 64 (ragged last tile), 16 query heads
+    "sel-1500": Workload(name="sel-1500", n_layers=1, n_kv_heads=4, head_dim=128,
+                         sections=(16, 24, 24), n_seqs=2, grids=((1, 30, 50),), selection="random",
+                         cache="contiguous", cur_pos=("uniform", 2000, 9000), extra=(1, 1, 1, 40)),
 }
 
 
 @pytest.mark.parametrize("name,Hq,k,layer", [("qwen25vl-7b", 28, 64, 5), ("qwen3vl-8b", 32, 300, 35),
                                              ("tiny", 2, 16, 1), ("qwen2vl-2b", 4, 100, 20),
-                                             ("sel-odd", 9, 20, 1), ("sel-d256", 4, 30, 0)])
+                                             ("sel-odd", 9, 20, 1), ("sel-d256", 4, 30, 0),
+                                             ("sel-1500", 16, 200, 0)])
 def test_select_parity(name, Hq, k, layer):
     wl = SHAPES.get(name) or get(name)
     batch = make_batch(wl, device=DEV)
