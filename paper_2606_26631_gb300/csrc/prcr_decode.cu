@@ -678,6 +678,49 @@ __global__ void __launch_bounds__(256) decode_merge_kernel(const __grid_constant
     }
 }
 
+// Merge for at most 32 chunks: one warp per (sequence, layer, query head).
+// Lane s holds chunk s's maximum and sum (one round trip), the maximum, the
+// weights exp(m_s - M) and the denominator stay in registers (shuffles), and
+// lane i accumulates dimensions 2i, 2i + 1 (+ 64 j) over the chunks' rows
+// with eight rows requested at a time.
+__global__ void __launch_bounds__(128) decode_merge_warp_kernel(const __grid_constant__ DecodeArgs a,
+                                                                int64_t n_out) {
+    pdl_allow();
+    pdl_wait();  // the decode grid's partials
+    const int D = a.head_dim, S = a.splits, R = D + 2;
+    const int lane = threadIdx.x & 31;
+    const int64_t o_idx = int64_t(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (o_idx >= n_out) return;
+    const float* part = a.partial + o_idx * S * R;
+    const float ms = lane < S ? part[int64_t(lane) * R + D] : -INFINITY;
+    const float ls = lane < S ? part[int64_t(lane) * R + D + 1] : 0.0f;
+    float M = ms;
+#pragma unroll
+    for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, o));
+    const float w = ms == -INFINITY ? 0.0f : expf(ms - M);
+    float den = w * ls;
+#pragma unroll
+    for (int o = 16; o; o >>= 1) den += __shfl_xor_sync(kFull, den, o);
+    const float inv = den > 0.0f ? 1.0f / den : 0.0f;
+    for (int d0 = 2 * lane; d0 < D; d0 += 64) {
+        float2 acc = make_float2(0.0f, 0.0f);
+        for (int s0 = 0; s0 < S; s0 += 8) {
+            float2 x[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                x[u] = s0 + u < S ? *reinterpret_cast<const float2*>(part + int64_t(s0 + u) * R + d0)
+                                  : make_float2(0.0f, 0.0f);
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const float wu = __shfl_sync(kFull, w, (s0 + u) & 31);
+                acc.x = fmaf(wu, x[u].x, acc.x);
+                acc.y = fmaf(wu, x[u].y, acc.y);
+            }
+        }
+        *reinterpret_cast<float2*>(a.out + o_idx * D + d0) = make_float2(acc.x * inv, acc.y * inv);
+    }
+}
+
 template <int GP>
 cudaError_t launch_gp(const DecodeArgs& a, dim3 grid, size_t smem, cudaStream_t stream) {
     const dim3 block(kDecodeThreads);
@@ -721,7 +764,11 @@ cudaError_t launch_decode(const DecodeArgs& a, int gp, dim3 grid, size_t smem,
         e = gp <= 4 ? launch_gp<4>(a, grid, smem, stream) : launch_gp<8>(a, grid, smem, stream);
     }
     if (e != cudaSuccess || a.splits == 1) return e;
-    return launch_pdl(decode_merge_kernel, dim3(unsigned(int64_t(grid.z) * a.n_layers * a.n_q_heads)),
+    const int64_t n_out = int64_t(grid.z) * a.n_layers * a.n_q_heads;
+    if (a.splits <= 32)
+        return launch_pdl(decode_merge_warp_kernel, dim3(unsigned((n_out + 3) / 4)), dim3(128), 0,
+                          stream, a, n_out);
+    return launch_pdl(decode_merge_kernel, dim3(unsigned(n_out)),
                       dim3(a.head_dim < 256 ? a.head_dim : 256), 0, stream, a);
 }
 
