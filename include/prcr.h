@@ -16,7 +16,10 @@
  *    device; the caller owns and allocates all of it. The library never
  *    allocates, frees or synchronises; work is enqueued on `stream`
  *    (a cudaStream_t; NULL = the legacy default stream) and runs
- *    asynchronously.
+ *    asynchronously. Kernels are launched with programmatic stream
+ *    serialization: one may become resident while the preceding kernel on
+ *    the stream drains, but it reads and writes no memory before that
+ *    kernel has completed, so stream order is exactly that of plain launches.
  *  - K/V elements are bf16 (IEEE binary16-brain bit patterns). A token row is
  *    [n_kv_heads][head_dim] contiguous elements; strides between rows,
  *    layers, sequences and blocks are given in elements. Every row start must

@@ -35,8 +35,8 @@ def nvcc() -> str:
 
 def _inputs():
     deps = [os.path.join(CSRC, s) for s in SOURCES]
-    deps += [os.path.join(CSRC, "prcr_internal.h"), os.path.join(CSRC, "prcr_device.cuh"),
-             os.path.join(INCLUDE, "prcr.h"), __file__]
+    deps += [os.path.join(CSRC, h) for h in sorted(os.listdir(CSRC)) if h.endswith((".h", ".cuh"))]
+    deps += [os.path.join(INCLUDE, "prcr.h"), __file__]
     return deps
 
 
