@@ -45,6 +45,9 @@ Readings taken where the paper is silent (each is a named choice below):
   on m at one layer, softmax over the M visual tokens' position-bound keys
   RoPE(k_raw, p_m), averaged over the query heads; the K most relevant tokens
   are selected (ties to the lower index) and listed in ascending token order.
+  Second reading (``ads_relevance_cached``): the same attention computed
+  over the keys the decoder's position-bound cache holds for the visual
+  tokens (RoPE(k_raw, p_m) as stored, e.g. in bf16), only the query rotated.
 
 Parity pins for every function here live in tests/test_oracle_pins.py; every
 function is pinned (no function is "parity unpinned").
@@ -292,6 +295,28 @@ def ads_relevance(q_raw: np.ndarray, q_pos: int, k_raw_bits: np.ndarray, coords,
     k = position_bound_keys(k_raw_bits, coords, head_dim, sections, theta, layout)  # [M, H, D]
     H = k.shape[1]
     group = Hq // H
+    q = rope(q_raw, angles(np.full((Hq, 3), float(q_pos)), head_dim, sections, theta, layout))
+    r = np.zeros(k.shape[0])
+    for h in range(Hq):
+        lg = k[:, h // group, :] @ q[h] / np.sqrt(head_dim)
+        w = np.exp(lg - lg.max())
+        r += w / w.sum()
+    return r / Hq
+
+
+def ads_relevance_cached(q_raw: np.ndarray, q_pos: int, k_cached: np.ndarray, head_dim: int,
+                         sections, theta: float, layout: int = LAYOUT_SECTIONED) -> np.ndarray:
+    """Relevance read from the decoder's position-bound cache (second reading
+    of the attention-driven selection named in Sec. 2.1): k_cached [M, H, D]
+    holds the visual tokens' keys as that cache keeps them, already rotated at
+    their own coordinates (Eq. "historical_position_bound_kv"), so only the
+    query is rotated: r_m = mean over query heads h of
+    softmax_m(RoPE(q_h, (p,p,p)) . k_m / sqrt(D)), query head h reading KV
+    head h // (Hq / H)."""
+    q_raw = np.asarray(q_raw, dtype=np.float64)
+    k = np.asarray(k_cached, dtype=np.float64)
+    Hq = q_raw.shape[0]
+    group = Hq // k.shape[1]
     q = rope(q_raw, angles(np.full((Hq, 3), float(q_pos)), head_dim, sections, theta, layout))
     r = np.zeros(k.shape[0])
     for h in range(Hq):

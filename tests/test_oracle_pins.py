@@ -473,11 +473,47 @@ def pin_ads(o):
     assert list(sel) == [0, 3]
 
 
+def pin_ads_cached(o):
+    """Selection over the position-bound cache (second reading): against a
+    direct loop (query turned by complex exponentials, keys used as given);
+    relevance sums to 1; with keys rotated exactly at their coordinates it is
+    the raw-store relevance (the relative-angle identity of Eq.
+    "direct_reuse_score"); moving the query position and every key position
+    by the same shift changes nothing."""
+    rng = np.random.default_rng(41)
+    D, sec, th = 16, (2, 3, 3), 1e6
+    M, H, Hq = 10, 2, 6
+    kc = rng.standard_normal((M, H, D))
+    q = rng.standard_normal((Hq, D))
+    r = o.ads_relevance_cached(q, 57, kc, D, sec, th)
+    assert abs(r.sum() - 1.0) < 1e-12 and (r > 0).all()
+    P = D // 2
+    ref = np.zeros(M)
+    for h in range(Hq):
+        qz = [complex(q[h, i], q[h, i + P]) * cmath.exp(1j * 57 * th ** (-2.0 * i / D)) for i in range(P)]
+        lg = [sum(qz[i].real * kc[m, h // 3, i] + qz[i].imag * kc[m, h // 3, i + P] for i in range(P))
+              / math.sqrt(D) for m in range(M)]
+        mx = max(lg)
+        w = [math.exp(x - mx) for x in lg]
+        for m in range(M):
+            ref[m] += w[m] / sum(w) / Hq
+    assert np.allclose(r, ref, rtol=1e-10, atol=0)
+    kb = rng.integers(0x3C00, 0x4100, size=(M, H, D)).astype(np.uint16)
+    kb[..., 1::2] |= 0x8000
+    coords = np.array([(2, 7 + m // 5, 30 + m % 5) for m in range(M)])
+    kpb = o.position_bound_keys(kb, coords, D, sec, th)
+    assert np.allclose(o.ads_relevance_cached(q, 90, kpb, D, sec, th),
+                       o.ads_relevance(q, 90, kb, coords, D, sec, th), rtol=1e-10, atol=0)
+    kps = o.position_bound_keys(kb, coords + 500, D, sec, th)
+    assert np.allclose(o.ads_relevance_cached(q, 590, kps, D, sec, th),
+                       o.ads_relevance_cached(q, 90, kpb, D, sec, th), rtol=1e-9, atol=0)
+
+
 PINS = [pin_worked_rect4x4, pin_worked_rect2x2, pin_pcr_closed_forms, pin_degenerate_center,
         pin_other_modes, pin_plan_slots_and_continuity, pin_rope_closed_forms,
         pin_mrope_equal_axes_is_textbook, pin_mrope_sections, pin_rope_invariants,
         pin_bf16_helpers, pin_brute_force_2x2, pin_original_mode_is_position_bound_cache,
-        pin_prefill_capture, pin_decode_attention, pin_ads]
+        pin_prefill_capture, pin_decode_attention, pin_ads, pin_ads_cached]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -582,6 +618,18 @@ def _m_decode_query_unrotated(q_raw, q_pos, k_act, v_act, head_dim, sections, th
 
 
 _orig_select = O.ads_select
+_orig_rel_cached = O.ads_relevance_cached
+
+
+def _m_rel_cached_query_unrotated(q_raw, q_pos, k_cached, head_dim, sections, theta, layout=0):
+    return _orig_rel_cached(q_raw, 0, k_cached, head_dim, sections, theta, layout)
+
+
+def _m_rel_cached_head_modulo(q_raw, q_pos, k_cached, head_dim, sections, theta, layout=0):
+    H = k_cached.shape[1]
+    Hq = q_raw.shape[0]
+    perm = np.array([(hq % H) * (Hq // H) + hq // H for hq in range(Hq)])
+    return _orig_rel_cached(q_raw[perm], q_pos, k_cached, head_dim, sections, theta, layout)
 
 
 def _m_select_unsorted(rel, K):
@@ -612,6 +660,8 @@ MUTANTS = [
     ("decode_attention", _m_decode_query_unrotated),
     ("ads_select", _m_select_unsorted),
     ("ads_select", _m_select_ties_high),
+    ("ads_relevance_cached", _m_rel_cached_query_unrotated),
+    ("ads_relevance_cached", _m_rel_cached_head_modulo),
 ]
 
 
