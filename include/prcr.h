@@ -320,6 +320,35 @@ PRCR_API int prcr_select_topk(const prcr_rope_cfg* cfg, const prcr_store_desc* s
                               int32_t* seq_rev_off, int32_t* rev_tok_off, float* score_out,
                               void* workspace, size_t workspace_bytes, void* stream);
 
+/* prcr_select_topk_cached - the same selection (Sec. 2.1, Eq. 3) read from
+ * the decoder's position-bound cache instead of the raw store: the visual
+ * tokens' keys there are already rotated at their own coordinates (Eq.
+ * "historical_position_bound_kv"; e.g. the cache rows prcr_prefill_capture
+ * wrote), so only the trigger query is rotated. Relevance of visual token m
+ * of sequence b: per query head h, softmax over the n_tokens tokens of
+ *   RoPE(q[b][h], (p, p, p)) . K_cache[b][layer][img_slot0[b] + m][h / group] / sqrt(D),
+ * p = q_pos[b], averaged over the heads (with keys rotated exactly this is
+ * prcr_select_topk's relevance; the cache's bf16 rounding of the keys is the
+ * only difference). Token m is the image's m-th token in the order its rows
+ * occupy slots img_slot0[b] .. img_slot0[b] + n_tokens - 1 (contiguous cache,
+ * or paged through the block table), the order prcr_prefill_capture and
+ * prcr_store_raw give the same token, so idx_out indexes the raw store too.
+ *   img_slot0   device int32 [n_seqs]  first cache slot of sequence b's image
+ *   status      device uint32 word: a token whose slot lies beyond the
+ *               sequence's capacity sets PRCR_ST_CAPACITY, one in an unmapped
+ *               block PRCR_ST_NO_BLOCK; such a token gets relevance 0 (the
+ *               selection of a sequence with no readable token is unspecified)
+ * Other arguments, outputs, limits and the workspace (prcr_select_workspace_size
+ * with the same n_seqs, n_q_heads, n_tokens) are those of prcr_select_topk;
+ * head_dim must be 64 or 128 (PRCR_EINVAL otherwise).                    */
+PRCR_API int prcr_select_topk_cached(const prcr_rope_cfg* cfg, const prcr_cache_desc* cache,
+                                     int32_t n_seqs, int32_t layer, int32_t n_q_heads,
+                                     int32_t n_tokens, const int32_t* img_slot0, const void* q,
+                                     const int64_t* q_pos, int32_t k, int32_t* idx_out,
+                                     int32_t* seq_rev_off, int32_t* rev_tok_off, float* score_out,
+                                     uint32_t* status, void* workspace, size_t workspace_bytes,
+                                     void* stream);
+
 /* prcr_next_text_pos - host helper: the position the next text token takes
  * after a revisit appended k_seq tokens to a sequence whose latest text token
  * is at p_txt: p_txt + 1 for PCR, ORIGINAL and UIR (Sec. 3.2, Sec. 3.3);

@@ -11,6 +11,6 @@ from ._binding import (  # noqa: F401
     ST_IDX_RANGE, ST_NO_BLOCK, ST_POS_RANGE, PrcrError, cache_contiguous, cache_paged,
     decode_attention, decode_workspace_size, lib,
     next_text_pos, outputs, plan, prefill_capture, rebind_apply, rebind_inject, rebind_inject_static,
-    revisit_batch, rope_cfg, select_topk, select_workspace_size,
+    revisit_batch, rope_cfg, select_topk, select_topk_cached, select_workspace_size,
     store_desc, store_raw, version, workspace_size)
 from .revisit import Revisit  # noqa: F401

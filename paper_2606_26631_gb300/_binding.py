@@ -27,7 +27,8 @@ CACHE_CONTIGUOUS, CACHE_PAGED = 0, 1
 EXPORTS = ("prcr_workspace_size", "prcr_rebind_inject", "prcr_plan", "prcr_rebind_apply",
            "prcr_store_raw", "prcr_next_text_pos", "prcr_error_string", "prcr_version",
            "prcr_rebind_inject_static", "prcr_prefill_capture", "prcr_decode_workspace_size",
-           "prcr_decode_attention", "prcr_select_workspace_size", "prcr_select_topk")
+           "prcr_decode_attention", "prcr_select_workspace_size", "prcr_select_topk",
+           "prcr_select_topk_cached")
 STATIC_MAX_TOKENS = 65536
 
 
@@ -106,6 +107,12 @@ def lib():
                                    C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p,
                                    C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p]
     L.prcr_select_topk.restype = C.c_int
+    L.prcr_select_topk_cached.argtypes = [P(RopeCfg), P(CacheDesc), C.c_int32, C.c_int32,
+                                          C.c_int32, C.c_int32, C.c_void_p, C.c_void_p,
+                                          C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p,
+                                          C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                          C.c_size_t, C.c_void_p]
+    L.prcr_select_topk_cached.restype = C.c_int
     L.prcr_next_text_pos.argtypes = [C.c_int64, C.c_int64, C.c_int32]
     L.prcr_next_text_pos.restype = C.c_int64
     L.prcr_error_string.argtypes = [C.c_int]
@@ -356,6 +363,30 @@ def select_topk(cfg, store, layer: int, q: torch.Tensor, q_pos: torch.Tensor, k:
                                 _ptr(score_out), workspace.data_ptr(),
                                 workspace.numel() * workspace.element_size(), _stream(stream))
     return _check(rc, "prcr_select_topk")
+
+
+def select_topk_cached(cfg, cache, layer: int, q: torch.Tensor, q_pos: torch.Tensor,
+                       img_slot0: torch.Tensor, n_tokens: int, k: int, idx_out: torch.Tensor,
+                       seq_rev_off: torch.Tensor, rev_tok_off: torch.Tensor, status: torch.Tensor,
+                       workspace: torch.Tensor, score_out: Optional[torch.Tensor] = None,
+                       stream=None):
+    """prcr_select_topk_cached: the selection read from the position-bound
+    cache `cache`; sequence b's n_tokens visual tokens occupy slots
+    img_slot0[b] .. (int32 [B]). Other arguments as select_topk; status is
+    the device status word (int32 [1])."""
+    if q.dtype != torch.bfloat16 or not q.is_contiguous():
+        raise TypeError("q must be a contiguous bfloat16 [B, Hq, D] tensor")
+    for name, t in (("idx_out", idx_out), ("seq_rev_off", seq_rev_off), ("rev_tok_off", rev_tok_off),
+                    ("img_slot0", img_slot0)):
+        if t.dtype != torch.int32 or not t.is_contiguous():
+            raise TypeError(f"{name} must be a contiguous int32 tensor")
+    rc = lib().prcr_select_topk_cached(C.byref(cfg), C.byref(cache), int(q.shape[0]), int(layer),
+                                       int(q.shape[1]), int(n_tokens), img_slot0.data_ptr(),
+                                       q.data_ptr(), q_pos.data_ptr(), int(k), idx_out.data_ptr(),
+                                       seq_rev_off.data_ptr(), rev_tok_off.data_ptr(),
+                                       _ptr(score_out), status.data_ptr(), workspace.data_ptr(),
+                                       workspace.numel() * workspace.element_size(), _stream(stream))
+    return _check(rc, "prcr_select_topk_cached")
 
 
 def next_text_pos(p_txt: int, k_seq: int, mode: int = MODE_PCR) -> int:

@@ -385,6 +385,63 @@ bool decode_shape_ok(const prcr_rope_cfg* cfg, int32_t n_q_heads) {
     return n_q_heads / cfg->n_kv_heads <= 8;
 }
 
+// Checks and fills what both selection entry points share: heads, k, the
+// output pointers and the workspace, laid out for token tiles of `tile`.
+int select_common(const prcr_rope_cfg* cfg, int32_t n_seqs, int32_t layer, int32_t n_q_heads,
+                  int32_t n_tokens, const void* q, const int64_t* q_pos, int32_t k,
+                  int32_t* idx_out, int32_t* seq_rev_off, int32_t* rev_tok_off, float* score_out,
+                  void* workspace, size_t workspace_bytes, int tile, SelectArgs& a) {
+    const int H = cfg->n_kv_heads;
+    if (n_seqs < 0 || layer < 0 || layer >= cfg->n_layers || n_q_heads < H || n_q_heads % H ||
+        n_q_heads / H > 8 || n_q_heads > kSelectMaxQHeads ||
+        int64_t(n_q_heads) * cfg->head_dim > PRCR_DECODE_MAX_Q_ELEMS ||
+        n_tokens > PRCR_SELECT_MAX_TOKENS || k < 1 || k > n_tokens)
+        return PRCR_EINVAL;
+    if (int64_t(n_seqs) * k > INT32_MAX) return PRCR_EINVAL;
+    if (n_seqs == 0) return PRCR_OK;
+    if (!q || !q_pos || !idx_out || !seq_rev_off || !rev_tok_off) return PRCR_EINVAL;
+    if (!aligned4(q) || !aligned8(q_pos) || !aligned4(idx_out) || !aligned4(seq_rev_off) ||
+        !aligned4(rev_tok_off) || (score_out && !aligned4(score_out)))
+        return PRCR_EALIGN;
+    if (!workspace || workspace_bytes < prcr_select_workspace_size(n_seqs, n_q_heads, n_tokens))
+        return PRCR_EWORKSPACE;
+    if (!aligned16(workspace)) return PRCR_EALIGN;
+    a.q = static_cast<const uint16_t*>(q);
+    a.q_pos = q_pos;
+    a.layer = layer;
+    a.n_tokens = n_tokens;
+    a.n_kv_heads = H;
+    a.n_q_heads = n_q_heads;
+    a.head_dim = cfg->head_dim;
+    a.k = k;
+    a.layout = cfg->layout;
+    a.sec_t = cfg->sections[0];
+    a.sec_h = cfg->sections[1];
+    a.sec_w = cfg->sections[2];
+    a.scale = float(1.0 / std::sqrt(double(cfg->head_dim)));
+    {
+        char* w = static_cast<char*>(workspace);
+        const int64_t Bn = n_seqs, Hn = n_q_heads, M = n_tokens;
+        a.n_seqs = n_seqs;
+        a.tok_tile = tile;
+        a.n_tiles = int32_t((M + tile - 1) / tile);
+        const int64_t max_tiles = (M + kSelectTokTile - 1) / kSelectTokTile;
+        a.logits = reinterpret_cast<float*>(w);
+        w += align256(size_t(4 * Bn * Hn * M));
+        a.tile_stats = reinterpret_cast<float*>(w);
+        w += align256(size_t(8 * Bn * Hn * max_tiles));
+        a.norm = reinterpret_cast<float*>(w);
+        w += align256(size_t(8 * Bn * Hn));
+        a.rel = reinterpret_cast<float*>(w);
+    }
+    a.score_out = score_out;
+    a.idx_out = idx_out;
+    a.rev_tok_off = rev_tok_off;
+    a.seq_rev_off = seq_rev_off;
+    copy_turn_freq(cfg, a.turn_freq);
+    return PRCR_OK;
+}
+
 }  // namespace
 }  // namespace prcr
 
@@ -600,67 +657,65 @@ int prcr_select_topk(const prcr_rope_cfg* cfg, const prcr_store_desc* store, int
     int rc = check_cfg(cfg);
     if (rc) return rc;
     if ((rc = check_store(cfg, store))) return rc;
-    const int H = cfg->n_kv_heads;
-    if (n_seqs < 0 || n_seqs > store->n_seqs || layer < 0 || layer >= cfg->n_layers ||
-        n_q_heads < H || n_q_heads % H || n_q_heads / H > 8 || n_q_heads > kSelectMaxQHeads ||
-        int64_t(n_q_heads) * cfg->head_dim > PRCR_DECODE_MAX_Q_ELEMS ||
-        store->n_tokens > PRCR_SELECT_MAX_TOKENS || k < 1 || k > store->n_tokens)
-        return PRCR_EINVAL;
-    if (int64_t(n_seqs) * k > INT32_MAX) return PRCR_EINVAL;
-    if (n_seqs == 0) return PRCR_OK;
-    if (!q || !q_pos || !idx_out || !seq_rev_off || !rev_tok_off) return PRCR_EINVAL;
-    if (!aligned4(q) || !aligned8(q_pos) || !aligned4(idx_out) || !aligned4(seq_rev_off) ||
-        !aligned4(rev_tok_off) || (score_out && !aligned4(score_out)))
-        return PRCR_EALIGN;
-    if (!workspace || workspace_bytes < prcr_select_workspace_size(n_seqs, n_q_heads, store->n_tokens))
-        return PRCR_EWORKSPACE;
-    if (!aligned16(workspace)) return PRCR_EALIGN;
+    if (n_seqs > store->n_seqs) return PRCR_EINVAL;
     SelectArgs a = {};
-    a.q = static_cast<const uint16_t*>(q);
-    a.q_pos = q_pos;
+    // token tiles of the logits kernel: 64 tokens (32 at head_dim 256, whose
+    // cos/sin rows are twice as long)
+    rc = select_common(cfg, n_seqs, layer, n_q_heads, store->n_tokens, q, q_pos, k, idx_out,
+                       seq_rev_off, rev_tok_off, score_out, workspace, workspace_bytes,
+                       cfg->head_dim > 128 ? 32 : 64, a);
+    if (rc || n_seqs == 0) return rc;
     a.store_k = static_cast<const uint16_t*>(store->k);
     a.store_seq_stride = store->seq_stride;
     a.store_layer_stride = store->layer_stride;
     a.store_token_stride = store->token_stride;
     a.coords = store->coords;
     a.coord_seq_stride = store->coord_seq_stride;
-    a.layer = layer;
-    a.n_tokens = store->n_tokens;
-    a.n_kv_heads = H;
-    a.n_q_heads = n_q_heads;
-    a.head_dim = cfg->head_dim;
-    a.k = k;
-    a.layout = cfg->layout;
-    a.sec_t = cfg->sections[0];
-    a.sec_h = cfg->sections[1];
-    a.sec_w = cfg->sections[2];
-    a.scale = float(1.0 / std::sqrt(double(cfg->head_dim)));
-    {
-        char* w = static_cast<char*>(workspace);
-        const int64_t Bn = n_seqs, Hn = n_q_heads, M = store->n_tokens;
-        // token tiles of the logits kernel: 64 tokens (32 at head_dim 256, whose
-        // cos/sin rows are twice as long)
-        const int tile = cfg->head_dim > 128 ? 32 : 64;
-        a.n_seqs = n_seqs;
-        a.tok_tile = tile;
-        a.n_tiles = int32_t((M + tile - 1) / tile);
-        const int64_t max_tiles = (M + kSelectTokTile - 1) / kSelectTokTile;
-        a.logits = reinterpret_cast<float*>(w);
-        w += align256(size_t(4 * Bn * Hn * M));
-        a.tile_stats = reinterpret_cast<float*>(w);
-        w += align256(size_t(8 * Bn * Hn * max_tiles));
-        a.norm = reinterpret_cast<float*>(w);
-        w += align256(size_t(8 * Bn * Hn));
-        a.rel = reinterpret_cast<float*>(w);
-    }
-    a.score_out = score_out;
-    a.idx_out = idx_out;
-    a.rev_tok_off = rev_tok_off;
-    a.seq_rev_off = seq_rev_off;
-    copy_turn_freq(cfg, a.turn_freq);
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return PRCR_ECUDA;
     return launch_select(a, n_seqs, sm_count(dev), static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? PRCR_OK
+               : PRCR_ECUDA;
+}
+
+int prcr_select_topk_cached(const prcr_rope_cfg* cfg, const prcr_cache_desc* cache, int32_t n_seqs,
+                            int32_t layer, int32_t n_q_heads, int32_t n_tokens,
+                            const int32_t* img_slot0, const void* q, const int64_t* q_pos, int32_t k,
+                            int32_t* idx_out, int32_t* seq_rev_off, int32_t* rev_tok_off,
+                            float* score_out, uint32_t* status, void* workspace,
+                            size_t workspace_bytes, void* stream) {
+    int rc = check_cfg(cfg);
+    if (rc) return rc;
+    if ((rc = check_cache(cfg, cache))) return rc;
+    if (n_seqs > cache->n_seqs || n_tokens < 1 ||
+        (cfg->head_dim != 64 && cfg->head_dim != 128))
+        return PRCR_EINVAL;
+    SelectArgs a = {};
+    // token tiles of 16: one warp's MMA tile of keys
+    rc = select_common(cfg, n_seqs, layer, n_q_heads, n_tokens, q, q_pos, k, idx_out, seq_rev_off,
+                       rev_tok_off, score_out, workspace, workspace_bytes, 16, a);
+    if (rc || n_seqs == 0) return rc;
+    if (!img_slot0 || !status) return PRCR_EINVAL;
+    if (!aligned4(img_slot0) || !aligned4(status)) return PRCR_EALIGN;
+    a.cache_k = static_cast<const uint16_t*>(cache->k);
+    a.cache_seq_stride = cache->seq_stride;
+    a.cache_layer_stride = cache->layer_stride;
+    a.cache_block_stride = cache->block_stride;
+    a.cache_slot_stride = cache->slot_stride;
+    a.cache_capacity = cache->kind == PRCR_CACHE_CONTIGUOUS
+                           ? int64_t(cache->max_slots)
+                           : int64_t(cache->bt_stride) * cache->block_size;
+    a.block_table = cache->block_table;
+    a.bt_stride = cache->bt_stride;
+    a.block_size = cache->kind == PRCR_CACHE_PAGED ? cache->block_size : 1;
+    a.n_blocks = cache->n_blocks;
+    a.cache_kind = cache->kind;
+    a.img_slot0 = img_slot0;
+    a.status = status;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return PRCR_ECUDA;
+    return launch_select_cached(a, n_seqs, sm_count(dev), static_cast<cudaStream_t>(stream)) ==
+                   cudaSuccess
                ? PRCR_OK
                : PRCR_ECUDA;
 }

@@ -257,10 +257,27 @@ struct SelectArgs {
     int32_t* idx_out;           // [B][k]
     int32_t* rev_tok_off;       // [B + 1]
     int32_t* seq_rev_off;       // [B + 1]
+    // keys from the position-bound cache (prcr_select_topk_cached)
+    const uint16_t* cache_k;
+    int64_t cache_seq_stride;   // contiguous
+    int64_t cache_layer_stride;
+    int64_t cache_block_stride; // paged
+    int64_t cache_slot_stride;
+    int64_t cache_capacity;     // slots per sequence
+    const int32_t* block_table;
+    int32_t bt_stride;
+    int32_t block_size;
+    int32_t n_blocks;
+    int32_t cache_kind;
+    const int32_t* img_slot0;   // [B] first slot of each sequence's image tokens
+    uint32_t* status;
     uint64_t turn_freq[kMaxPairs];  // pair i: round(inv_freq_i / (2 pi) * 2^64)
 };
 
 cudaError_t launch_select(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream);
+// the logits of the cached-key selection, then the same normaliser, relevance
+// and selection kernels
+cudaError_t launch_select_cached(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream);
 
 cudaError_t launch_decode(const DecodeArgs& a, int gp, dim3 grid, size_t smem,
                           cudaStream_t stream);

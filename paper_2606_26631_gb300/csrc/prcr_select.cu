@@ -414,6 +414,161 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
     }
 }
 
+// Logits of the selection over the position-bound cache (head_dim 64 or
+// 128). The cache already holds each visual token's key rotated at its own
+// coordinates, so only the query is turned, once, at (p, p, p); the step is
+// then a plain product with the cached rows and runs at memory speed. A
+// warp's work item is (sequence b, KV head kh, tile of 16 tokens); items run
+// (b, kh) major with tiles fastest and a warp takes a contiguous run of them,
+// so it rotates its group's queries once per (b, kh). As in the decode
+// kernel: S (16 rows = the group's query heads, rows >= g zero; two tiles of
+// 8 tokens) = Q K^T over D/16 k-steps of mma.sync m16n8k16, the bf16 keys
+// exact operands and the float32 query (pre-scaled by 1/sqrt(D)) entered as a
+// bf16 head and a bf16 remainder; the key dimensions are permuted per lane
+// group so that a lane loads its token's 64 contiguous bytes straight into B
+// fragments. The next item's rows are requested right after this item's
+// MMAs. An item writes its 16 logits per head and the tile's (max, sum of
+// exp) per head; a token without a readable row gets logit -inf.
+template <int D>
+__global__ void __launch_bounds__(256, 2) ads_logits_cache_kernel(const __grid_constant__ SelectArgs a) {
+    pdl_allow();
+    constexpr int KS = D / 16, LV = D / 32, P = D / 2;
+    extern __shared__ __align__(16) float sm[];
+    const int Hq = a.n_q_heads, H = a.n_kv_heads, g = Hq / H, M = a.n_tokens, NT = a.n_tiles;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, gid = lane >> 2, t = lane & 3;
+    float* qw = sm + warp * g * D;  // this warp's rotated query rows
+    const int64_t n_items = int64_t(a.n_seqs) * H * NT;
+    const int64_t n_warps = int64_t(gridDim.x) * (blockDim.x >> 5);
+    const int64_t gw = int64_t(blockIdx.x) * (blockDim.x >> 5) + warp;
+    const int64_t i_beg = n_items * gw / n_warps, i_end = n_items * (gw + 1) / n_warps;
+    uint32_t err = 0;
+    pdl_wait();
+
+    // element offset of KV head kh's key row for token m0 + (lane & 15) of
+    // `item`, or -1 (past the end, or no readable row)
+    auto row_of = [&](int64_t item) -> int64_t {
+        const int64_t bk = item / NT;
+        const int j = int(item - bk * NT);
+        const int b = int(bk / H), kh = int(bk - int64_t(b) * H);
+        const int m = 16 * j + (lane & 15);
+        if (m >= M) return -1;
+        const int64_t slot = int64_t(a.img_slot0[b]) + m;
+        if (slot < 0 || slot >= a.cache_capacity) {
+            err |= PRCR_ST_CAPACITY;
+            return -1;
+        }
+        int64_t row;
+        if (a.cache_kind == PRCR_CACHE_CONTIGUOUS) {
+            row = int64_t(b) * a.cache_seq_stride + slot * a.cache_slot_stride;
+        } else {
+            const int64_t lb = slot / a.block_size;
+            const int32_t blk = a.block_table[int64_t(b) * a.bt_stride + lb];
+            if (blk < 0 || blk >= a.n_blocks) {
+                err |= PRCR_ST_NO_BLOCK;
+                return -1;
+            }
+            row = int64_t(blk) * a.cache_block_stride + (slot - lb * a.block_size) * a.cache_slot_stride;
+        }
+        return row + int64_t(a.layer) * a.cache_layer_stride + int64_t(kh) * D;
+    };
+    uint4 kn[2][LV];
+    uint32_t mask_n = 0u;
+    auto fetch = [&](int64_t item) {
+        const int64_t row = row_of(item);
+        mask_n = __ballot_sync(0xffffffffu, row >= 0) & 0xffffu;
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt) {
+            const int64_t rr = __shfl_sync(0xffffffffu, row, nt * 8 + gid);
+#pragma unroll
+            for (int u = 0; u < LV; ++u)
+                kn[nt][u] = rr >= 0 ? ld_stream(a.cache_k + rr + t * (D / 4) + 8 * u)
+                                    : make_uint4(0u, 0u, 0u, 0u);
+        }
+    };
+
+    uint32_t qh[KS][2], ql[KS][2];
+    int64_t cur_bk = -1;
+    if (i_beg < i_end) fetch(i_beg);
+    for (int64_t item = i_beg; item < i_end; ++item) {
+        const int64_t bk = item / NT;
+        const int j = int(item - bk * NT);
+        const int b = int(bk / H), kh = int(bk - int64_t(b) * H);
+        if (bk != cur_bk) {
+            // the group's queries turned at (p, p, p), pre-scaled, as A fragments
+            const int64_t p = a.q_pos[b];
+            const uint16_t* qg = a.q + (int64_t(b) * Hq + kh * g) * D;
+            for (int i = lane; i < P; i += 32) {
+                float sn, cs;
+                sincos_turns(double(p), a.turn_freq[i], &sn, &cs);
+                for (int h = 0; h < g; ++h) {
+                    const float x = __uint_as_float(uint32_t(qg[h * D + i]) << 16);
+                    const float y = __uint_as_float(uint32_t(qg[h * D + i + P]) << 16);
+                    qw[h * D + i] = fmaf(x, cs, -y * sn) * a.scale;
+                    qw[h * D + i + P] = fmaf(y, cs, x * sn) * a.scale;
+                }
+            }
+            __syncwarp();
+            const bool hv = gid < g;
+            const float* qr = qw + (hv ? gid : 0) * D + t * (D / 4);
+#pragma unroll
+            for (int k = 0; k < KS; ++k) {
+                const float x0 = hv ? qr[4 * k] : 0.0f, x1 = hv ? qr[4 * k + 1] : 0.0f;
+                const float x2 = hv ? qr[4 * k + 2] : 0.0f, x3 = hv ? qr[4 * k + 3] : 0.0f;
+                split_bf16x2(x0, x1, qh[k][0], ql[k][0]);
+                split_bf16x2(x2, x3, qh[k][1], ql[k][1]);
+            }
+            __syncwarp();  // qw is rewritten for the next (b, kh)
+            cur_bk = bk;
+        }
+        const uint32_t mask = mask_n;
+        float sc[2][4];
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt) {
+            sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.0f;
+#pragma unroll
+            for (int k = 0; k < KS; ++k) {
+                const uint4& w = kn[nt][k >> 1];
+                const uint32_t b0 = (k & 1) ? w.z : w.x;
+                const uint32_t b1 = (k & 1) ? w.w : w.y;
+                mma_16816(sc[nt], qh[k][0], 0u, qh[k][1], 0u, b0, b1);
+                mma_16816(sc[nt], ql[k][0], 0u, ql[k][1], 0u, b0, b1);
+            }
+        }
+        if (item + 1 < i_end) fetch(item + 1);
+
+        // head row gid at tokens 2t, 2t + 1 (tile 0) and 8 + 2t, 9 + 2t (tile 1)
+        float v[4] = {sc[0][0], sc[0][1], sc[1][0], sc[1][1]};
+        const int sl[4] = {2 * t, 2 * t + 1, 8 + 2 * t, 9 + 2 * t};
+        float mx = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            if (!((mask >> sl[i]) & 1u)) v[i] = -INFINITY;
+            mx = fmaxf(mx, v[i]);
+        }
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+        float z = 0.0f;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) z += v[i] == -INFINITY ? 0.0f : expf(v[i] - mx);
+        z += __shfl_xor_sync(0xffffffffu, z, 1);
+        z += __shfl_xor_sync(0xffffffffu, z, 2);
+        if (gid < g) {
+            const int hq = kh * g + gid;
+            const int m0 = 16 * j;
+            float* lg = a.logits + (int64_t(b) * Hq + hq) * M + m0;
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                if (m0 + sl[i] < M) lg[sl[i]] = v[i];
+            if (t == 0) {
+                float* ts = a.tile_stats + ((int64_t(b) * Hq + hq) * NT + j) * 2;
+                ts[0] = mx;
+                ts[1] = mx == -INFINITY ? 0.0f : z;
+            }
+        }
+    }
+    if (err) atomicOr(a.status, err);
+}
+
 // Softmax normaliser of each (sequence, query head) from the tiles' statistics.
 __global__ void __launch_bounds__(256) ads_norm_kernel(const __grid_constant__ SelectArgs a) {
     pdl_allow();
@@ -661,6 +816,23 @@ cudaError_t launch_logits_mma(const SelectArgs& a, int n_seqs, int sms, cudaStre
                : launch_pdl(ads_logits_mma_kernel<D, false>, dim3(grid), dim3(256), smem, stream, b);
 }
 
+// The normalisers, relevances and selection after a logits kernel.
+static cudaError_t launch_select_tail(const SelectArgs& a, int n_seqs, cudaStream_t stream) {
+    cudaError_t e = launch_pdl(ads_norm_kernel, dim3(a.n_q_heads, n_seqs, 1), dim3(256), 0, stream, a);
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(ads_relevance_kernel, dim3((a.n_tokens + 255) / 256, n_seqs, 1), dim3(256), 0,
+                   stream, a);
+    if (e != cudaSuccess) return e;
+    const int M = a.n_tokens;
+    // just enough warps for PER tokens per thread: fewer warps, cheaper rounds
+    auto threads = [M](int per) { return int(((M + per - 1) / per + 31) / 32 * 32); };
+    const dim3 grid(unsigned(n_seqs), 1, 1);
+    if (M <= 4096) return launch_pdl(ads_select_kernel<4>, grid, dim3(threads(4)), 0, stream, a);
+    if (M <= 8192) return launch_pdl(ads_select_kernel<8>, grid, dim3(threads(8)), 0, stream, a);
+    if (M <= 16384) return launch_pdl(ads_select_kernel<16>, grid, dim3(threads(16)), 0, stream, a);
+    return launch_pdl(ads_select_kernel<32>, grid, dim3(threads(32)), 0, stream, a);
+}
+
 cudaError_t launch_select(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream) {
     cudaError_t e;
     if (a.head_dim == 128 && a.tok_tile == 64) {
@@ -674,19 +846,23 @@ cudaError_t launch_select(const SelectArgs& a, int n_seqs, int sms, cudaStream_t
                              : launch_logits<16>(a, n_seqs, sms, stream));
     }
     if (e != cudaSuccess) return e;
-    e = launch_pdl(ads_norm_kernel, dim3(a.n_q_heads, n_seqs, 1), dim3(256), 0, stream, a);
+    return launch_select_tail(a, n_seqs, stream);
+}
+
+cudaError_t launch_select_cached(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream) {
+    const int g = a.n_q_heads / a.n_kv_heads;
+    const size_t smem = size_t(8) * g * a.head_dim * sizeof(float);  // 8 warps
+    auto k = a.head_dim == 64 ? ads_logits_cache_kernel<64> : ads_logits_cache_kernel<128>;
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    int per_sm = 0;
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, 256, smem);
     if (e != cudaSuccess) return e;
-    e = launch_pdl(ads_relevance_kernel, dim3((a.n_tokens + 255) / 256, n_seqs, 1), dim3(256), 0,
-                   stream, a);
+    const int64_t items = int64_t(n_seqs) * a.n_kv_heads * a.n_tiles;
+    const int64_t ctas = (items + 7) / 8;
+    const int64_t resident = int64_t(sms) * (per_sm > 0 ? per_sm : 1);
+    e = launch_pdl(k, dim3(unsigned(ctas < resident ? ctas : resident)), dim3(256), smem, stream, a);
     if (e != cudaSuccess) return e;
-    const int M = a.n_tokens;
-    // just enough warps for PER tokens per thread: fewer warps, cheaper rounds
-    auto threads = [M](int per) { return int(((M + per - 1) / per + 31) / 32 * 32); };
-    const dim3 grid(unsigned(n_seqs), 1, 1);
-    if (M <= 4096) return launch_pdl(ads_select_kernel<4>, grid, dim3(threads(4)), 0, stream, a);
-    if (M <= 8192) return launch_pdl(ads_select_kernel<8>, grid, dim3(threads(8)), 0, stream, a);
-    if (M <= 16384) return launch_pdl(ads_select_kernel<16>, grid, dim3(threads(16)), 0, stream, a);
-    return launch_pdl(ads_select_kernel<32>, grid, dim3(threads(32)), 0, stream, a);
+    return launch_select_tail(a, n_seqs, stream);
 }
 
 }  // namespace prcr
