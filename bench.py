@@ -69,6 +69,9 @@ def parse():
                          "attention-driven selection of the revisited set; pipeline: select, "
                          "rebind+inject and the first decode step of one revisit, end to end")
     ap.add_argument("--seqs", type=int, default=0, help="capture/decode: sequences (0 = workload's)")
+    ap.add_argument("--select-source", choices=["raw", "cache"], default="raw",
+                    help="select / pipeline: rank from the raw store (prcr_select_topk) or from "
+                         "the position-bound cache (prcr_select_topk_cached)")
     ap.add_argument("--layers", type=int, default=0,
                     help="select: build the store with this many layers (0 = workload's); "
                          "the selection reads the last one")
@@ -667,10 +670,36 @@ def run_select_path(args):
     rto = torch.empty(B + 1, dtype=torch.int32, device=dev)
     ws = torch.empty(prcr.select_workspace_size(B, Hq, M), dtype=torch.uint8, device=dev)
 
-    def step():
-        prcr.select_topk(cfg, sd, layer, q, batch.p_txt, k, idx, sro, rto, ws)
+    if args.select_source == "raw":
+        def step():
+            prcr.select_topk(cfg, sd, layer, q, batch.p_txt, k, idx, sro, rto, ws)
+    else:
+        # the image tokens' keys as a one-layer position-bound cache laid out
+        # like the workload's cache (the store's keys serve as its values)
+        img0 = torch.zeros(B, dtype=torch.int32, device=dev)
+        cfg1 = prcr.rope_cfg(1, H, D, wl.sections, wl.theta)
+        status = torch.zeros(1, dtype=torch.int32, device=dev)
+        if batch.paged:
+            bs = wl.block_size
+            nblk = (M + bs - 1) // bs
+            perm = torch.randperm(B * nblk, device=dev,
+                                  generator=torch.Generator(device=dev).manual_seed(4))
+            bt = perm.to(torch.int32).view(B, nblk).contiguous()
+            ck = torch.empty((1, B * nblk, bs, H, D), dtype=torch.bfloat16, device=dev)
+            flat = ck.view(B * nblk * bs, H, D)
+            for b in range(B):
+                s_ = torch.arange(M, device=dev)
+                flat[bt[b][s_ // bs].long() * bs + s_ % bs] = batch.store_k[b, layer]
+            cd = prcr.cache_paged(ck, ck, bt)
+        else:
+            ck = batch.store_k[:, layer:layer + 1].clone()
+            cd = prcr.cache_contiguous(ck, ck)
 
-    nbytes = B * M * H * D * 2  # the layer's raw keys, read once
+        def step():
+            prcr.select_topk_cached(cfg1, cd, 0, q, batch.p_txt, img0, M, k, idx, sro, rto, status,
+                                    ws)
+
+    nbytes = B * M * H * D * 2  # the layer's keys, read once
     launched = kernel_launches(step)
     flush = L2Flush(dev, args.flush, nbytes)
     ms, clk = _timed(step, args.steps, args.warmup, local, flush)
@@ -678,16 +707,16 @@ def run_select_path(args):
     peak, kind = measured_peaks()
     value = nbytes * args.steps / t / 1e9
     print(json.dumps(dict(
-        metric="selection GB/s (raw keys read)", value=value, unit=UNIT, n_gpus=1,
+        metric=f"selection GB/s ({args.select_source} keys read)", value=value, unit=UNIT, n_gpus=1,
         steps=args.steps, warmup=args.warmup, ms_per_step=1e3 * t / args.steps,
         us_per_sequence=1e6 * t / args.steps / B, higher_is_better=True, scaling="weak",
         vs_baseline=None, dtype="f32", io_dtype="bf16", data="synthetic",
         config=dict(workload=wl.name, batch=B, tokens_per_seq=M, n_q_heads=Hq, k=k, layer=layer,
-                    bytes_per_step=nbytes, l2=flush.describe(nbytes)),
+                    source=args.select_source, bytes_per_step=nbytes, l2=flush.describe(nbytes)),
         roofline=dict(bound="hbm", achieved=value, peak=peak, unit="GB/s", frac=value / peak,
                       traffic=None, kernel="ads_*_kernel (whole selection step)",
                       peak_kind=f"{kind} copy (hbm_gbs)"),
-        **_launch_keys(launched, 5, args.steps), clocks=clk)), flush=True)
+        **_launch_keys(launched, 4, args.steps), clocks=clk)), flush=True)
 
 
 def run_pipeline_path(args):
@@ -729,8 +758,20 @@ def run_pipeline_path(args):
     nws = prcr.decode_workspace_size(cfg, B, Hq, max_len)
     ws_dec = torch.empty(max(nws, 16), dtype=torch.uint8, device=dev)
 
-    def select():
-        prcr.select_topk(cfg, sd, nL - 1, q_sel, batch.p_txt, k, idx, sro, rto, ws_sel)
+    if args.select_source == "raw":
+        def select():
+            prcr.select_topk(cfg, sd, nL - 1, q_sel, batch.p_txt, k, idx, sro, rto, ws_sel)
+    else:
+        # ranked from the cache: the image's position-bound rows taken to be
+        # the first M context slots (their values are the context data)
+        if int(batch.cache_len_in.min().item()) < M:
+            raise SystemExit("--select-source cache needs at least n_tokens context slots")
+        img0 = torch.zeros(B, dtype=torch.int32, device=dev)
+        sstat = torch.zeros(1, dtype=torch.int32, device=dev)
+
+        def select():
+            prcr.select_topk_cached(cfg, rv.cache, nL - 1, q_sel, batch.p_txt, img0, M, k, idx, sro,
+                                    rto, sstat, ws_sel)
 
     def decode():
         prcr.decode_attention(cfg, rv.cache, q_dec, rv.next_pos, rv.cache_len_out, max_len, out,
@@ -797,6 +838,7 @@ def run_pipeline_path(args):
         ms_per_step=statistics.mean(total) / 1e3, higher_is_better=False, scaling="weak",
         vs_baseline=None, dtype="f32", io_dtype="bf16", data="synthetic",
         config=dict(workload=wl.name, batch=B, tokens_per_seq=M, k=k, n_q_heads=Hq, n_layers=nL,
+                    select_source=args.select_source,
                     context_slots=int(batch.cache_len_in.max().item()), rebind_bytes=nbytes,
                     l2=flush.describe(nbytes)),
         timing="one CUDA graph per step (stages not timed separately)" if args.graph

@@ -420,14 +420,15 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
 // then a plain product with the cached rows and runs at memory speed. A
 // warp's work item is (sequence b, KV head kh, tile of 16 tokens); items run
 // (b, kh) major with tiles fastest and a warp takes a contiguous run of them,
-// so it rotates its group's queries once per (b, kh). As in the decode
-// kernel: S (16 rows = the group's query heads, rows >= g zero; two tiles of
-// 8 tokens) = Q K^T over D/16 k-steps of mma.sync m16n8k16, the bf16 keys
-// exact operands and the float32 query (pre-scaled by 1/sqrt(D)) entered as a
-// bf16 head and a bf16 remainder; the key dimensions are permuted per lane
-// group so that a lane loads its token's 64 contiguous bytes straight into B
-// fragments. The next item's rows are requested right after this item's
-// MMAs. An item writes its 16 logits per head and the tile's (max, sum of
+// so it rotates its group's queries once per (b, kh). S^T (16 rows = the
+// item's tokens; 8 columns = the group's query heads, columns >= g zero) =
+// K Q^T over D/16 k-steps of mma.sync m16n8k16: the bf16 keys are exact
+// operands and the float32 query (pre-scaled by 1/sqrt(D)) enters as a bf16
+// head and a bf16 remainder (two MMAs per k-step). The key dimensions are
+// permuted per lane group so that a lane loads its two tokens' 64 contiguous
+// bytes each straight into A fragments. The next item's rows are loaded
+// right after this item's MMAs, the rows of the one after that requested
+// into L2. An item writes its 16 logits per head and the tile's (max, sum of
 // exp) per head; a token without a readable row gets logit -inf.
 template <int D>
 __global__ void __launch_bounds__(256, 2) ads_logits_cache_kernel(const __grid_constant__ SelectArgs a) {
@@ -444,37 +445,59 @@ __global__ void __launch_bounds__(256, 2) ads_logits_cache_kernel(const __grid_c
     uint32_t err = 0;
     pdl_wait();
 
-    // element offset of KV head kh's key row for token m0 + (lane & 15) of
-    // `item`, or -1 (past the end, or no readable row)
-    auto row_of = [&](int64_t item) -> int64_t {
-        const int64_t bk = item / NT;
-        const int j = int(item - bk * NT);
-        const int b = int(bk / H), kh = int(bk - int64_t(b) * H);
-        const int m = 16 * j + (lane & 15);
+    // a work item as (sequence, KV head, tile); a warp's items are consecutive,
+    // so they are advanced in place rather than divided out of the index
+    struct Item {
+        int b, kh, j;
+    };
+    auto advance = [&](Item& x) {
+        if (++x.j == NT) {
+            x.j = 0;
+            if (++x.kh == H) {
+                x.kh = 0;
+                ++x.b;
+            }
+        }
+    };
+    // element offset of the item's key row for token 16 j + (lane & 15), or -1
+    // (past the end, or no readable row)
+    auto row_of = [&](const Item& x) -> int64_t {
+        const int m = 16 * x.j + (lane & 15);
         if (m >= M) return -1;
-        const int64_t slot = int64_t(a.img_slot0[b]) + m;
+        const int64_t slot = int64_t(a.img_slot0[x.b]) + m;
         if (slot < 0 || slot >= a.cache_capacity) {
             err |= PRCR_ST_CAPACITY;
             return -1;
         }
         int64_t row;
         if (a.cache_kind == PRCR_CACHE_CONTIGUOUS) {
-            row = int64_t(b) * a.cache_seq_stride + slot * a.cache_slot_stride;
+            row = int64_t(x.b) * a.cache_seq_stride + slot * a.cache_slot_stride;
         } else {
-            const int64_t lb = slot / a.block_size;
-            const int32_t blk = a.block_table[int64_t(b) * a.bt_stride + lb];
+            // block index and offset by a 32-bit division when the slot fits
+            // in 31 bits (a 64-bit division costs several times as many
+            // instructions as the rest of a row lookup)
+            int64_t lb, off;
+            if (slot <= INT32_MAX) {
+                const uint32_t us = uint32_t(slot), ubs = uint32_t(a.block_size);
+                lb = us / ubs;
+                off = us - uint32_t(lb) * ubs;
+            } else {
+                lb = slot / a.block_size;
+                off = slot - lb * a.block_size;
+            }
+            const int32_t blk = a.block_table[int64_t(x.b) * a.bt_stride + lb];
             if (blk < 0 || blk >= a.n_blocks) {
                 err |= PRCR_ST_NO_BLOCK;
                 return -1;
             }
-            row = int64_t(blk) * a.cache_block_stride + (slot - lb * a.block_size) * a.cache_slot_stride;
+            row = int64_t(blk) * a.cache_block_stride + off * a.cache_slot_stride;
         }
-        return row + int64_t(a.layer) * a.cache_layer_stride + int64_t(kh) * D;
+        return row + int64_t(a.layer) * a.cache_layer_stride + int64_t(x.kh) * D;
     };
     uint4 kn[2][LV];
     uint32_t mask_n = 0u;
-    auto fetch = [&](int64_t item) {
-        const int64_t row = row_of(item);
+    auto fetch = [&](const Item& x) {
+        const int64_t row = row_of(x);
         mask_n = __ballot_sync(0xffffffffu, row >= 0) & 0xffffu;
 #pragma unroll
         for (int nt = 0; nt < 2; ++nt) {
@@ -485,15 +508,35 @@ __global__ void __launch_bounds__(256, 2) ads_logits_cache_kernel(const __grid_c
                                     : make_uint4(0u, 0u, 0u, 0u);
         }
     };
+    // the rows of the item after next are requested into L2 (lanes 0..15,
+    // one token row each), so that its fetch finds them there
+    auto request = [&](const Item& x) {
+        const int64_t row = row_of(x);
+        if (lane < 16 && row >= 0) {
+            const char* p = reinterpret_cast<const char*>(a.cache_k + row);
+#pragma unroll
+            for (int o = 0; o < D * 2; o += 128) prefetch_l2(p + o);
+        }
+    };
 
     uint32_t qh[KS][2], ql[KS][2];
-    int64_t cur_bk = -1;
-    if (i_beg < i_end) fetch(i_beg);
-    for (int64_t item = i_beg; item < i_end; ++item) {
-        const int64_t bk = item / NT;
-        const int j = int(item - bk * NT);
-        const int b = int(bk / H), kh = int(bk - int64_t(b) * H);
-        if (bk != cur_bk) {
+    int cur_b = -1, cur_kh = -1;
+    Item cur, nxt, pf;
+    {
+        const int64_t bk = i_beg / NT;
+        cur.j = int(i_beg - bk * NT);
+        cur.b = int(bk / H);
+        cur.kh = int(bk - int64_t(cur.b) * H);
+    }
+    nxt = cur;
+    advance(nxt);
+    pf = nxt;
+    advance(pf);
+    if (i_beg < i_end) fetch(cur);
+    if (i_beg + 1 < i_end) request(nxt);
+    for (int64_t left = i_end - i_beg; left > 0; --left) {
+        const int b = cur.b, kh = cur.kh, j = cur.j;
+        if (b != cur_b || kh != cur_kh) {
             // the group's queries turned at (p, p, p), pre-scaled, as A fragments
             const int64_t p = a.q_pos[b];
             const uint16_t* qg = a.q + (int64_t(b) * Hq + kh * g) * D;
@@ -518,53 +561,64 @@ __global__ void __launch_bounds__(256, 2) ads_logits_cache_kernel(const __grid_c
                 split_bf16x2(x2, x3, qh[k][1], ql[k][1]);
             }
             __syncwarp();  // qw is rewritten for the next (b, kh)
-            cur_bk = bk;
+            cur_b = b;
+            cur_kh = kh;
         }
+        // S^T (16 tokens x 8 columns = the group's query heads, columns >= g
+        // zero) = K Q^T: rows gid (kn[0]) and gid + 8 (kn[1]) are this lane's
+        // tokens, and the query fragments serve as the B operand unchanged
         const uint32_t mask = mask_n;
-        float sc[2][4];
+        float c[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-        for (int nt = 0; nt < 2; ++nt) {
-            sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.0f;
-#pragma unroll
-            for (int k = 0; k < KS; ++k) {
-                const uint4& w = kn[nt][k >> 1];
-                const uint32_t b0 = (k & 1) ? w.z : w.x;
-                const uint32_t b1 = (k & 1) ? w.w : w.y;
-                mma_16816(sc[nt], qh[k][0], 0u, qh[k][1], 0u, b0, b1);
-                mma_16816(sc[nt], ql[k][0], 0u, ql[k][1], 0u, b0, b1);
-            }
+        for (int k = 0; k < KS; ++k) {
+            const uint4& w0 = kn[0][k >> 1];
+            const uint4& w1 = kn[1][k >> 1];
+            const uint32_t a0 = (k & 1) ? w0.z : w0.x, a2 = (k & 1) ? w0.w : w0.y;
+            const uint32_t a1 = (k & 1) ? w1.z : w1.x, a3 = (k & 1) ? w1.w : w1.y;
+            mma_16816(c, a0, a1, a2, a3, qh[k][0], qh[k][1]);
+            mma_16816(c, a0, a1, a2, a3, ql[k][0], ql[k][1]);
         }
-        if (item + 1 < i_end) fetch(item + 1);
+        if (left > 1) fetch(nxt);
+        if (left > 2) request(pf);
 
-        // head row gid at tokens 2t, 2t + 1 (tile 0) and 8 + 2t, 9 + 2t (tile 1)
-        float v[4] = {sc[0][0], sc[0][1], sc[1][0], sc[1][1]};
-        const int sl[4] = {2 * t, 2 * t + 1, 8 + 2 * t, 9 + 2 * t};
-        float mx = -INFINITY;
+        // token gid: heads 2t, 2t + 1 in c[0], c[1]; token gid + 8 in c[2], c[3]
+        const bool ok0 = (mask >> gid) & 1u, ok1 = (mask >> (gid + 8)) & 1u;
+        float v[4] = {ok0 ? c[0] : -INFINITY, ok0 ? c[1] : -INFINITY, ok1 ? c[2] : -INFINITY,
+                      ok1 ? c[3] : -INFINITY};
+        // per head (column): max and sum of exp over the 16 tokens (the eight
+        // lanes of one t hold them)
+        float mx0 = fmaxf(v[0], v[2]), mx1 = fmaxf(v[1], v[3]);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            if (!((mask >> sl[i]) & 1u)) v[i] = -INFINITY;
-            mx = fmaxf(mx, v[i]);
+        for (int o = 4; o < 32; o <<= 1) {
+            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
         }
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-        float z = 0.0f;
+        float z0 = (v[0] == -INFINITY ? 0.0f : expf(v[0] - mx0)) + (v[2] == -INFINITY ? 0.0f : expf(v[2] - mx0));
+        float z1 = (v[1] == -INFINITY ? 0.0f : expf(v[1] - mx1)) + (v[3] == -INFINITY ? 0.0f : expf(v[3] - mx1));
 #pragma unroll
-        for (int i = 0; i < 4; ++i) z += v[i] == -INFINITY ? 0.0f : expf(v[i] - mx);
-        z += __shfl_xor_sync(0xffffffffu, z, 1);
-        z += __shfl_xor_sync(0xffffffffu, z, 2);
-        if (gid < g) {
-            const int hq = kh * g + gid;
-            const int m0 = 16 * j;
+        for (int o = 4; o < 32; o <<= 1) {
+            z0 += __shfl_xor_sync(0xffffffffu, z0, o);
+            z1 += __shfl_xor_sync(0xffffffffu, z1, o);
+        }
+        const int m0 = 16 * j;
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int h = 2 * t + hh;
+            if (h >= g) continue;
+            const int hq = kh * g + h;
             float* lg = a.logits + (int64_t(b) * Hq + hq) * M + m0;
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-                if (m0 + sl[i] < M) lg[sl[i]] = v[i];
-            if (t == 0) {
+            if (m0 + gid < M) lg[gid] = v[hh];
+            if (m0 + gid + 8 < M) lg[gid + 8] = v[2 + hh];
+            if (gid == 0) {
+                const float mxh = hh ? mx1 : mx0;
                 float* ts = a.tile_stats + ((int64_t(b) * Hq + hq) * NT + j) * 2;
-                ts[0] = mx;
-                ts[1] = mx == -INFINITY ? 0.0f : z;
+                ts[0] = mxh;
+                ts[1] = mxh == -INFINITY ? 0.0f : (hh ? z1 : z0);
             }
         }
+        cur = nxt;
+        nxt = pf;
+        advance(pf);
     }
     if (err) atomicOr(a.status, err);
 }
