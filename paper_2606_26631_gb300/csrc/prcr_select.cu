@@ -520,6 +520,8 @@ __global__ void __launch_bounds__(256, 2) ads_logits_cache_kernel(const __grid_c
     };
 
     uint32_t qh[KS][2], ql[KS][2];
+    float* lg_base[2] = {nullptr, nullptr};
+    float* ts_base[2] = {nullptr, nullptr};
     int cur_b = -1, cur_kh = -1;
     Item cur, nxt, pf;
     {
@@ -563,6 +565,12 @@ __global__ void __launch_bounds__(256, 2) ads_logits_cache_kernel(const __grid_c
             __syncwarp();  // qw is rewritten for the next (b, kh)
             cur_b = b;
             cur_kh = kh;
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {  // rows of this lane's heads 2t, 2t + 1
+                const int64_t r = int64_t(b) * Hq + kh * g + min(2 * t + hh, g - 1);
+                lg_base[hh] = a.logits + r * M;
+                ts_base[hh] = a.tile_stats + r * NT * 2;
+            }
         }
         // S^T (16 tokens x 8 columns = the group's query heads, columns >= g
         // zero) = K Q^T: rows gid (kn[0]) and gid + 8 (kn[1]) are this lane's
@@ -593,25 +601,30 @@ __global__ void __launch_bounds__(256, 2) ads_logits_cache_kernel(const __grid_c
             mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
             mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
         }
-        float z0 = (v[0] == -INFINITY ? 0.0f : expf(v[0] - mx0)) + (v[2] == -INFINITY ? 0.0f : expf(v[2] - mx0));
-        float z1 = (v[1] == -INFINITY ? 0.0f : expf(v[1] - mx1)) + (v[3] == -INFINITY ? 0.0f : expf(v[3] - mx1));
+        // arguments <= 0: __expf's few-ulp error is far below the relevance bar
+        float z0 = (v[0] == -INFINITY ? 0.0f : __expf(v[0] - mx0)) + (v[2] == -INFINITY ? 0.0f : __expf(v[2] - mx0));
+        float z1 = (v[1] == -INFINITY ? 0.0f : __expf(v[1] - mx1)) + (v[3] == -INFINITY ? 0.0f : __expf(v[3] - mx1));
 #pragma unroll
         for (int o = 4; o < 32; o <<= 1) {
             z0 += __shfl_xor_sync(0xffffffffu, z0, o);
             z1 += __shfl_xor_sync(0xffffffffu, z1, o);
         }
         const int m0 = 16 * j;
+        const bool full = m0 + 16 <= M;
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
-            const int h = 2 * t + hh;
-            if (h >= g) continue;
-            const int hq = kh * g + h;
-            float* lg = a.logits + (int64_t(b) * Hq + hq) * M + m0;
-            if (m0 + gid < M) lg[gid] = v[hh];
-            if (m0 + gid + 8 < M) lg[gid + 8] = v[2 + hh];
+            if (2 * t + hh >= g) continue;
+            float* lg = lg_base[hh] + m0;
+            if (full) {
+                lg[gid] = v[hh];
+                lg[gid + 8] = v[2 + hh];
+            } else {
+                if (m0 + gid < M) lg[gid] = v[hh];
+                if (m0 + gid + 8 < M) lg[gid + 8] = v[2 + hh];
+            }
             if (gid == 0) {
                 const float mxh = hh ? mx1 : mx0;
-                float* ts = a.tile_stats + ((int64_t(b) * Hq + hq) * NT + j) * 2;
+                float* ts = ts_base[hh] + 2 * j;
                 ts[0] = mxh;
                 ts[1] = mxh == -INFINITY ? 0.0f : (hh ? z1 : z0);
             }
