@@ -284,7 +284,8 @@ PRCR_API int prcr_prefill_capture(const prcr_rope_cfg* cfg, const prcr_store_des
  * workspace: device, >= prcr_decode_workspace_size(...) bytes (0 when the
  * sequence axis is not split), 16-byte aligned. A seq_len beyond the
  * capacity sets PRCR_ST_CAPACITY (clamped); an unmapped block in range sets
- * PRCR_ST_NO_BLOCK and its slots are left out of the softmax.              */
+ * PRCR_ST_NO_BLOCK and its slots are left out of the softmax. A sequence
+ * with seq_len 0 (or no readable slot) gets an output of zeros.           */
 #define PRCR_DECODE_MAX_Q_ELEMS 8192
 PRCR_API size_t prcr_decode_workspace_size(const prcr_rope_cfg* cfg, int32_t n_seqs,
                                            int32_t n_q_heads, int64_t max_len);

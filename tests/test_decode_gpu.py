@@ -86,6 +86,39 @@ def test_decode_parity(case):
             assert err <= 1e-4, (b, l, err)
 
 
+@pytest.mark.parametrize("H,Hq,D,paged", [(8, 32, 128, False), (4, 16, 128, True), (2, 14, 64, False),
+                                         (4, 8, 256, True)])
+def test_decode_empty_and_single_slot(H, Hq, D, paged):
+    """A sequence with no slots gets zeros; one with a single slot gets that
+    slot's V row exactly (its softmax weight is exactly 1); a longer one
+    beside them still matches the oracle. Covers the head-split kernel
+    (8 KV heads), the one-CTA-per-chunk kernel, head_dim 64 and the
+    CUDA-core kernel (head_dim 256)."""
+    import paper_2606_26631_gb300 as prcr
+    B, nL, max_len = 3, 2, 300
+    sec = (D // 8, D // 8 + (D // 2 - 3 * (D // 8)) // 2, 0)
+    sec = (sec[0], sec[1], D // 2 - sec[0] - sec[1])
+    inp = make_decode_inputs(B, nL, H, Hq, D, max_len, paged, device=DEV, seed=19)
+    seq_len = torch.tensor([0, 1, max_len], dtype=torch.int32, device=DEV)
+    cfg = prcr.rope_cfg(nL, H, D, sec, 1e6)
+    cd = (prcr.cache_paged(inp["cache_k"], inp["cache_v"], inp["block_table"]) if paged
+          else prcr.cache_contiguous(inp["cache_k"], inp["cache_v"]))
+    out, st = _run_decode(cfg, cd, inp["q"], inp["q_pos"], seq_len, max_len)
+    assert st == 0
+    got = out.cpu().numpy()
+    assert np.all(got[0] == 0.0)
+    g = Hq // H
+    K1, V1 = _cache_rows(inp["cache_k"], inp["cache_v"], inp["block_table"], 1, 1, paged)
+    for l in range(nL):
+        for h in range(Hq):
+            assert np.array_equal(got[1, l, h], V1[0, l, h // g].astype(np.float32)), (l, h)
+    K, V = _cache_rows(inp["cache_k"], inp["cache_v"], inp["block_table"], 2, max_len, paged)
+    qv = _f64(inp["q"])
+    for l in range(nL):
+        ref = O.decode_attention(qv[2, l], int(inp["q_pos"][2]), K[:, l], V[:, l], D, sec, 1e6)
+        assert np.abs(got[2, l] - ref).max() / np.abs(V[:, l]).max() <= 1e-4
+
+
 def test_decode_unaligned_query():
     """Query rows only 4-byte aligned (the ABI's minimum) take the scalar
     loads of the rotation: the output is bit-identical to the aligned call."""
