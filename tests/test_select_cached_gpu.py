@@ -225,3 +225,35 @@ def test_select_cached_after_prefill_capture():
         # bf16 keys carry 2^-9 relative rounding: for these query and key
         # scales a logit moves by ~6e-3 (one sigma), the relevance by as much
         assert (np.abs(score[b] - raw) / raw).max() <= 5e-2
+
+
+def test_select_single_token_both_sources():
+    """One visual token, k = 1: the softmax over one token is 1 for every
+    head, so the relevance is exactly 1 (4 heads x 0.25) and the token is
+    selected, from the raw store and from the cache alike."""
+    import paper_2606_26631_gb300 as prcr
+    B, H, Hq, D, M, sec = 2, 2, 4, 64, 1, (8, 12, 12)
+    g = torch.Generator(device=DEV).manual_seed(2)
+    cfg = prcr.rope_cfg(1, H, D, sec, 1e6)
+    q = torch.randn((B, Hq, D), device=DEV, generator=g).to(torch.bfloat16)
+    q_pos = torch.tensor([50, 70], dtype=torch.int64, device=DEV)
+    ws = torch.empty(prcr.select_workspace_size(B, Hq, M), dtype=torch.uint8, device=DEV)
+    sk = torch.randn((B, 1, M, H, D), device=DEV, generator=g).to(torch.bfloat16)
+    coords = torch.tensor([[[0, 3, 4]], [[0, 5, 6]]], dtype=torch.int32, device=DEV)
+    for source in ("raw", "cache"):
+        idx = torch.full((B,), -7, dtype=torch.int32, device=DEV)
+        sro = torch.full((B + 1,), -7, dtype=torch.int32, device=DEV)
+        rto = torch.full((B + 1,), -7, dtype=torch.int32, device=DEV)
+        score = torch.full((B, M), -1.0, dtype=torch.float32, device=DEV)
+        if source == "raw":
+            prcr.select_topk(cfg, prcr.store_desc(sk, sk, coords), 0, q, q_pos, 1, idx, sro, rto, ws,
+                             score)
+        else:
+            status = torch.zeros(1, dtype=torch.int32, device=DEV)
+            img0 = torch.zeros(B, dtype=torch.int32, device=DEV)
+            prcr.select_topk_cached(cfg, prcr.cache_contiguous(sk, sk), 0, q, q_pos, img0, M, 1, idx,
+                                    sro, rto, status, ws, score)
+        torch.cuda.synchronize()
+        assert idx.tolist() == [0, 0], source
+        assert sro.tolist() == [0, 1, 2] and rto.tolist() == [0, 1, 2], source
+        assert score.cpu().tolist() == [[1.0], [1.0]], source
