@@ -459,8 +459,10 @@ __global__ void __launch_bounds__(256, 2) ads_logits_cache_kernel(const __grid_c
             }
         }
     };
-    // element offset of the item's key row for token 16 j + (lane & 15), or -1
-    // (past the end, or no readable row)
+    // element offset, without the KV head's D elements, of the key row of
+    // token 16 j + (lane & 15) of sequence b, or -1 (past the end, or no
+    // readable row). Computed once per item, when its rows are requested.
+    const int64_t layer_off = int64_t(a.layer) * a.cache_layer_stride;
     auto row_of = [&](const Item& x) -> int64_t {
         const int m = 16 * x.j + (lane & 15);
         if (m >= M) return -1;
@@ -492,28 +494,28 @@ __global__ void __launch_bounds__(256, 2) ads_logits_cache_kernel(const __grid_c
             }
             row = int64_t(blk) * a.cache_block_stride + off * a.cache_slot_stride;
         }
-        return row + int64_t(a.layer) * a.cache_layer_stride + int64_t(x.kh) * D;
+        return row + layer_off;
     };
     uint4 kn[2][LV];
     uint32_t mask_n = 0u;
-    auto fetch = [&](const Item& x) {
-        const int64_t row = row_of(x);
+    // loads an item's 16 key rows (row: this lane's token, from row_of). A
+    // token without a row reads the cache's first row instead: its logit is
+    // set to -inf whatever the row holds (tokens are separate MMA rows).
+    auto fetch = [&](int64_t row, int kh) {
         mask_n = __ballot_sync(0xffffffffu, row >= 0) & 0xffffu;
+        const int64_t r0 = (row >= 0 ? row : 0) + int64_t(kh) * D;
 #pragma unroll
         for (int nt = 0; nt < 2; ++nt) {
-            const int64_t rr = __shfl_sync(0xffffffffu, row, nt * 8 + gid);
+            const uint16_t* kp = a.cache_k + __shfl_sync(0xffffffffu, r0, nt * 8 + gid) + t * (D / 4);
 #pragma unroll
-            for (int u = 0; u < LV; ++u)
-                kn[nt][u] = rr >= 0 ? ld_stream(a.cache_k + rr + t * (D / 4) + 8 * u)
-                                    : make_uint4(0u, 0u, 0u, 0u);
+            for (int u = 0; u < LV; ++u) kn[nt][u] = ld_stream(kp + 8 * u);
         }
     };
     // the rows of the item after next are requested into L2 (lanes 0..15,
     // one token row each), so that its fetch finds them there
-    auto request = [&](const Item& x) {
-        const int64_t row = row_of(x);
+    auto request = [&](int64_t row, int kh) {
         if (lane < 16 && row >= 0) {
-            const char* p = reinterpret_cast<const char*>(a.cache_k + row);
+            const char* p = reinterpret_cast<const char*>(a.cache_k + row + int64_t(kh) * D);
 #pragma unroll
             for (int o = 0; o < D * 2; o += 128) prefetch_l2(p + o);
         }
@@ -534,8 +536,12 @@ __global__ void __launch_bounds__(256, 2) ads_logits_cache_kernel(const __grid_c
     advance(nxt);
     pf = nxt;
     advance(pf);
-    if (i_beg < i_end) fetch(cur);
-    if (i_beg + 1 < i_end) request(nxt);
+    int64_t row_nxt = -1, row_pf = -1;
+    if (i_beg < i_end) fetch(row_of(cur), cur.kh);
+    if (i_beg + 1 < i_end) {
+        row_nxt = row_of(nxt);
+        request(row_nxt, nxt.kh);
+    }
     for (int64_t left = i_end - i_beg; left > 0; --left) {
         const int b = cur.b, kh = cur.kh, j = cur.j;
         if (b != cur_b || kh != cur_kh) {
@@ -586,8 +592,11 @@ __global__ void __launch_bounds__(256, 2) ads_logits_cache_kernel(const __grid_c
             mma_16816(c, a0, a1, a2, a3, qh[k][0], qh[k][1]);
             mma_16816(c, a0, a1, a2, a3, ql[k][0], ql[k][1]);
         }
-        if (left > 1) fetch(nxt);
-        if (left > 2) request(pf);
+        if (left > 1) fetch(row_nxt, nxt.kh);
+        if (left > 2) {
+            row_pf = row_of(pf);
+            request(row_pf, pf.kh);
+        }
 
         // token gid: heads 2t, 2t + 1 in c[0], c[1]; token gid + 8 in c[2], c[3]
         const bool ok0 = (mask >> gid) & 1u, ok1 = (mask >> (gid + 8)) & 1u;
@@ -631,6 +640,7 @@ __global__ void __launch_bounds__(256, 2) ads_logits_cache_kernel(const __grid_c
         }
         cur = nxt;
         nxt = pf;
+        row_nxt = row_pf;
         advance(pf);
     }
     if (err) atomicOr(a.status, err);
