@@ -344,11 +344,13 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
         const uint16_t* krow = a.store_k + int64_t(b) * a.store_seq_stride +
                                int64_t(a.layer) * a.store_layer_stride +
                                int64_t(m) * a.store_token_stride + tq * PL;
+        // a dead lane (token past the tile's end) reads its octet's first
+        // token: its logits are never written out, so its data need not be zero
         uint4 xn[NW], yn[NW];
 #pragma unroll
         for (int u = 0; u < NW; ++u) {
-            xn[u] = live ? ld_stream(krow + kh_a * D + 8 * u) : make_uint4(0u, 0u, 0u, 0u);
-            yn[u] = live ? ld_stream(krow + kh_a * D + P + 8 * u) : make_uint4(0u, 0u, 0u, 0u);
+            xn[u] = ld_stream(krow + kh_a * D + 8 * u);
+            yn[u] = ld_stream(krow + kh_a * D + P + 8 * u);
         }
         for (int kh = kh_a; kh < kh_b; ++kh) {
             uint32_t xw[4 * NW], yw[4 * NW];
@@ -360,8 +362,8 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
             if (kh + 1 < kh_b) {  // the next head's pairs, in flight during this head's MMAs
 #pragma unroll
                 for (int u = 0; u < NW; ++u) {
-                    xn[u] = live ? ld_stream(krow + (kh + 1) * D + 8 * u) : make_uint4(0u, 0u, 0u, 0u);
-                    yn[u] = live ? ld_stream(krow + (kh + 1) * D + P + 8 * u) : make_uint4(0u, 0u, 0u, 0u);
+                    xn[u] = ld_stream(krow + (kh + 1) * D + 8 * u);
+                    yn[u] = ld_stream(krow + (kh + 1) * D + P + 8 * u);
                 }
             }
             float c[4] = {0.0f, 0.0f, 0.0f, 0.0f};
