@@ -70,3 +70,125 @@ def test_fuzz_rebind_inject(i):
     assert rv.status_value() == 0
     pu.full_check(batch, rv, mode=mode, L=L, degenerate="center" if center else "zero",
                   layout=layout)
+
+
+def _decode_case(i: int):
+    rng = np.random.default_rng(2000 + i)
+    D = int(rng.choice([64, 128, 256]))
+    H = int(rng.choice([1, 2, 3, 4, 8]))
+    g = int(rng.choice([1, 2, 3, 4, 7, 8]))
+    while H * g * D > 8192:
+        g = max(1, g // 2)
+    B = int(rng.integers(1, 6))
+    nL = int(rng.integers(1, 5))
+    max_len = int(rng.choice([17, 64, 300, 933, 2500, 6000]))
+    paged = bool(rng.integers(0, 2))
+    bs = int(rng.choice([1, 7, 16, 32])) if paged else 16
+    P = D // 2
+    cut = np.sort(rng.integers(0, P + 1, size=2))
+    sec = (int(cut[0]), int(cut[1] - cut[0]), int(P - cut[1]))
+    return B, nL, H, H * g, D, max_len, paged, bs, sec
+
+
+@pytest.mark.parametrize("i", range(12))
+def test_fuzz_decode(i):
+    """Random decode shapes (chunking, head split, merge kernels and the
+    CUDA-core kernel all vary with them) against the oracle."""
+    import torch
+    import paper_2606_26631_gb300 as prcr
+    from workloads import make_decode_inputs
+    B, nL, H, Hq, D, max_len, paged, bs, sec = _decode_case(i)
+    inp = make_decode_inputs(B, nL, H, Hq, D, max_len, paged, device=DEV, seed=60 + i, block_size=bs)
+    cfg = prcr.rope_cfg(nL, H, D, sec, 1e6)
+    cd = (prcr.cache_paged(inp["cache_k"], inp["cache_v"], inp["block_table"]) if paged
+          else prcr.cache_contiguous(inp["cache_k"], inp["cache_v"]))
+    out = torch.full(inp["q"].shape, float("nan"), dtype=torch.float32, device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    ws = torch.empty(max(prcr.decode_workspace_size(cfg, B, Hq, max_len), 16), dtype=torch.uint8,
+                     device=DEV)
+    prcr.decode_attention(cfg, cd, inp["q"], inp["q_pos"], inp["seq_len"], max_len, out, status, ws)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    got = out.cpu().numpy()
+    qv = O.bf16_bits_to_f64(inp["q"].view(torch.int16).cpu().numpy())
+    for b in range(B):
+        n = int(inp["seq_len"][b])
+        s = torch.arange(n, device=DEV)
+        if paged:
+            blk = inp["block_table"][b][s // bs].long()
+            K = inp["cache_k"][:, blk, s % bs].transpose(0, 1)
+            V = inp["cache_v"][:, blk, s % bs].transpose(0, 1)
+        else:
+            K = inp["cache_k"][b, :, :n].transpose(0, 1)
+            V = inp["cache_v"][b, :, :n].transpose(0, 1)
+        K = O.bf16_bits_to_f64(K.contiguous().view(torch.int16).cpu().numpy())
+        V = O.bf16_bits_to_f64(V.contiguous().view(torch.int16).cpu().numpy())
+        for l in range(nL):
+            ref = O.decode_attention(qv[b, l], int(inp["q_pos"][b]), K[:, l], V[:, l], D, sec, 1e6)
+            assert np.abs(got[b, l] - ref).max() / np.abs(V[:, l]).max() <= 1e-4, (b, l)
+
+
+def _select_case(i: int):
+    rng = np.random.default_rng(3000 + i)
+    D = int(rng.choice([64, 128]))
+    H = int(rng.choice([1, 2, 3, 4, 8]))
+    g = int(rng.choice([1, 2, 3, 4, 7, 8]))
+    while H * g * D > 8192:
+        g = max(1, g // 2)
+    B = int(rng.integers(1, 6))
+    M = int(rng.choice([1, 15, 16, 17, 100, 767, 1024, 1025, 4099, 9000]))
+    k = int(rng.integers(1, M + 1))
+    P = D // 2
+    cut = np.sort(rng.integers(0, P + 1, size=2))
+    sec = (int(cut[0]), int(cut[1] - cut[0]), int(P - cut[1]))
+    return B, H, H * g, D, M, k, sec, bool(i % 2)
+
+
+@pytest.mark.parametrize("i", range(12))
+def test_fuzz_select(i):
+    """Random selection shapes from the raw store (even cases) and from the
+    cache (odd cases): relevance against the oracle, the set the exact top-k
+    of the reported relevance and a valid top-k of the oracle's."""
+    import torch
+    import paper_2606_26631_gb300 as prcr
+    B, H, Hq, D, M, k, sec, cached = _select_case(i)
+    g = torch.Generator(device=DEV).manual_seed(70 + i)
+    sk = torch.randn((B, 1, M, H, D), device=DEV, generator=g).to(torch.bfloat16)
+    coords = torch.randint(0, 64, (B, M, 3), device=DEV, generator=g, dtype=torch.int32)
+    q = (2.0 * torch.randn((B, Hq, D), device=DEV, generator=g)).to(torch.bfloat16)
+    q_pos = torch.randint(100, 20000, (B,), device=DEV, generator=g, dtype=torch.int64)
+    cfg = prcr.rope_cfg(1, H, D, sec, 1e6)
+    idx = torch.full((B * k,), -7, dtype=torch.int32, device=DEV)
+    sro = torch.full((B + 1,), -7, dtype=torch.int32, device=DEV)
+    rto = torch.full((B + 1,), -7, dtype=torch.int32, device=DEV)
+    score = torch.full((B, M), -1.0, dtype=torch.float32, device=DEV)
+    ws = torch.empty(prcr.select_workspace_size(B, Hq, M), dtype=torch.uint8, device=DEV)
+    if cached:
+        status = torch.zeros(1, dtype=torch.int32, device=DEV)
+        img0 = torch.zeros(B, dtype=torch.int32, device=DEV)
+        prcr.select_topk_cached(cfg, prcr.cache_contiguous(sk, sk), 0, q, q_pos, img0, M, k, idx, sro,
+                                rto, status, ws, score)
+    else:
+        prcr.select_topk(cfg, prcr.store_desc(sk, sk, coords), 0, q, q_pos, k, idx, sro, rto, ws, score)
+    torch.cuda.synchronize()
+    if cached:
+        assert int(status.item()) == 0
+    idx = idx.view(B, k).cpu().numpy()
+    score = score.cpu().numpy()
+    qv = O.bf16_bits_to_f64(q.view(torch.int16).cpu().numpy())
+    kb = sk.view(torch.int16).cpu().numpy()
+    crd = coords.cpu().numpy()
+    for b in range(B):
+        if cached:
+            ref = O.ads_relevance_cached(qv[b], int(q_pos[b]), O.bf16_bits_to_f64(kb[b, 0]), D, sec, 1e6)
+        else:
+            ref = O.ads_relevance(qv[b], int(q_pos[b]), kb[b, 0], crd[b], D, sec, 1e6)
+        assert (np.abs(score[b] - ref) / ref).max() <= 1e-4
+        sel = idx[b]
+        order = np.lexsort((np.arange(M), -score[b].astype(np.float64)))
+        assert np.array_equal(sel, np.sort(order[:k]))
+        if k < M:
+            tol = 2 * np.abs(score[b] - ref).max() + 1e-12
+            chosen = np.zeros(M, dtype=bool)
+            chosen[sel] = True
+            assert ref[chosen].min() >= ref[~chosen].max() - tol
