@@ -248,3 +248,35 @@ def test_new_entry_points_validate_on_host():
     assert sel(ws=None) == B.EWORKSPACE
     assert sel(wsb=16) == B.EWORKSPACE
     assert prcr.select_workspace_size(2, 4, 64) >= 2 * 4 * 64 * 4 + 2 * 64 * 4
+
+
+def test_select_cached_validates_on_host():
+    """prcr_select_topk_cached rejects bad arguments before any CUDA call:
+    the shared selection checks, its own head_dim limit, the image slot
+    array and the status word."""
+    a = _descs()
+    L = prcr.lib()
+    ca = C.byref(a["ca"]); cfg = C.byref(a["cfg"])
+    Q, QP, IMG, STAT = FAKE + 2 ** 27, FAKE + 2 ** 28, FAKE + 2 ** 29, FAKE + 2 ** 26
+    IDX, SRO, RTO, WS = FAKE + 2 ** 31, FAKE + 2 ** 32, FAKE + 2 ** 33, FAKE + 2 ** 34
+
+    def sel(cfg_=cfg, **k):
+        return L.prcr_select_topk_cached(cfg_, ca, k.get("B", 1), k.get("layer", 0), k.get("Hq", 4),
+                                         k.get("M", 64), k.get("img", IMG), Q, QP, k.get("k", 8),
+                                         IDX, SRO, RTO, None, k.get("status", STAT),
+                                         k.get("ws", WS), k.get("wsb", 1 << 20), None)
+    assert sel(k=0) == B.EINVAL
+    assert sel(k=65) == B.EINVAL           # more than the image's 64 tokens
+    assert sel(M=0) == B.EINVAL
+    assert sel(M=40000) == B.EINVAL        # beyond PRCR_SELECT_MAX_TOKENS
+    assert sel(layer=2) == B.EINVAL
+    assert sel(Hq=3) == B.EINVAL
+    assert sel(B=2) == B.EINVAL            # more sequences than the cache holds
+    assert sel(img=None) == B.EINVAL
+    assert sel(status=None) == B.EINVAL
+    assert sel(img=IMG + 2) == B.EALIGN
+    assert sel(ws=None) == B.EWORKSPACE
+    assert sel(wsb=16) == B.EWORKSPACE
+    assert sel(B=0) == B.OK
+    cfg48 = prcr.rope_cfg(2, 2, 48, (8, 8, 8))
+    assert sel(cfg_=C.byref(cfg48)) == B.EINVAL  # head_dim 48: the cached path takes 64 and 128
