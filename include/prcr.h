@@ -341,7 +341,7 @@ PRCR_API int prcr_select_topk(const prcr_rope_cfg* cfg, const prcr_store_desc* s
  *               selection of a sequence with no readable token is unspecified)
  * Other arguments, outputs, limits and the workspace (prcr_select_workspace_size
  * with the same n_seqs, n_q_heads, n_tokens) are those of prcr_select_topk;
- * head_dim must be 64 or 128 (PRCR_EINVAL otherwise).                    */
+ * head_dim must be 64, 128 or 256 (PRCR_EINVAL otherwise).               */
 PRCR_API int prcr_select_topk_cached(const prcr_rope_cfg* cfg, const prcr_cache_desc* cache,
                                      int32_t n_seqs, int32_t layer, int32_t n_q_heads,
                                      int32_t n_tokens, const int32_t* img_slot0, const void* q,

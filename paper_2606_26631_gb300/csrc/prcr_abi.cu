@@ -688,7 +688,7 @@ int prcr_select_topk_cached(const prcr_rope_cfg* cfg, const prcr_cache_desc* cac
     if (rc) return rc;
     if ((rc = check_cache(cfg, cache))) return rc;
     if (n_seqs > cache->n_seqs || n_tokens < 1 ||
-        (cfg->head_dim != 64 && cfg->head_dim != 128))
+        (cfg->head_dim != 64 && cfg->head_dim != 128 && cfg->head_dim != 256))
         return PRCR_EINVAL;
     SelectArgs a = {};
     // token tiles of 16: one warp's MMA tile of keys

@@ -433,7 +433,8 @@ __global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_con
 // into L2. An item writes its 16 logits per head and the tile's (max, sum of
 // exp) per head; a token without a readable row gets logit -inf.
 template <int D>
-__global__ void __launch_bounds__(256, 2) ads_logits_cache_kernel(const __grid_constant__ SelectArgs a) {
+__global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
+    ads_logits_cache_kernel(const __grid_constant__ SelectArgs a) {
     pdl_allow();
     constexpr int KS = D / 16, LV = D / 32, P = D / 2;
     extern __shared__ __align__(16) float sm[];
@@ -931,7 +932,9 @@ cudaError_t launch_select(const SelectArgs& a, int n_seqs, int sms, cudaStream_t
 cudaError_t launch_select_cached(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream) {
     const int g = a.n_q_heads / a.n_kv_heads;
     const size_t smem = size_t(8) * g * a.head_dim * sizeof(float);  // 8 warps
-    auto k = a.head_dim == 64 ? ads_logits_cache_kernel<64> : ads_logits_cache_kernel<128>;
+    auto k = a.head_dim == 64 ? ads_logits_cache_kernel<64>
+             : a.head_dim == 128 ? ads_logits_cache_kernel<128>
+                                 : ads_logits_cache_kernel<256>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     int per_sm = 0;
     if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, 256, smem);

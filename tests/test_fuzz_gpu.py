@@ -130,7 +130,7 @@ def test_fuzz_decode(i):
 
 def _select_case(i: int):
     rng = np.random.default_rng(3000 + i)
-    D = int(rng.choice([64, 128]))
+    D = int(rng.choice([64, 128, 256]))
     H = int(rng.choice([1, 2, 3, 4, 8]))
     g = int(rng.choice([1, 2, 3, 4, 7, 8]))
     while H * g * D > 8192:

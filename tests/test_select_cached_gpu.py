@@ -4,7 +4,8 @@ the oracle's header), against the oracle's float64 ads_relevance_cached on
 the same bf16 cache rows.
 
 Caches are filled with random bf16 rows directly (contiguous, and paged with
-shuffled blocks of 16 or 7 slots), so nothing but this call is under test.
+shuffled blocks of 16 or 7 slots; head_dim 64, 128 and 256), so nothing but
+this call is under test.
 Relevance: relative error <= 1e-4. Selection: as for the raw-store call,
 (a) the set is exactly the top-k of the relevance the kernel reports (ties to
 the lower index), (b) it is a valid top-k of the oracle's relevance up to
@@ -91,6 +92,7 @@ CASES = [  # (B, n_layers, layer, H, Hq, D, M, k, paged, block_size, sections, t
     (3, 2, 1, 4, 16, 128, 2116, 300, True, 16, (16, 24, 24), 1e6),
     (3, 1, 0, 2, 14, 64, 91, 20, True, 7, (8, 12, 12), 5e5),
     (1, 2, 0, 3, 9, 64, 1500, 200, False, 0, (8, 12, 12), 1e6),
+    (2, 1, 0, 4, 16, 256, 700, 64, True, 16, (40, 44, 44), 1e6),
 ]
 
 
