@@ -31,6 +31,10 @@ import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
+# the oracle legs run on one host thread (their `cores`): numpy's BLAS and
+# OpenMP pools are fixed before anything imports numpy
+for _v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, "1")
 
 METRIC = "rebind+inject GB/s (read+write)"
 UNIT = "GB/s"
@@ -288,6 +292,18 @@ def cpu_baseline(wl, n_layers: int, n_samples: int = 1, device="cpu"):
                         f"{wl.n_kv_heads} KV heads, one sequence per oracle call "
                         f"({total_b / 1e9:.2f} GB algorithmic); numpy float64, one thread"),
                 seconds=total_t)
+
+
+def oracle_leg(args, fn, nbytes: int, sample: str):
+    """The oracle as it stands, timed once on the host on a bounded sample of
+    the path's workload: GB/s of the sample's algorithmic bytes."""
+    if args.no_cpu_baseline:
+        return None
+    t0 = time.perf_counter()
+    fn()
+    dt = time.perf_counter() - t0
+    return dict(value=nbytes / dt / 1e9, unit=UNIT, cores=1, host_cores=os.cpu_count(),
+                kind="oracle", sample=sample + "; numpy float64, one thread", seconds=dt)
 
 
 # ----------------------------------------------------------------------------
@@ -578,6 +594,19 @@ def run_capture_path(args):
     t = sum(ms) / 1e3
     peak, kind = measured_peaks()
     value = nbytes * args.steps / t / 1e9
+    mc = min(M, 1024)
+    kb = src.store_k[0, :, :mc].contiguous().view(torch.int16).cpu().numpy()  # [nL, mc, H, D]
+    vb = src.store_v[0, :, :mc].contiguous().view(torch.int16).cpu().numpy()
+    crd = src.coords[0, :mc].cpu().numpy()
+
+    def oracle():
+        from oracle import prcr_oracle as O
+        for l in range(nL):
+            O.prefill_capture(kb[l], vb[l], crd, D, wl.sections, wl.theta)
+
+    cpu = oracle_leg(args, oracle, mc * nL * H * D * 2 * 6,
+                     f"sequence 0 of '{wl.name}': its first {mc} visual tokens x {nL} layers x "
+                     f"{H} KV heads, one layer per oracle call")
     print(json.dumps(dict(
         metric="prefill capture GB/s (read+write)", value=value, unit=UNIT, n_gpus=1,
         steps=args.steps, warmup=args.warmup, ms_per_step=1e3 * t / args.steps,
@@ -587,7 +616,7 @@ def run_capture_path(args):
                                       l2=flush.describe(nbytes)),
         roofline=dict(bound="hbm", achieved=value, peak=peak, unit="GB/s", frac=value / peak,
                       traffic=None, kernel="capture_kernel", peak_kind=f"{kind} copy (hbm_gbs)"),
-        **_launch_keys(launched, B, args.steps), clocks=clk)), flush=True)
+        cpu_baseline=cpu, **_launch_keys(launched, B, args.steps), clocks=clk)), flush=True)
 
 
 def run_decode_path(args):
@@ -629,6 +658,23 @@ def run_decode_path(args):
     t = sum(ms) / 1e3
     peak, kind = measured_peaks()
     value = nbytes * args.steps / t / 1e9
+    n0 = int(inp["seq_len"][0])
+    s0 = torch.arange(n0, device=dev)
+    blk = inp["block_table"][0][s0 // 16].long()
+    K0 = inp["cache_k"][:, blk, s0 % 16].transpose(0, 1).contiguous().view(torch.int16).cpu().numpy()
+    V0 = inp["cache_v"][:, blk, s0 % 16].transpose(0, 1).contiguous().view(torch.int16).cpu().numpy()
+    q0 = inp["q"][0].contiguous().view(torch.int16).cpu().numpy()
+    p0 = int(inp["q_pos"][0])
+
+    def oracle():
+        from oracle import prcr_oracle as O
+        qv, Kv, Vv = O.bf16_bits_to_f64(q0), O.bf16_bits_to_f64(K0), O.bf16_bits_to_f64(V0)
+        for l in range(wl.n_layers):
+            O.decode_attention(qv[l], p0, Kv[:, l], Vv[:, l], wl.head_dim, wl.sections, wl.theta)
+
+    cpu = oracle_leg(args, oracle, n0 * wl.n_layers * wl.n_kv_heads * wl.head_dim * 2 * 2,
+                     f"sequence 0 of the batch ({n0} slots) x {wl.n_layers} layers x "
+                     f"{wl.n_kv_heads} KV heads, {Hq} query heads, one layer per oracle call")
     print(json.dumps(dict(
         metric="decode attention GB/s (K/V read)", value=value, unit=UNIT, n_gpus=1,
         steps=args.steps, warmup=args.warmup, ms_per_step=1e3 * t / args.steps,
@@ -639,7 +685,8 @@ def run_decode_path(args):
         roofline=dict(bound="hbm", achieved=value, peak=peak, unit="GB/s", frac=value / peak,
                       traffic=None, kernel="decode_kernel (+ merge)",
                       peak_kind=f"{kind} copy (hbm_gbs)"),
-        **_launch_keys(launched, 2 if nws else 1, args.steps), clocks=clk)), flush=True)
+        cpu_baseline=cpu, **_launch_keys(launched, 2 if nws else 1, args.steps), clocks=clk)),
+        flush=True)
 
 
 def run_select_path(args):
@@ -706,6 +753,23 @@ def run_select_path(args):
     t = sum(ms) / 1e3
     peak, kind = measured_peaks()
     value = nbytes * args.steps / t / 1e9
+    kb0 = batch.store_k[0, layer].contiguous().view(torch.int16).cpu().numpy()  # [M, H, D]
+    crd0 = batch.coords[0].cpu().numpy()
+    q0 = q[0].contiguous().view(torch.int16).cpu().numpy()
+    p0 = int(batch.p_txt[0])
+
+    def oracle():
+        from oracle import prcr_oracle as O
+        qv = O.bf16_bits_to_f64(q0)
+        if args.select_source == "raw":
+            rel = O.ads_relevance(qv, p0, kb0, crd0, D, wl.sections, wl.theta)
+        else:
+            rel = O.ads_relevance_cached(qv, p0, O.bf16_bits_to_f64(kb0), D, wl.sections, wl.theta)
+        O.ads_select(rel, k)
+
+    cpu = oracle_leg(args, oracle, M * H * D * 2,
+                     f"sequence 0 of '{wl.name}' ({M} tokens x {H} KV heads, {Hq} query heads, "
+                     f"k = {k}), relevance and selection")
     print(json.dumps(dict(
         metric=f"selection GB/s ({args.select_source} keys read)", value=value, unit=UNIT, n_gpus=1,
         steps=args.steps, warmup=args.warmup, ms_per_step=1e3 * t / args.steps,
@@ -716,7 +780,7 @@ def run_select_path(args):
         roofline=dict(bound="hbm", achieved=value, peak=peak, unit="GB/s", frac=value / peak,
                       traffic=None, kernel="ads_*_kernel (whole selection step)",
                       peak_kind=f"{kind} copy (hbm_gbs)"),
-        **_launch_keys(launched, 4, args.steps), clocks=clk)), flush=True)
+        cpu_baseline=cpu, **_launch_keys(launched, 4, args.steps), clocks=clk)), flush=True)
 
 
 def run_pipeline_path(args):

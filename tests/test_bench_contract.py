@@ -53,3 +53,20 @@ def test_gpu_arm_line():
     for k in ("sm_mhz", "sm_max_mhz", "reasons"):
         assert k in d["clocks"], k
     assert d["config"]["workload"] == "tiny"
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("path", ["capture", "decode", "select", "pipeline"])
+def test_gpu_other_paths_line(path):
+    """The capture, decode, selection and pipeline bench paths print one
+    well-formed line each; the first three time the oracle beside the kernel."""
+    args = ["--path", path, "--workload", "tiny", "--steps", "3", "--warmup", "3"]
+    d = _run(args)
+    for k in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+              "higher_is_better", "config", "gpu_launches", "clocks"):
+        assert k in d, (path, k)
+    assert d["value"] > 0 and d["gpu_launches"] >= d["steps"]
+    if path != "pipeline":
+        assert d["roofline"]["bound"] == "hbm" and d["roofline"]["achieved"] > 0
+        c = d["cpu_baseline"]
+        assert c["kind"] == "oracle" and c["cores"] == 1 and c["value"] > 0 and c["sample"]
