@@ -60,6 +60,9 @@ CASES = [  # (B, layers, H, Hq, D, max_len, paged)
     # CTAs, chunk rows requested into L2 ahead of the tile loop)
     (1, 36, 8, 32, 128, 933, False),
     (2, 2, 8, 16, 64, 500, True),
+    # the head-split kernel at the ends of the GQA range: 1 and 8 query heads per KV head
+    (1, 2, 8, 8, 128, 500, False),
+    (1, 2, 8, 64, 128, 300, True),
 ]
 
 

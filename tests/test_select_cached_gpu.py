@@ -259,3 +259,40 @@ def test_select_single_token_both_sources():
         assert idx.tolist() == [0, 0], source
         assert sro.tolist() == [0, 1, 2] and rto.tolist() == [0, 1, 2], source
         assert score.cpu().tolist() == [[1.0], [1.0]], source
+
+
+@pytest.mark.parametrize("cached", [False, True])
+def test_select_most_query_heads(cached):
+    """128 query heads (16 KV heads x 8, head_dim 64: the largest head count
+    the selection takes) from the raw store and from the cache."""
+    import paper_2606_26631_gb300 as prcr
+    B, H, Hq, D, M, k, sec = 2, 16, 128, 64, 300, 40, (8, 12, 12)
+    g = torch.Generator(device=DEV).manual_seed(21)
+    sk = torch.randn((B, 1, M, H, D), device=DEV, generator=g).to(torch.bfloat16)
+    coords = torch.randint(0, 40, (B, M, 3), device=DEV, generator=g, dtype=torch.int32)
+    q = (2.0 * torch.randn((B, Hq, D), device=DEV, generator=g)).to(torch.bfloat16)
+    q_pos = torch.tensor([700, 3000], dtype=torch.int64, device=DEV)
+    cfg = prcr.rope_cfg(1, H, D, sec, 1e6)
+    ws = torch.empty(prcr.select_workspace_size(B, Hq, M), dtype=torch.uint8, device=DEV)
+    idx = torch.full((B * k,), -7, dtype=torch.int32, device=DEV)
+    sro = torch.full((B + 1,), -7, dtype=torch.int32, device=DEV)
+    rto = torch.full((B + 1,), -7, dtype=torch.int32, device=DEV)
+    score = torch.full((B, M), -1.0, dtype=torch.float32, device=DEV)
+    if cached:
+        status = torch.zeros(1, dtype=torch.int32, device=DEV)
+        prcr.select_topk_cached(cfg, prcr.cache_contiguous(sk, sk), 0, q, q_pos,
+                                torch.zeros(B, dtype=torch.int32, device=DEV), M, k, idx, sro, rto,
+                                status, ws, score)
+    else:
+        prcr.select_topk(cfg, prcr.store_desc(sk, sk, coords), 0, q, q_pos, k, idx, sro, rto, ws, score)
+    torch.cuda.synchronize()
+    qv = O.bf16_bits_to_f64(q.view(torch.int16).cpu().numpy())
+    kb = sk.view(torch.int16).cpu().numpy()
+    idx = idx.view(B, k).cpu().numpy()
+    score = score.cpu().numpy()
+    for b in range(B):
+        if cached:
+            ref = O.ads_relevance_cached(qv[b], int(q_pos[b]), O.bf16_bits_to_f64(kb[b, 0]), D, sec, 1e6)
+        else:
+            ref = O.ads_relevance(qv[b], int(q_pos[b]), kb[b, 0], coords[b].cpu().numpy(), D, sec, 1e6)
+        _check_seq(score[b], ref, idx[b], k, M)
