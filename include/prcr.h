@@ -42,7 +42,8 @@
 extern "C" {
 #endif
 
-#define PRCR_VERSION 1
+/* 2: adds prcr_select_topk_cached (1: every other entry point) */
+#define PRCR_VERSION 2
 
 #if defined(__GNUC__)
 #define PRCR_API __attribute__((visibility("default")))

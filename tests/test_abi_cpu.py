@@ -27,7 +27,7 @@ def test_library_exports_every_declared_symbol():
     L = prcr.lib()
     for name in _declared():
         assert hasattr(L, name), name
-    assert prcr.version() == 1
+    assert prcr.version() == 2
 
 
 def test_header_constants_match_binding():
