@@ -284,7 +284,9 @@ PRCR_API int prcr_prefill_capture(const prcr_rope_cfg* cfg, const prcr_store_des
  * n_seqs and n_layers at most 65535 (launch grid limits).
  * workspace: device, >= prcr_decode_workspace_size(...) bytes (0 when the
  * sequence axis is not split), 16-byte aligned. A seq_len beyond the
- * capacity sets PRCR_ST_CAPACITY (clamped); an unmapped block in range sets
+ * capacity, or above max_len, sets PRCR_ST_CAPACITY (the slots past the
+ * capacity, or past the split made for max_len, are left out); an unmapped
+ * block in range sets
  * PRCR_ST_NO_BLOCK and its slots are left out of the softmax. A sequence
  * with seq_len 0 (or no readable slot) gets an output of zeros.           */
 #define PRCR_DECODE_MAX_Q_ELEMS 8192

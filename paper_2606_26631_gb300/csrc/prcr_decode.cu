@@ -69,6 +69,10 @@ __global__ void __launch_bounds__(kDecodeThreads, 3) decode_kernel(const __grid_
         err |= PRCR_ST_CAPACITY;
         len = len < 0 ? 0 : a.capacity;
     }
+    if (len > int64_t(a.splits) * a.chunk) {  // above the host's max_len: past the split
+        err |= PRCR_ST_CAPACITY;
+        len = int64_t(a.splits) * a.chunk;
+    }
     const int64_t s_begin = int64_t(split) * a.chunk;
     const int64_t s_end = min(len, s_begin + a.chunk);
 
@@ -342,6 +346,10 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     if (len < 0 || len > a.capacity) {
         err |= PRCR_ST_CAPACITY;
         len = len < 0 ? 0 : a.capacity;
+    }
+    if (len > int64_t(a.splits) * a.chunk) {  // above the host's max_len: past the split
+        err |= PRCR_ST_CAPACITY;
+        len = int64_t(a.splits) * a.chunk;
     }
     const int64_t s_begin = int64_t(split) * a.chunk;
     const int64_t s_end = min(len, s_begin + a.chunk);

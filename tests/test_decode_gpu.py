@@ -122,6 +122,55 @@ def test_decode_empty_and_single_slot(H, Hq, D, paged):
         assert np.abs(got[2, l] - ref).max() / np.abs(V[:, l]).max() <= 1e-4
 
 
+def test_decode_device_errors():
+    """Device-detected errors: an unmapped block in a sequence's range sets
+    PRCR_ST_NO_BLOCK and its slots are left out of the softmax; a length
+    beyond the capacity sets PRCR_ST_CAPACITY and is clamped to it; a length
+    above max_len sets PRCR_ST_CAPACITY too. Outputs stay the oracle's
+    attention over the slots that remain (where those are defined)."""
+    import paper_2606_26631_gb300 as prcr
+    nL, H, Hq, D, sec = 2, 2, 8, 64, (8, 12, 12)
+    cfg = prcr.rope_cfg(nL, H, D, sec, 1e6)
+    # (a) paged: block 3 of sequence 1 (its slots 48..63) unmapped
+    inp = make_decode_inputs(2, nL, H, Hq, D, 200, True, device=DEV, seed=23)
+    bt = inp["block_table"].clone()
+    bt[1, 3] = -1
+    cd = prcr.cache_paged(inp["cache_k"], inp["cache_v"], bt)
+    out, st = _run_decode(cfg, cd, inp["q"], inp["q_pos"], inp["seq_len"], 200)
+    assert st & prcr.ST_NO_BLOCK
+    got = out.cpu().numpy()
+    qv = _f64(inp["q"])
+    n1 = int(inp["seq_len"][1])
+    K, V = _cache_rows(inp["cache_k"], inp["cache_v"], inp["block_table"], 1, n1, True)
+    keep = np.array([s for s in range(n1) if s // 16 != 3])
+    for l in range(nL):
+        ref = O.decode_attention(qv[1, l], int(inp["q_pos"][1]), K[keep, l], V[keep, l], D, sec, 1e6)
+        assert np.abs(got[1, l] - ref).max() / np.abs(V[:, l]).max() <= 1e-4
+    K0, V0 = _cache_rows(inp["cache_k"], inp["cache_v"], inp["block_table"], 0, int(inp["seq_len"][0]),
+                         True)
+    for l in range(nL):
+        ref = O.decode_attention(qv[0, l], int(inp["q_pos"][0]), K0[:, l], V0[:, l], D, sec, 1e6)
+        assert np.abs(got[0, l] - ref).max() / np.abs(V0[:, l]).max() <= 1e-4
+    # (b) contiguous, capacity 208 slots: a length of 300 is clamped to 208
+    inp = make_decode_inputs(1, nL, H, Hq, D, 200, False, device=DEV, seed=24)
+    cap = inp["cache_k"].shape[2]
+    cd = prcr.cache_contiguous(inp["cache_k"], inp["cache_v"])
+    seq_len = torch.tensor([300], dtype=torch.int32, device=DEV)
+    out, st = _run_decode(cfg, cd, inp["q"], inp["q_pos"], seq_len, cap)
+    assert st & prcr.ST_CAPACITY
+    got = out.cpu().numpy()
+    qv = _f64(inp["q"])
+    K, V = _cache_rows(inp["cache_k"], inp["cache_v"], None, 0, cap, False)
+    for l in range(nL):
+        ref = O.decode_attention(qv[0, l], int(inp["q_pos"][0]), K[:, l], V[:, l], D, sec, 1e6)
+        assert np.abs(got[0, l] - ref).max() / np.abs(V[:, l]).max() <= 1e-4
+    # (c) a length above the max_len the call was split for
+    seq_len = torch.tensor([150], dtype=torch.int32, device=DEV)
+    out, st = _run_decode(cfg, cd, inp["q"], inp["q_pos"], seq_len, 100)
+    assert st & prcr.ST_CAPACITY
+    assert torch.isfinite(out).all()
+
+
 def test_decode_unaligned_query():
     """Query rows only 4-byte aligned (the ABI's minimum) take the scalar
     loads of the rotation: the output is bit-identical to the aligned call."""
