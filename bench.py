@@ -44,8 +44,8 @@ SPEC_HBM_GBS = 8000.0
 # workload, from an ncu capture; valid only for the kernel source it was
 # measured on (its sha256 prefix), reported as null otherwise.
 TRAFFIC = {
-    # profiles/rebind_kernel_stress_dram.md: 19,308,455,168 B read + 19,268,777,472 B written
-    ("stress", "c218e17c64a8cfc9"): 38577232640,
+    # profiles/rebind_kernel_stress_dram.md: 19,309,795,840 B read + 19,268,509,184 B written
+    ("stress", "36f2c98b3efb3176"): 38578305024,
 }
 
 

@@ -63,8 +63,11 @@ extern "C" {
 #define PRCR_ST_NO_BLOCK   2u  /* paged: block-table entry < 0 or >= n_blocks         */
 #define PRCR_ST_CAPACITY   4u  /* a slot lies beyond the sequence's cache capacity     */
 #define PRCR_ST_CSR        8u  /* offsets not monotone / not spanning [0, total_k)     */
-#define PRCR_ST_POS_RANGE 16u  /* a position's exact rational exceeds 2^53: the value
-                                  is still computed but not correctly rounded          */
+#define PRCR_ST_POS_RANGE 16u  /* a position's exact rational exceeds 2^53 (the value
+                                  is still computed but not correctly rounded), or a
+                                  position or query position has magnitude 2^31 or
+                                  more: beyond the range of the rotation's exact
+                                  fixed-point angle reduction                          */
 
 /* Position rules (Sec. 3.2; Table 2) */
 #define PRCR_MODE_PCR      0  /* Position-Consistent Reinsertion (the method)        */

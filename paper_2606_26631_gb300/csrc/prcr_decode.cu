@@ -81,6 +81,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3) decode_kernel(const __grid_
     // whatever its band, so each pair's cos/sin serves all heads.
     __shared__ float s_cos[kMaxPairs], s_sin[kMaxPairs];
     const int64_t p = a.q_pos[b];
+    if (p <= -2147483648LL || p >= 2147483648LL) err |= PRCR_ST_POS_RANGE;  // fixed-point angle range
     for (int i = threadIdx.x; i < P; i += blockDim.x) {
         sincos_turns(double(p), a.turn_freq[i], &s_sin[i], &s_cos[i]);
     }
@@ -385,6 +386,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     __shared__ __align__(16) float s_cos[kMaxPairs];
     __shared__ __align__(16) float s_sin[kMaxPairs];
     const int64_t p = a.q_pos[b];
+    if (p <= -2147483648LL || p >= 2147483648LL) err |= PRCR_ST_POS_RANGE;  // fixed-point angle range
     for (int i = threadIdx.x; i < P; i += blockDim.x) {
         sincos_turns(double(p), a.turn_freq[i], &s_sin[i], &s_cos[i]);
     }

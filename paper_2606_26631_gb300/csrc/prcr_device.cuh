@@ -287,6 +287,10 @@ __device__ __forceinline__ void token_plan(const PlanArgs& a, const RevisitCtx& 
             break;
         }
     }
+    // the rotation reduces angles in 32.32 fixed point: |position| < 2^31
+    if (!(fabs(pos[0]) < 2147483648.0 && fabs(pos[1]) < 2147483648.0 &&
+          fabs(pos[2]) < 2147483648.0))
+        err |= PRCR_ST_POS_RANGE;
     src = int64_t(r.b) * a.store_seq_stride + int64_t(m) * a.store_token_stride;
     dst = dest_row(a, r, slot, blk, err);
 }

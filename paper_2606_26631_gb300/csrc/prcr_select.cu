@@ -550,6 +550,7 @@ __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
         if (b != cur_b || kh != cur_kh) {
             // the group's queries turned at (p, p, p), pre-scaled, as A fragments
             const int64_t p = a.q_pos[b];
+            if (p <= -2147483648LL || p >= 2147483648LL) err |= PRCR_ST_POS_RANGE;
             const uint16_t* qg = a.q + (int64_t(b) * Hq + kh * g) * D;
             for (int i = lane; i < P; i += 32) {
                 float sn, cs;

@@ -171,6 +171,22 @@ def test_decode_device_errors():
     assert torch.isfinite(out).all()
 
 
+def test_decode_query_position_range():
+    """A query position of 2^31 or more is beyond the fixed-point angle
+    reduction: PRCR_ST_POS_RANGE (head-split and one-CTA-per-chunk kernels)."""
+    import paper_2606_26631_gb300 as prcr
+    for H, Hq in ((8, 32), (2, 8)):
+        inp = make_decode_inputs(1, 2, H, Hq, 128, 300, False, device=DEV, seed=5)
+        cfg = prcr.rope_cfg(2, H, 128, (16, 24, 24), 1e6)
+        cd = prcr.cache_contiguous(inp["cache_k"], inp["cache_v"])
+        qp = torch.tensor([2 ** 31], dtype=torch.int64, device=DEV)
+        _, st = _run_decode(cfg, cd, inp["q"], qp, inp["seq_len"], 300)
+        assert st & prcr.ST_POS_RANGE
+        qp = torch.tensor([2 ** 31 - 1], dtype=torch.int64, device=DEV)
+        _, st = _run_decode(cfg, cd, inp["q"], qp, inp["seq_len"], 300)
+        assert st == 0
+
+
 def test_decode_unaligned_query():
     """Query rows only 4-byte aligned (the ABI's minimum) take the scalar
     loads of the rotation: the output is bit-identical to the aligned call."""

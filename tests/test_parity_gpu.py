@@ -395,3 +395,20 @@ def test_bad_index_small_batch():
     assert rv.status_value() & pu.prcr.ST_IDX_RANGE
     written = np.array([j for j in range(batch.total_k) if j != 7])
     pu.check_untouched(batch, pl, written=written)
+
+
+def test_position_beyond_angle_range_is_flagged():
+    """Text positions of 2^31 and more are beyond the fixed-point angle
+    reduction: the call sets PRCR_ST_POS_RANGE (one-kernel and two-kernel
+    paths); a position well inside the range does not."""
+    import paper_2606_26631_gb300 as prcr
+    import parity_util as pu
+    for name in ("tiny", "qwen25vl-7b"):
+        batch = make_batch(get(name), device=DEV, seed=4)
+        batch.p_txt.fill_(2 ** 31 + 100)
+        rv = _run(batch)
+        assert rv.status_value() & prcr.ST_POS_RANGE, name
+        batch = make_batch(get(name), device=DEV, seed=4)
+        batch.p_txt.fill_(2 ** 31 - 2 ** 20)
+        rv = _run(batch)
+        assert rv.status_value() == 0, name

@@ -296,3 +296,15 @@ def test_select_most_query_heads(cached):
         else:
             ref = O.ads_relevance(qv[b], int(q_pos[b]), kb[b, 0], coords[b].cpu().numpy(), D, sec, 1e6)
         _check_seq(score[b], ref, idx[b], k, M)
+
+
+def test_select_cached_query_position_range():
+    """A query position of 2^31 or more sets PRCR_ST_POS_RANGE."""
+    import paper_2606_26631_gb300 as prcr
+    cache_k, bt, img0 = _make_cache(1, 1, 2, 64, 40, False, 0, seed=3)
+    cfg = prcr.rope_cfg(1, 2, 64, (8, 12, 12), 1e6)
+    q = torch.randn((1, 4, 64), device=DEV).to(torch.bfloat16)
+    for pos, bad in ((2 ** 31 + 7, True), (2 ** 31 - 1, False)):
+        qp = torch.tensor([pos], dtype=torch.int64, device=DEV)
+        _, _, _, _, st = _run(cfg, prcr.cache_contiguous(cache_k, cache_k), 0, q, qp, img0, 40, 5)
+        assert bool(st & prcr.ST_POS_RANGE) == bad
