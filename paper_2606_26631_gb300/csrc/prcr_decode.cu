@@ -343,6 +343,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     }
 
     pdl_wait();
+    const int64_t p = a.q_pos[b];  // requested together with the length
     int64_t len = a.seq_len[b];
     if (len < 0 || len > a.capacity) {
         err |= PRCR_ST_CAPACITY;
@@ -385,7 +386,6 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
 
     __shared__ __align__(16) float s_cos[kMaxPairs];
     __shared__ __align__(16) float s_sin[kMaxPairs];
-    const int64_t p = a.q_pos[b];
     if (p <= -2147483648LL || p >= 2147483648LL) err |= PRCR_ST_POS_RANGE;  // fixed-point angle range
     for (int i = threadIdx.x; i < P; i += blockDim.x) {
         sincos_turns(double(p), a.turn_freq[i], &s_sin[i], &s_cos[i]);
