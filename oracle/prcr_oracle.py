@@ -49,8 +49,32 @@ Readings taken where the paper is silent (each is a named choice below):
   over the keys the decoder's position-bound cache holds for the visual
   tokens (RoPE(k_raw, p_m) as stored, e.g. in bf16), only the query rotated.
 
-Parity pins for every function here live in tests/test_oracle_pins.py; every
-function is pinned (no function is "parity unpinned").
+Every function here is pinned in tests/test_oracle_pins.py against facts
+from outside this module (no function is "parity unpinned"):
+
+* coord_range, normalized_coord, pcr_position, reassign_revisit: hand-worked
+  4x4 and 2x2 rectangles (tests/golden), closed forms of the PCR rule, the
+  centre reading, the other position rules (pin_worked_rect*,
+  pin_pcr_closed_forms, pin_degenerate_center, pin_other_modes)
+* next_text_pos, plan: pin_worked_rect4x4, pin_other_modes,
+  pin_plan_slots_and_continuity
+* inv_freq, pair_axes, angles, rope, rebind_keys: textbook rotary values and
+  complex-number RoPE, band membership, norm preservation, R(a)R(b) = R(a+b),
+  the relative-offset logit identity (pin_rope_closed_forms,
+  pin_mrope_equal_axes_is_textbook, pin_mrope_sections, pin_rope_invariants)
+* bf16_bits_to_f64, f64_to_bf16_rne: pin_bf16_helpers
+* rebind_inject, position_bound_keys, prefill_capture: a pure-Python brute
+  force on a 2x2 region, the ORIGINAL rule against Eq.
+  "historical_position_bound_kv" (pin_brute_force_2x2,
+  pin_original_mode_is_position_bound_cache, pin_prefill_capture)
+* decode_attention: a direct softmax and the relative-offset identity
+  (pin_decode_attention)
+* ads_relevance, ads_relevance_cached, ads_select: pin_ads, pin_ads_cached
+* pair_norms: hand-worked rows (tests/golden/pair_norms.txt) and the norm
+  kept by any rotation (pin_pair_norms)
+
+Planted mistakes in each of them are caught by some pin
+(test_planted_mistakes).
 """
 from __future__ import annotations
 
@@ -336,14 +360,6 @@ def ads_select(relevance: np.ndarray, K: int) -> np.ndarray:
 # ----------------------------------------------------------------------------
 # Whole call on small inputs: gather, reassign, rebind, concat
 # ----------------------------------------------------------------------------
-def cache_row(kind: str, b: int, slot: int, block_table=None, block_size: int = 16):
-    """Where slot ``slot`` of sequence ``b`` lives: (b, slot) for a contiguous
-    cache, (physical block, offset) for a paged one."""
-    if kind == "contiguous":
-        return b, slot
-    return int(block_table[b][slot // block_size]), slot % block_size
-
-
 def rebind_inject(store_k_bits, store_v_bits, coords, seq_rev_off, rev_tok_off, idx,
                   p_txt, cache_len_in, head_dim, sections, theta, L, mode=MODE_PCR,
                   degenerate="zero", layout=LAYOUT_SECTIONED, layers=None):
@@ -369,8 +385,10 @@ def rebind_inject(store_k_bits, store_v_bits, coords, seq_rev_off, rev_tok_off, 
 
 
 def pair_norms(k_raw_bits: np.ndarray) -> np.ndarray:
-    """Norm of each rotation pair, repeated on both of its elements: the
-    quantity RoPE preserves (used to scale errors near zero)."""
+    """Norm of each rotation pair (x_i, x_{i+D/2}) of the raw keys, repeated on
+    both of its elements: the quantity a rotary embedding preserves (Sec. 2.3
+    and Sec. 3.3, Eq. "cache_reconstruction": the rebound key differs from the
+    raw key by a rotation of each pair). Used to scale errors near zero."""
     x = bf16_bits_to_f64(k_raw_bits)
     P = x.shape[-1] // 2
     r = np.sqrt(x[..., :P] ** 2 + x[..., P:] ** 2)

@@ -509,11 +509,43 @@ def pin_ads_cached(o):
                        o.ads_relevance_cached(q, 90, kpb, D, sec, th), rtol=1e-9, atol=0)
 
 
+def pin_pair_norms(o):
+    """Norm of each rotation pair (the scale of the K error bar near zero):
+    hand-worked rows (tests/golden/pair_norms.txt), shapes kept for batched
+    rows, and the invariant it stands for: a rotary embedding at any angles
+    leaves every pair's norm unchanged (Sec. 2.3; Sec. 3.3, Eq.
+    "cache_reconstruction"), so the norms of the raw row equal the pair
+    lengths of the rebound row."""
+    for r in _golden_rows("pair_norms.txt"):
+        D = int(r[0])
+        raw = np.array([int(h, 16) for h in r[1:1 + D]], dtype=np.uint16)
+        want = [float(x) for x in r[1 + D:1 + 2 * D]]
+        got = o.pair_norms(raw)
+        assert got.shape == (D,), (got.shape, D)
+        assert list(got) == want, (r, list(got))
+        # a batch of rows [N, H, D] keeps its shape and gives each row's norms
+        batch = np.stack([raw, raw[::-1].copy()])[:, None, :]
+        gb = o.pair_norms(batch)
+        assert gb.shape == (2, 1, D)
+        assert list(gb[0, 0]) == want
+    rng = np.random.default_rng(23)
+    D = 128
+    P = D // 2
+    bits = rng.integers(0x3C00, 0x4100, size=(6, 4, D)).astype(np.uint16)
+    bits[..., 1::3] |= 0x8000
+    rho = o.pair_norms(bits)
+    x = o.bf16_bits_to_f64(bits).reshape(-1, D)
+    for ang in (rng.uniform(-40, 40, size=(x.shape[0], P)), np.zeros((x.shape[0], P))):
+        y = o.rope(x, ang)
+        n = np.sqrt(y[:, :P] ** 2 + y[:, P:] ** 2)
+        assert np.allclose(np.concatenate([n, n], axis=1), rho.reshape(-1, D), rtol=1e-13, atol=0)
+
+
 PINS = [pin_worked_rect4x4, pin_worked_rect2x2, pin_pcr_closed_forms, pin_degenerate_center,
         pin_other_modes, pin_plan_slots_and_continuity, pin_rope_closed_forms,
         pin_mrope_equal_axes_is_textbook, pin_mrope_sections, pin_rope_invariants,
         pin_bf16_helpers, pin_brute_force_2x2, pin_original_mode_is_position_bound_cache,
-        pin_prefill_capture, pin_decode_attention, pin_ads, pin_ads_cached]
+        pin_prefill_capture, pin_decode_attention, pin_ads, pin_ads_cached, pin_pair_norms]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -642,6 +674,31 @@ def _m_select_ties_high(rel, K):
     return np.array(sorted(order[:K]), dtype=np.int64)
 
 
+def _m_pair_norms_no_sqrt(k_raw_bits):
+    x = O.bf16_bits_to_f64(k_raw_bits)
+    P = x.shape[-1] // 2
+    r = x[..., :P] ** 2 + x[..., P:] ** 2
+    return np.concatenate([r, r], axis=-1)
+
+
+def _m_pair_norms_first_half(k_raw_bits):
+    x = O.bf16_bits_to_f64(k_raw_bits)
+    P = x.shape[-1] // 2
+    r = np.abs(x[..., :P])
+    return np.concatenate([r, r], axis=-1)
+
+
+def _m_pair_norms_whole_row(k_raw_bits):
+    x = O.bf16_bits_to_f64(k_raw_bits)
+    return np.broadcast_to(np.sqrt((x ** 2).sum(axis=-1, keepdims=True)), x.shape).copy()
+
+
+def _m_pair_norms_adjacent(k_raw_bits):
+    x = O.bf16_bits_to_f64(k_raw_bits)
+    r = np.sqrt(x[..., 0::2] ** 2 + x[..., 1::2] ** 2)
+    return np.concatenate([r, r], axis=-1)
+
+
 MUTANTS = [
     ("pcr_position", _m_pcr_k_not_k_minus_1),
     ("pcr_position", _m_pcr_denominator_k),
@@ -662,6 +719,10 @@ MUTANTS = [
     ("ads_select", _m_select_ties_high),
     ("ads_relevance_cached", _m_rel_cached_query_unrotated),
     ("ads_relevance_cached", _m_rel_cached_head_modulo),
+    ("pair_norms", _m_pair_norms_no_sqrt),
+    ("pair_norms", _m_pair_norms_first_half),
+    ("pair_norms", _m_pair_norms_whole_row),
+    ("pair_norms", _m_pair_norms_adjacent),
 ]
 
 
