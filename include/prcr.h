@@ -26,11 +26,23 @@
  *    be 16-byte aligned (base pointers 16-byte aligned, strides multiples of 8).
  *  - Return value: PRCR_OK (0) or a negative PRCR_E* code. A negative code
  *    means nothing was enqueued. Errors found on the device (bad index,
- *    missing block, full cache, malformed offsets) are OR-ed as PRCR_ST_* bits
- *    into the caller's device status word; the offending rows are skipped,
- *    nothing is written out of bounds and no kernel traps.
- *  - Entry points keep no state between calls and may be called from several
- *    host threads at once.
+ *    missing block, full cache, malformed offsets, a position out of range)
+ *    are OR-ed as PRCR_ST_* bits into the caller's device status word; the
+ *    offending rows are skipped (each entry point states what it outputs
+ *    for them), nothing is written out of bounds and no kernel traps.
+ *  - Rotation angles: position x theta^(-2i/D) is reduced modulo one turn
+ *    exactly in integer fixed point (the position in signed 32.32, the pair's
+ *    rate theta^(-2i/D) / (2 pi) in unsigned 0.64, computed once on the host
+ *    in long double), giving the angle to 2^-32 of a turn; only the final
+ *    sin/cos is float32. This needs |position| < 2^31 (PRCR_ST_POS_RANGE
+ *    otherwise).
+ *  - State: the outputs of a call depend only on its arguments. The library
+ *    keeps process-wide caches that are filled on first use and read-only
+ *    afterwards (guarded by a mutex): the turn rates per (theta, head_dim),
+ *    the SM count and kernel occupancies per device, and, for
+ *    prcr_rebind_inject_static only, a fixed scratch array per device and its
+ *    address. Every entry point except prcr_rebind_inject_static may be
+ *    called from several host threads at once.
  */
 #ifndef PRCR_H_
 #define PRCR_H_
@@ -63,11 +75,13 @@ extern "C" {
 #define PRCR_ST_NO_BLOCK   2u  /* paged: block-table entry < 0 or >= n_blocks         */
 #define PRCR_ST_CAPACITY   4u  /* a slot lies beyond the sequence's cache capacity     */
 #define PRCR_ST_CSR        8u  /* offsets not monotone / not spanning [0, total_k)     */
-#define PRCR_ST_POS_RANGE 16u  /* a position's exact rational exceeds 2^53 (the value
-                                  is still computed but not correctly rounded), or a
-                                  position or query position has magnitude 2^31 or
-                                  more: beyond the range of the rotation's exact
-                                  fixed-point angle reduction                          */
+#define PRCR_ST_POS_RANGE 16u  /* a reassigned position cannot be formed as a correctly
+                                  rounded exact rational (operands of 2^52 or more),
+                                  or a position or query position has magnitude 2^31
+                                  or more (beyond the exact fixed-point angle
+                                  reduction): the rebind skips that token's rows;
+                                  decode and cached selection treat that sequence as
+                                  having no readable slot                             */
 
 /* Position rules (Sec. 3.2; Table 2) */
 #define PRCR_MODE_PCR      0  /* Position-Consistent Reinsertion (the method)        */
@@ -183,12 +197,15 @@ PRCR_API size_t prcr_workspace_size(int64_t total_k);
  *     among sequence b's tokens in this call) and source/destination rows.
  *  2. rebind + inject (Sec. 3.3): for every (token, layer, kv head) the raw
  *     key row is gathered, rotated with sectioned/interleaved M-RoPE at the
- *     new positions (angles in float64 reduced mod 2*pi, then float32
- *     sin/cos and float32 arithmetic, rounded to bf16 to nearest even), the
- *     raw value row is copied bit for bit, and both are written to the slot.
+ *     new positions (angle reduced exactly modulo one turn in fixed point,
+ *     then float32 sin/cos and float32 arithmetic, rounded to bf16 to
+ *     nearest even), the raw value row is copied bit for bit, and both are
+ *     written to the slot.
  * L is the left extension (L >= 0; the paper's default is 2, Sec. 4.4).
- * Rows of tokens with a device error are not written; slots outside the
- * appended span are never touched. The call is re-runnable: the same inputs
+ * Rows of tokens with a device error are not written (a token whose position
+ * sets PRCR_ST_POS_RANGE included: pos_out / slot_out still receive its
+ * computed position and slot); slots outside the appended span are never
+ * touched. cache_len_out and next_pos_out count every token of the call. The call is re-runnable: the same inputs
  * give the same outputs. workspace: device, >= prcr_workspace_size(total_k)
  * bytes, 16-byte aligned, not shared with a concurrent call.              */
 PRCR_API int prcr_rebind_inject(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
@@ -224,6 +241,11 @@ PRCR_API int prcr_rebind_apply(const prcr_rope_cfg* cfg, const prcr_store_desc* 
  *  - total_k > PRCR_STATIC_MAX_TOKENS returns PRCR_EWORKSPACE, nothing enqueued.
  *  - The first call on a device looks up the array's device address (set-up
  *    done once per device); make that first call before any stream capture.
+ *    The address is kept for the process: do not call this entry point on a
+ *    device after a reset of that device (cudaDeviceReset, or its primary
+ *    context released and created again), which leaves the kept address stale.
+ *  - Arguments are checked as prcr_rebind_inject checks them (same codes)
+ *    before the size limit and before any set-up.
  *  - Every call shares the one array: calls whose work overlaps on the GPU
  *    (other streams, other host threads) race and must be serialised by the
  *    caller. Nothing in the array needs to start at zero.                    */
@@ -290,8 +312,10 @@ PRCR_API int prcr_prefill_capture(const prcr_rope_cfg* cfg, const prcr_store_des
  * capacity, or above max_len, sets PRCR_ST_CAPACITY (the slots past the
  * capacity, or past the split made for max_len, are left out); an unmapped
  * block in range sets
- * PRCR_ST_NO_BLOCK and its slots are left out of the softmax. A sequence
- * with seq_len 0 (or no readable slot) gets an output of zeros.           */
+ * PRCR_ST_NO_BLOCK and its slots are left out of the softmax. A query
+ * position of magnitude 2^31 or more sets PRCR_ST_POS_RANGE and the sequence
+ * reads no slot. A sequence with seq_len 0 (or no readable slot) gets an
+ * output of zeros.                                                         */
 #define PRCR_DECODE_MAX_Q_ELEMS 8192
 PRCR_API size_t prcr_decode_workspace_size(const prcr_rope_cfg* cfg, int32_t n_seqs,
                                            int32_t n_q_heads, int64_t max_len);
@@ -308,7 +332,11 @@ PRCR_API int prcr_decode_attention(const prcr_rope_cfg* cfg, const prcr_cache_de
  * relevance of visual token m is the trigger query's attention on m at layer
  * `layer`: per query head h, softmax over the store's M tokens of
  * RoPE(q[b][h], (p, p, p)) . RoPE(k_raw[b][layer][m][h / group], p_m) / sqrt(D),
- * p = q_pos[b], averaged over the heads. The k most relevant tokens (equal
+ * p = q_pos[b], averaged over the heads. The rotation is applied as
+ * RoPE(q, (p,p,p)) . RoPE(k, c) = q . R(c - p) k, the integer offset c - p
+ * reduced modulo one turn in 64-bit integer arithmetic (to 2^-32 of a turn
+ * while |c - p| < 2^31; no status word: larger offsets lose accuracy as
+ * |c - p| * 2^-65 of a turn). The k most relevant tokens (equal
  * relevance: lower index first) are written in ascending token order as one
  * revisit per sequence, ready for prcr_rebind_inject:
  *   idx_out     device int32 [n_seqs * k]   selected token ids
@@ -343,8 +371,11 @@ PRCR_API int prcr_select_topk(const prcr_rope_cfg* cfg, const prcr_store_desc* s
  *   img_slot0   device int32 [n_seqs]  first cache slot of sequence b's image
  *   status      device uint32 word: a token whose slot lies beyond the
  *               sequence's capacity sets PRCR_ST_CAPACITY, one in an unmapped
- *               block PRCR_ST_NO_BLOCK; such a token gets relevance 0 (the
- *               selection of a sequence with no readable token is unspecified)
+ *               block PRCR_ST_NO_BLOCK; such a token gets relevance 0. A query
+ *               position of magnitude 2^31 or more sets PRCR_ST_POS_RANGE and
+ *               every token of that sequence gets relevance 0. A sequence
+ *               whose tokens all have relevance 0 selects its first k tokens
+ *               (equal relevance: lower index first)
  * Other arguments, outputs, limits and the workspace (prcr_select_workspace_size
  * with the same n_seqs, n_q_heads, n_tokens) are those of prcr_select_topk;
  * head_dim must be 64, 128 or 256 (PRCR_EINVAL otherwise).               */

@@ -85,10 +85,12 @@ int check_cache(const prcr_rope_cfg* c, const prcr_cache_desc* k) {
     return PRCR_OK;
 }
 
-int check_call(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
-               const prcr_cache_desc* cache, const prcr_revisit_batch* b,
-               const prcr_outputs* o, int32_t mode, int32_t L, int32_t flags, void* ws,
-               size_t ws_bytes) {
+}  // namespace
+
+// Every check of a revisit call except the workspace's.
+int check_revisit_args(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+                       const prcr_cache_desc* cache, const prcr_revisit_batch* b,
+                       const prcr_outputs* o, int32_t mode, int32_t L, int32_t flags) {
     int rc = check_cfg(cfg);
     if (rc) return rc;
     if ((rc = check_store(cfg, store))) return rc;
@@ -110,6 +112,17 @@ int check_call(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
         !aligned8(o->next_pos_out) || !aligned4(o->status) ||
         (o->pos_out && !aligned8(o->pos_out)) || (o->slot_out && !aligned4(o->slot_out)))
         return PRCR_EALIGN;
+    return PRCR_OK;
+}
+
+namespace {
+
+int check_call(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+               const prcr_cache_desc* cache, const prcr_revisit_batch* b,
+               const prcr_outputs* o, int32_t mode, int32_t L, int32_t flags, void* ws,
+               size_t ws_bytes) {
+    const int rc = check_revisit_args(cfg, store, cache, b, o, mode, L, flags);
+    if (rc || b->n_seqs == 0) return rc;
     if (b->total_k > 0) {
         if (!ws || ws_bytes < workspace_bytes(b->total_k)) return PRCR_EWORKSPACE;
         if (!aligned16(ws)) return PRCR_EALIGN;

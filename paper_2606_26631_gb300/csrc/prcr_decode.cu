@@ -73,6 +73,13 @@ __global__ void __launch_bounds__(kDecodeThreads, 3) decode_kernel(const __grid_
         err |= PRCR_ST_CAPACITY;
         len = int64_t(a.splits) * a.chunk;
     }
+    // A query position beyond the fixed-point angle reduction (|p| >= 2^31)
+    // is reported and the sequence attends to nothing: its output is zeros.
+    const int64_t p = a.q_pos[b];
+    if (p <= -2147483648LL || p >= 2147483648LL) {
+        err |= PRCR_ST_POS_RANGE;
+        len = 0;
+    }
     const int64_t s_begin = int64_t(split) * a.chunk;
     const int64_t s_end = min(len, s_begin + a.chunk);
 
@@ -80,8 +87,6 @@ __global__ void __launch_bounds__(kDecodeThreads, 3) decode_kernel(const __grid_
     // With the same position on every axis, pair i turns by p * inv_freq_i
     // whatever its band, so each pair's cos/sin serves all heads.
     __shared__ float s_cos[kMaxPairs], s_sin[kMaxPairs];
-    const int64_t p = a.q_pos[b];
-    if (p <= -2147483648LL || p >= 2147483648LL) err |= PRCR_ST_POS_RANGE;  // fixed-point angle range
     for (int i = threadIdx.x; i < P; i += blockDim.x) {
         sincos_turns(double(p), a.turn_freq[i], &s_sin[i], &s_cos[i]);
     }
@@ -353,6 +358,12 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
         err |= PRCR_ST_CAPACITY;
         len = int64_t(a.splits) * a.chunk;
     }
+    // A query position beyond the fixed-point angle reduction (|p| >= 2^31)
+    // is reported and the sequence attends to nothing: its output is zeros.
+    if (p <= -2147483648LL || p >= 2147483648LL) {
+        err |= PRCR_ST_POS_RANGE;
+        len = 0;
+    }
     const int64_t s_begin = int64_t(split) * a.chunk;
     const int64_t s_end = min(len, s_begin + a.chunk);
     if constexpr (HG) {
@@ -386,7 +397,6 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
 
     __shared__ __align__(16) float s_cos[kMaxPairs];
     __shared__ __align__(16) float s_sin[kMaxPairs];
-    if (p <= -2147483648LL || p >= 2147483648LL) err |= PRCR_ST_POS_RANGE;  // fixed-point angle range
     for (int i = threadIdx.x; i < P; i += blockDim.x) {
         sincos_turns(double(p), a.turn_freq[i], &s_sin[i], &s_cos[i]);
     }

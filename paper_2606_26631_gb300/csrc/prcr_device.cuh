@@ -210,7 +210,27 @@ struct RevisitCtx {
     int lo[3], hi[3];
     bool tab[3];
     bool center;
+    bool inexact;  // some position of this revisit cannot be formed exactly
 };
+
+// Whether every position of revisit r is an exact rational with operands
+// below 2^52 (the condition pcr_position / uir_position test per token; it
+// depends only on the revisit: p, L, K and the axis spans). Needs r.lo/r.hi.
+__device__ __forceinline__ void revisit_exactness(const PlanArgs& a, RevisitCtx& r) {
+    bool ok = true;
+    if (a.mode == PRCR_MODE_PCR) {
+#pragma unroll
+        for (int ax = 0; ax < 3; ++ax) {
+            const int64_t span = int64_t(r.hi[ax]) - int64_t(r.lo[ax]);
+            const double Q = span > 0 ? double(r.K + 1) * double(span)
+                                      : double(r.center ? 2 * (r.K + 1) : r.K + 1);
+            ok = ok && exact_ok(r.p - a.L, a.L, Q);
+        }
+    } else if (a.mode == PRCR_MODE_UIR) {
+        ok = exact_ok(r.p, 0, double(r.K + 1));
+    }
+    r.inexact = !ok;
+}
 
 // Physical destination row offset of `slot` (layer term excluded), or -1.
 __device__ __forceinline__ int64_t dest_row(const PlanArgs& a, const RevisitCtx& r, int64_t slot,
@@ -287,11 +307,16 @@ __device__ __forceinline__ void token_plan(const PlanArgs& a, const RevisitCtx& 
             break;
         }
     }
-    // the rotation reduces angles in 32.32 fixed point: |position| < 2^31
-    if (!(fabs(pos[0]) < 2147483648.0 && fabs(pos[1]) < 2147483648.0 &&
-          fabs(pos[2]) < 2147483648.0))
-        err |= PRCR_ST_POS_RANGE;
     src = int64_t(r.b) * a.store_seq_stride + int64_t(m) * a.store_token_stride;
+    // The rotation reduces angles in 32.32 fixed point (|position| < 2^31),
+    // and a position must be the correctly rounded exact value: otherwise the
+    // status bit is set and the token's rows are skipped (its position
+    // outputs keep the value computed).
+    if (r.inexact || !(fabs(pos[0]) < 2147483648.0 && fabs(pos[1]) < 2147483648.0 &&
+                       fabs(pos[2]) < 2147483648.0)) {
+        err |= PRCR_ST_POS_RANGE;
+        return;
+    }
     dst = dest_row(a, r, slot, blk, err);
 }
 
@@ -320,6 +345,7 @@ __device__ __forceinline__ bool revisit_ctx(const PlanArgs& a, int r, RevisitCtx
     x.center = (a.flags & PRCR_FLAG_DEGENERATE_CENTER) != 0;
     x.capacity = a.cache_kind == PRCR_CACHE_CONTIGUOUS ? int64_t(a.max_slots)
                                                        : int64_t(a.bt_stride) * a.block_size;
+    x.inexact = false;
     return true;
 }
 

@@ -143,6 +143,7 @@ __global__ void __launch_bounds__(512) fused_kernel(const __grid_constant__ Fuse
             x.hi[ax] = mx[ax];
             x.tab[ax] = false;
         }
+        revisit_exactness(a, x);
         const int64_t j0 = max(int64_t(x.beg), tok0), j1 = min(int64_t(x.end), tok1);
         for (int64_t j = j0 + threadIdx.x; j < j1; j += blockDim.x) {
             const int m = a.idx[j];

@@ -274,6 +274,12 @@ struct SelectArgs {
     uint64_t turn_freq[kMaxPairs];  // pair i: round(inv_freq_i / (2 pi) * 2^64)
 };
 
+// Every argument check of prcr_rebind_inject except the workspace's: PRCR_OK
+// or the negative code that call would return.
+int check_revisit_args(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
+                       const prcr_cache_desc* cache, const prcr_revisit_batch* b,
+                       const prcr_outputs* o, int32_t mode, int32_t L, int32_t flags);
+
 cudaError_t launch_select(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream);
 // the logits of the cached-key selection, then the same normaliser, relevance
 // and selection kernels

@@ -108,6 +108,7 @@ __device__ void plan_revisit(const PlanArgs& a, int r, int* s_part, double (*s_t
         const int64_t span = int64_t(mx[ax]) - int64_t(mn[ax]);
         x.tab[ax] = a.mode == PRCR_MODE_PCR && span >= 0 && span < kPosTable;
     }
+    revisit_exactness(a, x);
 
     // A PCR position depends on the token only through c - lo: tabulate the
     // span + 1 exact values of each axis once (one division each).

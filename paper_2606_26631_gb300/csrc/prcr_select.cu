@@ -528,6 +528,7 @@ __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
     float* lg_base[2] = {nullptr, nullptr};
     float* ts_base[2] = {nullptr, nullptr};
     int cur_b = -1, cur_kh = -1;
+    bool q_ok = true;  // the sequence's query position is within the angle range
     Item cur, nxt, pf;
     {
         const int64_t bk = i_beg / NT;
@@ -549,8 +550,11 @@ __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
         const int b = cur.b, kh = cur.kh, j = cur.j;
         if (b != cur_b || kh != cur_kh) {
             // the group's queries turned at (p, p, p), pre-scaled, as A fragments
+            // a query position beyond the fixed-point angle reduction is
+            // reported and the sequence's logits are all -inf (relevance 0)
             const int64_t p = a.q_pos[b];
-            if (p <= -2147483648LL || p >= 2147483648LL) err |= PRCR_ST_POS_RANGE;
+            q_ok = p > -2147483648LL && p < 2147483648LL;
+            if (!q_ok) err |= PRCR_ST_POS_RANGE;
             const uint16_t* qg = a.q + (int64_t(b) * Hq + kh * g) * D;
             for (int i = lane; i < P; i += 32) {
                 float sn, cs;
@@ -585,7 +589,7 @@ __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
         // S^T (16 tokens x 8 columns = the group's query heads, columns >= g
         // zero) = K Q^T: rows gid (kn[0]) and gid + 8 (kn[1]) are this lane's
         // tokens, and the query fragments serve as the B operand unchanged
-        const uint32_t mask = mask_n;
+        const uint32_t mask = q_ok ? mask_n : 0u;
         float c[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
         for (int k = 0; k < KS; ++k) {
@@ -676,8 +680,10 @@ __global__ void __launch_bounds__(256) ads_norm_kernel(const __grid_constant__ S
         float zt = 0.0f;
         for (int w = 0; w < nw; ++w) zt += s_z[w];
         float* nrm = a.norm + (int64_t(b) * a.n_q_heads + hq) * 2;
-        nrm[0] = mx;
-        nrm[1] = 1.0f / (zt * float(a.n_q_heads));
+        // no finite logit (no readable token, or a query position out of
+        // range): every weight of this head is taken as 0
+        nrm[0] = mx == -INFINITY ? 0.0f : mx;
+        nrm[1] = mx == -INFINITY ? 0.0f : 1.0f / (zt * float(a.n_q_heads));
     }
 }
 

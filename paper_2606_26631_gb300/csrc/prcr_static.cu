@@ -13,7 +13,11 @@
 // device address is looked up once per device (cudaGetSymbolAddress, with
 // that device current) on the first call made on that device, and passed to
 // the kernels as their workspace. That first call therefore does set-up work
-// and should come before any stream capture.
+// and should come before any stream capture. The address is kept for the
+// life of the process: after a reset of the device (cudaDeviceReset, or its
+// primary context released and created again) the library's module is
+// loaded anew and the kept address is stale, so this entry point must not be
+// called on a device after such a reset.
 //
 // All calls share the one array and it keeps whatever the last call left:
 // calls whose work overlaps on the GPU (different streams, or several host
@@ -59,7 +63,10 @@ extern "C" PRCR_API int prcr_rebind_inject_static(const prcr_rope_cfg* cfg,
                                                   const prcr_revisit_batch* batch,
                                                   const prcr_outputs* out, int32_t mode,
                                                   int32_t L, int32_t flags, void* stream) {
-    if (batch == nullptr || batch->total_k < 0) return PRCR_EINVAL;
+    // the call's own checks first, so that a malformed call gets the code
+    // prcr_rebind_inject would return and does no set-up
+    const int rc0 = prcr::check_revisit_args(cfg, store, cache, batch, out, mode, L, flags);
+    if (rc0 != PRCR_OK || batch->n_seqs == 0) return rc0;
     if (batch->total_k > PRCR_STATIC_MAX_TOKENS) return PRCR_EWORKSPACE;
     if (prcr::workspace_bytes(batch->total_k) > kStaticBytes) return PRCR_EWORKSPACE;
     void* ws = nullptr;

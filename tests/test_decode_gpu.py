@@ -173,17 +173,32 @@ def test_decode_device_errors():
 
 def test_decode_query_position_range():
     """A query position of 2^31 or more is beyond the fixed-point angle
-    reduction: PRCR_ST_POS_RANGE (head-split and one-CTA-per-chunk kernels)."""
+    reduction: PRCR_ST_POS_RANGE, and that sequence reads no slot (its output
+    is zeros) while the other sequence of the batch matches the oracle.
+    Head-split and one-CTA-per-chunk kernels, split and unsplit sequences."""
     import paper_2606_26631_gb300 as prcr
-    for H, Hq in ((8, 32), (2, 8)):
-        inp = make_decode_inputs(1, 2, H, Hq, 128, 300, False, device=DEV, seed=5)
-        cfg = prcr.rope_cfg(2, H, 128, (16, 24, 24), 1e6)
+    sec = (16, 24, 24)
+    for H, Hq, max_len in ((8, 32, 300), (2, 8, 300), (8, 32, 3000)):
+        inp = make_decode_inputs(2, 2, H, Hq, 128, max_len, False, device=DEV, seed=5)
+        cfg = prcr.rope_cfg(2, H, 128, sec, 1e6)
         cd = prcr.cache_contiguous(inp["cache_k"], inp["cache_v"])
-        qp = torch.tensor([2 ** 31], dtype=torch.int64, device=DEV)
-        _, st = _run_decode(cfg, cd, inp["q"], qp, inp["seq_len"], 300)
-        assert st & prcr.ST_POS_RANGE
-        qp = torch.tensor([2 ** 31 - 1], dtype=torch.int64, device=DEV)
-        _, st = _run_decode(cfg, cd, inp["q"], qp, inp["seq_len"], 300)
+        qp = inp["q_pos"].clone()
+        qp[0] = 2 ** 31
+        out, st = _run_decode(cfg, cd, inp["q"], qp, inp["seq_len"], max_len)
+        assert st == prcr.ST_POS_RANGE
+        got = out.cpu().numpy()
+        assert np.all(got[0] == 0.0)
+        n = int(inp["seq_len"][1])
+        K, V = _cache_rows(inp["cache_k"], inp["cache_v"], None, 1, n, False)
+        qv = _f64(inp["q"])
+        for l in range(2):
+            ref = O.decode_attention(qv[1, l], int(qp[1]), K[:, l], V[:, l], 128, sec, 1e6)
+            assert np.abs(got[1, l] - ref).max() / np.abs(V[:, l]).max() <= 1e-4
+        qp[0] = -(2 ** 31)
+        out, st = _run_decode(cfg, cd, inp["q"], qp, inp["seq_len"], max_len)
+        assert st == prcr.ST_POS_RANGE and bool((out[0] == 0).all().item())
+        qp[0] = 2 ** 31 - 1
+        _, st = _run_decode(cfg, cd, inp["q"], qp, inp["seq_len"], max_len)
         assert st == 0
 
 

@@ -399,15 +399,34 @@ def test_bad_index_small_batch():
 
 def test_position_beyond_angle_range_is_flagged():
     """Text positions of 2^31 and more are beyond the fixed-point angle
-    reduction: the call sets PRCR_ST_POS_RANGE (one-kernel and two-kernel
-    paths); a position well inside the range does not."""
+    reduction: the call sets PRCR_ST_POS_RANGE and skips those tokens' rows
+    (they keep the canary), while the other sequences of the same batch get
+    the oracle's positions and rows. One-kernel path (2 sequences, ~1000
+    tokens) and two-kernel path (8 sequences); a position well inside the
+    range sets nothing."""
+    import dataclasses
     import paper_2606_26631_gb300 as prcr
     import parity_util as pu
+    for n_seqs, bad_seqs in ((2, [1]), (8, [0, 5])):
+        wl = dataclasses.replace(get("qwen25vl-7b"), n_seqs=n_seqs, n_layers=3)
+        batch = make_batch(wl, device=DEV, seed=4)
+        for b in bad_seqs:
+            batch.p_txt[b] = 2 ** 31 + 100 + b
+        pl = pu.oracle_plan(batch)
+        rv = pu.make_revisit(batch)
+        launched = _kernel_names(rv.run)  # runs the call once
+        assert launched == (["fused_kernel"] if n_seqs == 2 else ["plan_kernel", "rebind_kernel"]), launched
+        assert rv.status_value() == prcr.ST_POS_RANGE, (n_seqs, rv.status_value())
+        good = np.nonzero(~np.isin(pl["seq"], bad_seqs))[0]
+        assert 0 < len(good) < batch.total_k
+        got_pos = rv.pos.cpu().numpy()
+        assert np.array_equal(got_pos[good].view(np.int64), pl["pos"][good].view(np.int64))
+        assert np.array_equal(rv.slot.cpu().numpy()[good].astype(np.int64), pl["slot"][good])
+        assert np.array_equal(rv.cache_len_out.cpu().numpy().astype(np.int64), pl["cache_len_out"])
+        assert np.array_equal(rv.next_pos.cpu().numpy(), pl["next_pos"])
+        pu.check_rows(batch, rv, pl, good, range(wl.n_layers))
+        pu.check_untouched(batch, pl, written=good)
     for name in ("tiny", "qwen25vl-7b"):
-        batch = make_batch(get(name), device=DEV, seed=4)
-        batch.p_txt.fill_(2 ** 31 + 100)
-        rv = _run(batch)
-        assert rv.status_value() & prcr.ST_POS_RANGE, name
         batch = make_batch(get(name), device=DEV, seed=4)
         batch.p_txt.fill_(2 ** 31 - 2 ** 20)
         rv = _run(batch)

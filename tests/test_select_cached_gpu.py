@@ -299,12 +299,24 @@ def test_select_most_query_heads(cached):
 
 
 def test_select_cached_query_position_range():
-    """A query position of 2^31 or more sets PRCR_ST_POS_RANGE."""
+    """A query position of 2^31 or more sets PRCR_ST_POS_RANGE; every token of
+    that sequence gets relevance 0, so it selects its first k tokens (equal
+    relevance: lower index first), while the other sequence of the batch keeps
+    the oracle's relevance and a valid selection."""
     import paper_2606_26631_gb300 as prcr
-    cache_k, bt, img0 = _make_cache(1, 1, 2, 64, 40, False, 0, seed=3)
-    cfg = prcr.rope_cfg(1, 2, 64, (8, 12, 12), 1e6)
-    q = torch.randn((1, 4, 64), device=DEV).to(torch.bfloat16)
-    for pos, bad in ((2 ** 31 + 7, True), (2 ** 31 - 1, False)):
-        qp = torch.tensor([pos], dtype=torch.int64, device=DEV)
-        _, _, _, _, st = _run(cfg, prcr.cache_contiguous(cache_k, cache_k), 0, q, qp, img0, 40, 5)
-        assert bool(st & prcr.ST_POS_RANGE) == bad
+    D, H, Hq, M, k, sec = 64, 2, 8, 40, 5, (8, 12, 12)
+    cache_k, bt, img0 = _make_cache(2, 1, H, D, M, False, 0, seed=3)
+    cfg = prcr.rope_cfg(1, H, D, sec, 1e6)
+    q = torch.randn((2, Hq, D), device=DEV).to(torch.bfloat16)
+    qv = O.bf16_bits_to_f64(q.view(torch.int16).cpu().numpy())
+    cd = prcr.cache_contiguous(cache_k, cache_k)
+    for pos, bad in ((2 ** 31 + 7, True), (-(2 ** 31), True), (2 ** 31 - 1, False)):
+        qp = torch.tensor([pos, 700], dtype=torch.int64, device=DEV)
+        idx, _, _, score, st = _run(cfg, cd, 0, q, qp, img0, M, k)
+        assert st == (prcr.ST_POS_RANGE if bad else 0)
+        if bad:
+            assert np.all(score[0] == 0.0)
+            assert np.array_equal(idx[0], np.arange(k))
+        kc = _image_rows(cache_k, None, img0.cpu().numpy(), 1, 0, M)
+        ref = O.ads_relevance_cached(qv[1], 700, kc, D, sec, 1e6)
+        _check_seq(score[1], ref, idx[1], k, M)
