@@ -505,7 +505,9 @@ int prcr_rebind_inject(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
         int dev = 0;
         if (cudaGetDevice(&dev) != cudaSuccess) return PRCR_ECUDA;
         const int64_t resident = int64_t(sm_count(dev)) * blocks_per_sm(dev, block, smem, kFused);
-        if (int64_t(grid.x) * grid.y <= resident) {
+        // (its CTA loads the offsets with one thread per entry)
+        if (int64_t(grid.x) * grid.y <= resident && block > kFusedMaxRevisits &&
+            block > kFusedMaxSeqs) {
             fa.plan = make_plan_args(store, cache, batch, out, mode, L, flags, workspace);
             return launch_fused(fa, grid, block, smem, s) == cudaSuccess ? PRCR_OK : PRCR_ECUDA;
         }

@@ -124,15 +124,26 @@ __device__ __forceinline__ void stream_layers(const uint16_t* sk, const uint16_t
     }
 }
 
-constexpr double kExactLimit = 4503599627370496.0;  // 2^52
 constexpr int kTokPerThread = 4;   // tokens of a revisit each thread keeps in registers
 constexpr int kPosTable = 1024;    // exact PCR positions tabulated per axis when span < this
 
-// True when every integer formed for p_hat = ((p - L) * Q + tail) / Q with
-// 0 <= tail <= (L+1) * Q stays below 2^52 in magnitude, so that the integer
-// products cannot overflow and the float64 division sees exact operands.
-__device__ __forceinline__ bool exact_ok(int64_t p_minus_l, int32_t L, double Q) {
-    return (fabs(double(p_minus_l)) + double(L) + 1.0) * Q < kExactLimit;
+// True when (|p - L| + L + 1) * Q < 2^52 (Q >= 1), i.e. every integer formed
+// for p_hat = ((p - L) * Q + tail) / Q with 0 <= tail <= (L+1) * Q stays
+// below 2^52 in magnitude, so that the integer products cannot overflow and
+// the float64 division sees exact operands. Integer arithmetic only (GB300's
+// float64 pipe is narrow and shared by every warp of an SM sub-partition).
+__device__ __forceinline__ bool exact_ok(int64_t p_minus_l, int32_t L, uint64_t Q) {
+    const int64_t lim = int64_t(1) << 62;
+    if (p_minus_l <= -lim || p_minus_l >= lim) return false;
+    const uint64_t a = uint64_t(p_minus_l < 0 ? -p_minus_l : p_minus_l) + uint64_t(L) + 1u;
+    return __umul64hi(a, Q) == 0 && a * Q < (uint64_t(1) << 52);
+}
+
+// The denominator Q of the PCR position on an axis of the given span:
+// (K+1) * span, or (K+1) (2 (K+1) with the centre reading) when the axis is
+// degenerate (span <= 0).
+__device__ __forceinline__ uint64_t pcr_denominator(int64_t K, int64_t span, bool center) {
+    return span > 0 ? uint64_t(K + 1) * uint64_t(span) : uint64_t(center ? 2 * (K + 1) : K + 1);
 }
 
 __device__ __forceinline__ double pcr_position(int64_t p, int32_t L, int64_t K, int32_t c,
@@ -140,27 +151,26 @@ __device__ __forceinline__ double pcr_position(int64_t p, int32_t L, int64_t K, 
                                                uint32_t& err) {
     const int64_t span = int64_t(hi) - int64_t(lo);
     const int64_t pl = p - L;
+    const uint64_t Q = pcr_denominator(K, span, center);
     if (span > 0) {
-        if (exact_ok(pl, L, double(K + 1) * double(span))) {
-            const int64_t Q = (K + 1) * span;
+        if (exact_ok(pl, L, Q)) {
             const int64_t tail = int64_t(L + 1) * (span + (K - 1) * (int64_t(c) - lo));
-            return double(pl * Q + tail) / double(Q);
+            return double(pl * int64_t(Q) + tail) / double(Q);
         }
         err |= PRCR_ST_POS_RANGE;
         const double u = double(int64_t(c) - lo) / double(span);
         return double(pl) + double(L + 1) * (1.0 + double(K - 1) * u) / double(K + 1);
     }
     // degenerate axis: u = 0, or u = 1/2 with the centre reading
-    const int64_t Q = center ? 2 * (K + 1) : K + 1;
     const int64_t tail = center ? int64_t(L + 1) * (K + 1) : int64_t(L + 1);
-    if (exact_ok(pl, L, double(Q))) return double(pl * Q + tail) / double(Q);
+    if (exact_ok(pl, L, Q)) return double(pl * int64_t(Q) + tail) / double(Q);
     err |= PRCR_ST_POS_RANGE;
     return double(pl) + double(tail) / double(Q);
 }
 
 // p + num / (K + 1), exact while representable (UIR).
 __device__ __forceinline__ double uir_position(int64_t p, int64_t num, int64_t K, uint32_t& err) {
-    if (exact_ok(p, 0, double(K + 1))) return double(p * (K + 1) + num) / double(K + 1);
+    if (exact_ok(p, 0, uint64_t(K + 1))) return double(p * (K + 1) + num) / double(K + 1);
     err |= PRCR_ST_POS_RANGE;
     return double(p) + double(num) / double(K + 1);
 }
@@ -213,6 +223,12 @@ struct RevisitCtx {
     bool inexact;  // some position of this revisit cannot be formed exactly
 };
 
+// |pos| < 2^31 (and not NaN), tested on the bits (no float64 instruction).
+__device__ __forceinline__ bool pos_in_range(double pos) {
+    return (static_cast<unsigned long long>(__double_as_longlong(pos)) & 0x7fffffffffffffffull) <
+           0x41e0000000000000ull;
+}
+
 // Whether every position of revisit r is an exact rational with operands
 // below 2^52 (the condition pcr_position / uir_position test per token; it
 // depends only on the revisit: p, L, K and the axis spans). Needs r.lo/r.hi.
@@ -220,14 +236,11 @@ __device__ __forceinline__ void revisit_exactness(const PlanArgs& a, RevisitCtx&
     bool ok = true;
     if (a.mode == PRCR_MODE_PCR) {
 #pragma unroll
-        for (int ax = 0; ax < 3; ++ax) {
-            const int64_t span = int64_t(r.hi[ax]) - int64_t(r.lo[ax]);
-            const double Q = span > 0 ? double(r.K + 1) * double(span)
-                                      : double(r.center ? 2 * (r.K + 1) : r.K + 1);
-            ok = ok && exact_ok(r.p - a.L, a.L, Q);
-        }
+        for (int ax = 0; ax < 3; ++ax)
+            ok = ok && exact_ok(r.p - a.L, a.L,
+                                pcr_denominator(r.K, int64_t(r.hi[ax]) - int64_t(r.lo[ax]), r.center));
     } else if (a.mode == PRCR_MODE_UIR) {
-        ok = exact_ok(r.p, 0, double(r.K + 1));
+        ok = exact_ok(r.p, 0, uint64_t(r.K + 1));
     }
     r.inexact = !ok;
 }
@@ -312,8 +325,7 @@ __device__ __forceinline__ void token_plan(const PlanArgs& a, const RevisitCtx& 
     // and a position must be the correctly rounded exact value: otherwise the
     // status bit is set and the token's rows are skipped (its position
     // outputs keep the value computed).
-    if (r.inexact || !(fabs(pos[0]) < 2147483648.0 && fabs(pos[1]) < 2147483648.0 &&
-                       fabs(pos[2]) < 2147483648.0)) {
+    if (r.inexact || !(pos_in_range(pos[0]) && pos_in_range(pos[1]) && pos_in_range(pos[2]))) {
         err |= PRCR_ST_POS_RANGE;
         return;
     }

@@ -2,14 +2,26 @@
 //
 // For a few revisits of modest size the two-kernel path is pure latency: the
 // plan kernel, the wait for it, and the rebind kernel's reload of the plan.
-// Here every CTA plans the tokens it moves itself. It first checks the whole
-// offset structure (small by construction: the host sends only batches of a
-// few revisits here), so that a malformed batch is reported and writes
-// nothing, exactly as on the two-kernel path; then, for each revisit its
-// tokens belong to, it reduces the revisit's coordinate range cooperatively
-// and gives its tokens their positions, slots and rows with the same exact
-// arithmetic as the plan kernel (token_plan); then it streams the rows as the
-// rebind kernel does.
+// Here every CTA plans the tokens it moves itself, with as few dependent
+// memory round trips as the data allow:
+//   A. the offsets, text positions, cache lengths and every selected index of
+//      the batch (at most kFusedMaxTokens) are loaded into shared memory in
+//      one round trip, and the offsets are checked there: a malformed batch
+//      is reported and writes nothing, exactly as on the two-kernel path;
+//   B. the first rows of the CTA's own tokens, their block-table entries and
+//      coordinates, and the coordinates of every token of the revisits the
+//      tile touches are requested together;
+//   C. per revisit the coordinate range is reduced (Eq. "selected_coord_range")
+//      and the positions of Eq. "image_range_fractional_reinsert" (or the
+//      rule the mode selects) are formed with the plan kernel's exact
+//      arithmetic, one (token, axis) per lane: GB300's float64 pipe takes
+//      many cycles per warp instruction whatever its active lanes, so the
+//      divisions of a tile share warp instructions instead of following each
+//      other;
+//   D. cos/sin of the tile from the positions in 32.32 fixed point;
+//   E. the rows already in registers are rotated and stored, and the
+//      group's other layers streamed as in the rebind kernel.
+// Results are bit-identical to plan + rebind.
 #include "prcr_device.cuh"
 #include "prcr_pdl.cuh"
 
@@ -18,114 +30,196 @@ namespace {
 
 constexpr int kFusedMaxTile = 256;  // tokens per CTA (256 / lanes at most)
 
+// Last index r in [0, n) with off[r] <= v (off non-decreasing, off[0] <= v).
+__device__ __forceinline__ int last_at_or_before(const int* off, int n, int64_t v) {
+    int lo = 0, hi = n;
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (off[mid] <= v) lo = mid; else hi = mid;
+    }
+    return lo;
+}
+
 __global__ void __launch_bounds__(512) fused_kernel(const __grid_constant__ FusedArgs fa) {
     const PlanArgs& a = fa.plan;
     const RebindArgs& rb = fa.rebind;
-    extern __shared__ float smem[];
-    __shared__ int64_t s_src[kFusedMaxTile], s_dst[kFusedMaxTile];
-    __shared__ double s_pos[3 * kFusedMaxTile];
+    extern __shared__ float smem[];  // cos / sin of the tile
+    __shared__ int s_idx[kFusedMaxTokens];
+    __shared__ int s_rto[kFusedMaxRevisits + 1];
+    __shared__ int s_sro[kFusedMaxSeqs + 1];
+    __shared__ long long s_p[kFusedMaxSeqs];
+    __shared__ int s_clen[kFusedMaxSeqs];
+    __shared__ long long s_pf[kFusedMaxTile][3];  // positions in 32.32 fixed point
+    __shared__ int s_c[kFusedMaxTile][3];         // stored coordinates of the tile's tokens
+    __shared__ long long s_dst[kFusedMaxTile];    // cache row (layer term excluded), -1 = skip
+    __shared__ int s_skip[kFusedMaxTile];         // position out of range: rows skipped
     __shared__ int s_part[33 * 6];
-    __shared__ int s_bad;
-    const bool lead = blockIdx.x == 0 && blockIdx.y == 0;
 
-    // 0. the per-sequence inputs are prefetched while the grid this one
-    // depends on finishes; this thread's token index is requested before the
-    // offsets are checked, so that their latencies overlap
-    pdl_allow();
+    const int tid = threadIdx.x, bd = blockDim.x;
+    const bool lead = blockIdx.x == 0 && blockIdx.y == 0;
     const int T = rb.tok_per_cta;
-    const int64_t tok0 = int64_t(blockIdx.x) * T;
     const int lanes = rb.lanes;
-    const int my_t = threadIdx.x / lanes;
-    const int64_t my_j = tok0 + my_t;
-    const bool my_tok = my_t < T && my_j < a.total_k;
-    if (threadIdx.x < a.n_seqs) {
-        prefetch_l2(a.cache_len_in + threadIdx.x);
-        prefetch_l2(a.p_txt + threadIdx.x);
+    const int64_t tok0 = int64_t(blockIdx.x) * T;
+    const int total = int(a.total_k);
+    const int64_t tok1 = min(tok0 + T, int64_t(total));
+    const int n_seqs = a.n_seqs, n_rev = a.n_revisits;
+
+    // 0. the per-sequence inputs are requested into L2 while the grid this
+    // one depends on finishes
+    pdl_allow();
+    if (tid < n_seqs) {
+        prefetch_l2(a.cache_len_in + tid);
+        prefetch_l2(a.p_txt + tid);
     }
     pdl_wait();
-    const int my_m = my_tok ? a.idx[my_j] : -1;
 
-    // 1. the offsets: monotone, spanning [0, total_k) and [0, n_revisits)
-    if (threadIdx.x == 0) s_bad = 0;
+    // A. offsets, positions, lengths and indices into shared memory, one
+    // round trip (loads first, then the shared stores)
+    {
+        int ro = 0, so = 0, cl = 0;
+        long long pt = 0;
+        if (tid <= n_rev) ro = a.rev_tok_off[tid];
+        if (tid <= n_seqs) so = a.seq_rev_off[tid];
+        if (tid < n_seqs) {
+            pt = a.p_txt[tid];
+            cl = a.cache_len_in[tid];
+        }
+        for (int base = 0; base < total; base += 8 * bd) {
+            int v[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int i = base + tid + u * bd;
+                v[u] = i < total ? a.idx[i] : 0;
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int i = base + tid + u * bd;
+                if (i < total) s_idx[i] = v[u];
+            }
+        }
+        if (tid <= n_rev) s_rto[tid] = ro;
+        if (tid <= n_seqs) s_sro[tid] = so;
+        if (tid < n_seqs) {
+            s_p[tid] = pt;
+            s_clen[tid] = cl;
+        }
+    }
     __syncthreads();
+    // the offsets: monotone, spanning [0, total_k) and [0, n_revisits)
     bool bad = false;
-    for (int i = threadIdx.x; i < a.n_seqs; i += blockDim.x) {
-        const int r0 = a.seq_rev_off[i], r1 = a.seq_rev_off[i + 1];
-        bad |= r0 < 0 || r1 < r0 || r1 > a.n_revisits;
-    }
-    for (int r = threadIdx.x; r < a.n_revisits; r += blockDim.x) {
-        const int t0 = a.rev_tok_off[r], t1 = a.rev_tok_off[r + 1];
-        bad |= t0 < 0 || t1 < t0 || int64_t(t1) > a.total_k;
-    }
-    if (threadIdx.x == 0)
-        bad |= a.seq_rev_off[0] != 0 || a.seq_rev_off[a.n_seqs] != a.n_revisits ||
-               a.rev_tok_off[0] != 0 || int64_t(a.rev_tok_off[a.n_revisits]) != a.total_k;
-    if (bad) atomicOr(&s_bad, 1);
-    __syncthreads();
-    if (s_bad) {
-        if (lead && threadIdx.x == 0) atomicOr(a.status, PRCR_ST_CSR);
+    if (tid < n_seqs) bad = s_sro[tid] < 0 || s_sro[tid + 1] < s_sro[tid] || s_sro[tid + 1] > n_rev;
+    if (tid < n_rev) bad |= s_rto[tid] < 0 || s_rto[tid + 1] < s_rto[tid] || s_rto[tid + 1] > total;
+    if (tid == 0)
+        bad |= s_sro[0] != 0 || s_sro[n_seqs] != n_rev || s_rto[0] != 0 || s_rto[n_rev] != total;
+    if (__syncthreads_or(bad)) {
+        if (lead && tid == 0) atomicOr(a.status, PRCR_ST_CSR);
         return;
     }
-    // 1b. with the offsets checked (and in L1): the token's revisit and
-    // sequence, then its coordinates and its first layer's rows are
-    // prefetched while the revisit ranges are reduced
-    if (my_tok && my_m >= 0 && my_m < a.n_tokens) {
-        int r0 = 0, r1 = a.n_revisits;  // last revisit starting at or before my_j
-        while (r1 - r0 > 1) {
-            const int mid = (r0 + r1) >> 1;
-            if (a.rev_tok_off[mid] <= my_j) r0 = mid; else r1 = mid;
-        }
-        int s0 = 0, s1 = a.n_seqs;  // last sequence whose first revisit is at or before r0
-        while (s1 - s0 > 1) {
-            const int mid = (s0 + s1) >> 1;
-            if (a.seq_rev_off[mid] <= r0) s0 = mid; else s1 = mid;
-        }
-        const int lane = threadIdx.x - my_t * lanes;
-        if (lane == 0) prefetch_l2(a.coords + int64_t(s0) * a.coord_seq_stride + 3 * int64_t(my_m));
-        if (lane == 1 && a.cache_kind == PRCR_CACHE_PAGED) {
-            // the block-table entry of the token's slot (as token_plan finds it)
-            const int64_t slot = int64_t(a.cache_len_in[s0]) + (my_j - a.rev_tok_off[a.seq_rev_off[s0]]);
-            if (slot >= 0 && slot < int64_t(a.bt_stride) * a.block_size)
-                prefetch_l2(a.block_table + int64_t(s0) * a.bt_stride + slot / a.block_size);
-        }
-        const int vph = rb.head_dim >> 4;
-        const int64_t row = int64_t(s0) * a.store_seq_stride + int64_t(my_m) * a.store_token_stride +
-                            int64_t(blockIdx.y) * rb.layers_per_cta * rb.store_layer_stride +
-                            int64_t(lane / vph) * rb.head_dim + (lane % vph) * 8;
-        prefetch_l2(rb.store_k + row);
-        prefetch_l2(rb.store_k + row + (rb.head_dim >> 1));
-        prefetch_l2(rb.store_v + row);
-        prefetch_l2(rb.store_v + row + (rb.head_dim >> 1));
-    }
+
     uint32_t err = 0;
     if (lead) {
-        for (int b = threadIdx.x; b < a.n_seqs; b += blockDim.x) {
-            const int64_t k = int64_t(a.rev_tok_off[a.seq_rev_off[b + 1]]) - a.rev_tok_off[a.seq_rev_off[b]];
-            const int64_t len = int64_t(a.cache_len_in[b]) + k;
+        for (int b = tid; b < n_seqs; b += bd) {
+            const int64_t k = int64_t(s_rto[s_sro[b + 1]]) - s_rto[s_sro[b]];
+            const int64_t len = int64_t(s_clen[b]) + k;
             if (len > INT_MAX) err |= PRCR_ST_CAPACITY;
             a.cache_len_out[b] = int32_t(len > INT_MAX ? INT_MAX : len);
-            const int64_t p = a.p_txt[b];
-            a.next_pos_out[b] = a.mode == PRCR_MODE_LPA ? p + k + 1 : p + 1;
+            a.next_pos_out[b] = a.mode == PRCR_MODE_LPA ? s_p[b] + k + 1 : s_p[b] + 1;
         }
     }
 
-    // 2. plan of this CTA's tokens [tok0, tok1)
-    const int64_t tok1 = min(tok0 + T, a.total_k);
-    int ra = 0, hi = a.n_revisits;  // last revisit starting at or before tok0
-    while (hi - ra > 1) {
-        const int mid = (ra + hi) >> 1;
-        if (a.rev_tok_off[mid] <= tok0) ra = mid; else hi = mid;
+    // B. this thread's token: its sequence, index, slot and source row; the
+    // first layers' rows go to registers now, the block-table entry and the
+    // coordinates (lane 0) to shared memory
+    const int D = rb.head_dim;
+    const int P = D >> 1;
+    const int my_t = tid / lanes;
+    const int lane = tid - my_t * lanes;
+    const int64_t my_j = tok0 + my_t;
+    const bool my_tok = my_t < T && my_j < tok1;
+    const int l0 = blockIdx.y * rb.layers_per_cta;
+    const int l1 = min(l0 + rb.layers_per_cta, rb.n_layers);
+    const int64_t sls = rb.store_layer_stride;
+    const int64_t cls = rb.cache_layer_stride;
+    const int vph = D >> 4;
+    const int64_t off = int64_t(lane / vph) * D + (lane % vph) * 8;
+    uint4 k0a = {}, k1a = {}, v0a = {}, v1a = {}, k0b = {}, k1b = {}, v0b = {}, v1b = {};
+    int my_m = -1;
+    int my_b = 0;
+    int64_t my_slot = 0;
+    if (my_tok) {
+        const int r = last_at_or_before(s_rto, n_rev, my_j);
+        my_b = last_at_or_before(s_sro, n_seqs, r);
+        my_m = s_idx[my_j];
+        my_slot = int64_t(s_clen[my_b]) + (my_j - s_rto[s_sro[my_b]]);
+        if (my_m >= 0 && my_m < a.n_tokens) {
+            const int64_t src = int64_t(my_b) * a.store_seq_stride + int64_t(my_m) * a.store_token_stride;
+            const uint16_t* sk = rb.store_k + src + int64_t(l0) * sls + off;
+            const uint16_t* sv = rb.store_v + src + int64_t(l0) * sls + off;
+            k0a = ld_stream(sk);
+            k1a = ld_stream(sk + P);
+            v0a = ld_stream(sv);
+            v1a = ld_stream(sv + P);
+            if (l0 + 1 < l1) {
+                k0b = ld_stream(sk + sls);
+                k1b = ld_stream(sk + sls + P);
+                v0b = ld_stream(sv + sls);
+                v1b = ld_stream(sv + sls + P);
+            }
+            for (int l = l0 + 2; l < l1 && l < l0 + 4; ++l) {  // the next two layers into L2
+                prefetch_l2(sk + int64_t(l - l0) * sls);
+                prefetch_l2(sk + int64_t(l - l0) * sls + P);
+                prefetch_l2(sv + int64_t(l - l0) * sls);
+                prefetch_l2(sv + int64_t(l - l0) * sls + P);
+            }
+        }
+        if (lane == 0) {
+            // the token's coordinates and its cache row
+            int c[3];
+            load_coords(a.coords + int64_t(my_b) * a.coord_seq_stride, my_m, a.n_tokens, c);
+            const int64_t capacity = a.cache_kind == PRCR_CACHE_CONTIGUOUS
+                                         ? int64_t(a.max_slots)
+                                         : int64_t(a.bt_stride) * a.block_size;
+            const bool slot_ok = s_clen[my_b] >= 0 && my_slot < capacity;
+            int32_t blk = -1;
+            if (a.cache_kind == PRCR_CACHE_PAGED && slot_ok)
+                blk = a.block_table[int64_t(my_b) * a.bt_stride + my_slot / a.block_size];
+            s_c[my_t][0] = c[0];
+            s_c[my_t][1] = c[1];
+            s_c[my_t][2] = c[2];
+            s_skip[my_t] = 0;
+            int64_t dst = -1;
+            if (my_m < 0 || my_m >= a.n_tokens) {
+                err |= PRCR_ST_IDX_RANGE;
+            } else if (!slot_ok) {
+                err |= PRCR_ST_CAPACITY;
+            } else if (a.cache_kind == PRCR_CACHE_CONTIGUOUS) {
+                dst = int64_t(my_b) * a.cache_seq_stride + my_slot * a.slot_stride;
+            } else if (blk < 0 || blk >= a.n_blocks) {
+                err |= PRCR_ST_NO_BLOCK;
+            } else {
+                const int64_t lb = my_slot / a.block_size;
+                dst = int64_t(blk) * a.block_stride + (my_slot - lb * a.block_size) * a.slot_stride;
+            }
+            s_dst[my_t] = dst;
+            if (blockIdx.y == 0 && a.slot_out)
+                a.slot_out[my_j] = int32_t(my_slot > INT_MAX ? INT_MAX : my_slot);
+        }
     }
-    for (int r = ra; r < a.n_revisits && a.rev_tok_off[r] < tok1; ++r) {
-        RevisitCtx x;
-        revisit_ctx(a, r, x);  // consistent: checked above
-        if (x.K == 0) continue;
-        const int32_t* crd = a.coords + int64_t(x.b) * a.coord_seq_stride;
+
+    // C. per revisit the tile touches: its coordinate range, then the
+    // positions of its tokens in the tile, one (token, axis) per thread
+    const int ra = last_at_or_before(s_rto, n_rev, tok0);
+    for (int r = ra; r < n_rev && s_rto[r] < tok1; ++r) {
+        const int beg = s_rto[r], end = s_rto[r + 1];
+        if (end == beg) continue;
+        const int b = last_at_or_before(s_sro, n_seqs, r);
+        const int t0s = s_rto[s_sro[b]];  // the sequence's first token in this call
         int mn[3] = {INT_MAX, INT_MAX, INT_MAX};
         int mx[3] = {INT_MIN, INT_MIN, INT_MIN};
         if (a.mode == PRCR_MODE_PCR) {
-            for (int j = x.beg + threadIdx.x; j < x.end; j += blockDim.x) {
-                const int m = a.idx[j];
+            const int32_t* crd = a.coords + int64_t(b) * a.coord_seq_stride;
+            for (int j = beg + tid; j < end; j += bd) {
+                const int m = s_idx[j];
                 if (m >= 0 && m < a.n_tokens) {
 #pragma unroll
                     for (int ax = 0; ax < 3; ++ax) {
@@ -135,84 +229,104 @@ __global__ void __launch_bounds__(512) fused_kernel(const __grid_constant__ Fuse
                     }
                 }
             }
-            block_minmax(mn, mx, s_part);
+            block_minmax(mn, mx, s_part);  // ends with a barrier: s_c, s_dst are visible
+        } else {
+            __syncthreads();  // s_c, s_dst are visible
         }
-#pragma unroll
-        for (int ax = 0; ax < 3; ++ax) {
-            x.lo[ax] = mn[ax];
-            x.hi[ax] = mx[ax];
-            x.tab[ax] = false;
-        }
-        revisit_exactness(a, x);
-        const int64_t j0 = max(int64_t(x.beg), tok0), j1 = min(int64_t(x.end), tok1);
-        for (int64_t j = j0 + threadIdx.x; j < j1; j += blockDim.x) {
-            const int m = a.idx[j];
-            int c[3];
-            load_coords(crd, m, a.n_tokens, c);
-            double pos[3];
-            int64_t src, dst, slot;
-            token_plan(a, x, nullptr, int(j), m, c, block_of(a, x, x.clen + (j - x.t0)), err, pos,
-                       src, dst, slot);
-            const int t = int(j - tok0);
-            s_src[t] = src;
-            s_dst[t] = dst;
-            s_pos[3 * t] = pos[0];
-            s_pos[3 * t + 1] = pos[1];
-            s_pos[3 * t + 2] = pos[2];
-            if (blockIdx.y == 0) {
-                if (a.pos_out) {
-                    a.pos_out[3 * j] = pos[0];
-                    a.pos_out[3 * j + 1] = pos[1];
-                    a.pos_out[3 * j + 2] = pos[2];
+        const int64_t K = end - beg;
+        const int64_t p = s_p[b];
+        const bool center = (a.flags & PRCR_FLAG_DEGENERATE_CENTER) != 0;
+        const int j0 = max(beg, int(tok0)), j1 = min(end, int(tok1));
+        for (int q = tid; q < 3 * (j1 - j0); q += bd) {
+            const int j = j0 + q / 3, ax = q - (q / 3) * 3;
+            const int t = j - int(tok0);
+            const int m = s_idx[j];
+            double pos;
+            uint32_t e = 0;
+            if (m < 0 || m >= a.n_tokens) {
+                pos = __longlong_as_double(0x7ff8000000000000LL);
+            } else {
+                switch (a.mode) {
+                    case PRCR_MODE_PCR: {
+                        // (selects, not an indexed register array: no local memory)
+                        const int lo = ax == 0 ? mn[0] : (ax == 1 ? mn[1] : mn[2]);
+                        const int hi = ax == 0 ? mx[0] : (ax == 1 ? mx[1] : mx[2]);
+                        pos = pcr_position(p, a.L, K, s_c[t][ax], lo, hi, center, e);
+                        break;
+                    }
+                    case PRCR_MODE_ORIGINAL:
+                        pos = double(s_c[t][ax]);
+                        break;
+                    case PRCR_MODE_UIR:
+                        pos = uir_position(p, int64_t(j - beg + 1), K, e);
+                        break;
+                    default:  // PRCR_MODE_LPA: p + rank in sequence + 1
+                        pos = double(p + (j - t0s) + 1);
+                        break;
                 }
-                if (a.slot_out) a.slot_out[j] = int32_t(slot > INT_MAX ? INT_MAX : slot);
+                // the angle reduction needs |position| < 2^31, and a position
+                // must be the correctly rounded exact value: else the token's
+                // rows are skipped
+                if (e || !pos_in_range(pos)) {
+                    err |= PRCR_ST_POS_RANGE;
+                    s_skip[t] = 1;
+                }
             }
+            s_pf[t][ax] = fixed_32_32(pos);
+            if (blockIdx.y == 0 && a.pos_out) a.pos_out[3 * int64_t(j) + ax] = pos;
         }
     }
     if (err && blockIdx.y == 0) atomicOr(a.status, err);
     __syncthreads();
 
-    // 3. cos/sin of the tile, then 4. the rows (as in the rebind kernel)
-    const int D = rb.head_dim;
-    const int P = D >> 1;
+    // D. cos/sin of the tile
     float* cos_s = smem;
     float* sin_s = smem + T * P;
-    for (int q = threadIdx.x; q < T * P; q += blockDim.x) {
+    for (int q = tid; q < T * P; q += bd) {
         const int t = q / P;
         const int i = q - t * P;
         float c = 1.0f, s = 0.0f;
         if (tok0 + t < tok1) {
             const int ax = pair_axis(i, rb.layout, rb.sec_t, rb.sec_h, rb.sec_w);
-            sincos_turns(s_pos[3 * t + ax], rb.turn_freq[i], &s, &c);
+            sincos_fixed(s_pf[t][ax], rb.turn_freq[i], &s, &c);
         }
         cos_s[q] = c;
         sin_s[q] = s;
     }
     __syncthreads();
 
-    const int t = threadIdx.x / lanes;
-    const int lane = threadIdx.x - t * lanes;
-    if (t >= T || tok0 + t >= tok1) return;
-    const int64_t dst = s_dst[t];
-    if (dst < 0) return;
-    const int64_t src = s_src[t];
-    const int vph = D >> 4;
-    const int h = lane / vph;
-    const int v = lane - h * vph;
-    const int64_t off = int64_t(h) * D + v * 8;
+    // E. the rows: rotate and store the layers in registers, stream the rest
+    if (!my_tok) return;
+    const int64_t dst = s_dst[my_t];
+    if (dst < 0 || s_skip[my_t]) return;
+    const int v = lane % vph;
     float c[8], s[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
-        c[e] = cos_s[t * P + v * 8 + e];
-        s[e] = sin_s[t * P + v * 8 + e];
+        c[e] = cos_s[my_t * P + v * 8 + e];
+        s[e] = sin_s[my_t * P + v * 8 + e];
     }
-    const int l0 = blockIdx.y * rb.layers_per_cta;
-    const int l1 = min(l0 + rb.layers_per_cta, rb.n_layers);
-    const int64_t sls = rb.store_layer_stride;
-    const int64_t cls = rb.cache_layer_stride;
-    stream_layers(rb.store_k + src + int64_t(l0) * sls + off, rb.store_v + src + int64_t(l0) * sls + off,
-                  rb.cache_k + dst + int64_t(l0) * cls + off, rb.cache_v + dst + int64_t(l0) * cls + off,
-                  sls, cls, P, l1 - l0, c, s);
+    uint16_t* ck = rb.cache_k + dst + int64_t(l0) * cls + off;
+    uint16_t* cv = rb.cache_v + dst + int64_t(l0) * cls + off;
+    uint4 o0, o1;
+    rotate_vec(k0a, k1a, c, s, o0, o1);
+    st_row(ck, o0);
+    st_row(ck + P, o1);
+    st_row(cv, v0a);
+    st_row(cv + P, v1a);
+    if (l0 + 1 < l1) {
+        rotate_vec(k0b, k1b, c, s, o0, o1);
+        st_row(ck + cls, o0);
+        st_row(ck + cls + P, o1);
+        st_row(cv + cls, v0b);
+        st_row(cv + cls + P, v1b);
+    }
+    if (l0 + 2 < l1) {
+        const int64_t src = int64_t(my_b) * a.store_seq_stride + int64_t(my_m) * a.store_token_stride;
+        stream_layers(rb.store_k + src + int64_t(l0 + 2) * sls + off,
+                      rb.store_v + src + int64_t(l0 + 2) * sls + off, ck + 2 * cls, cv + 2 * cls, sls,
+                      cls, P, l1 - l0 - 2, c, s);
+    }
 }
 
 }  // namespace

@@ -45,11 +45,21 @@ inline void fill_turn_freq(const prcr_rope_cfg* cfg, uint64_t* out) {
 // half of the 128-bit product's high word, read as signed) are the angle in
 // [-pi, pi) to 2^-32 of a turn. Needs |pos| < 2^31. Only the final sin/cos
 // runs in float32 (CUDA's sincosf).
-__device__ __forceinline__ void sincos_turns(double pos, uint64_t turn_freq, float* s, float* c) {
-    const long long pf = __double2ll_rn(pos * 4294967296.0);
+// The position in signed 32.32 fixed point (round to nearest).
+__device__ __forceinline__ long long fixed_32_32(double pos) {
+    return __double2ll_rn(pos * 4294967296.0);
+}
+
+// sin and cos from a 32.32 fixed-point position (integer arithmetic up to
+// the final float32 sincosf).
+__device__ __forceinline__ void sincos_fixed(long long pf, uint64_t turn_freq, float* s, float* c) {
     const long long hi = __mul64hi(pf, static_cast<long long>(turn_freq));
     const int frac = static_cast<int>(static_cast<unsigned int>(static_cast<unsigned long long>(hi)));
     sincosf(static_cast<float>(frac) * 1.46291807926715968e-09f, s, c);  // 2 pi / 2^32
+}
+
+__device__ __forceinline__ void sincos_turns(double pos, uint64_t turn_freq, float* s, float* c) {
+    sincos_fixed(fixed_32_32(pos), turn_freq, s, c);
 }
 #endif
 
