@@ -265,6 +265,7 @@ int rebind_setup(const prcr_rope_cfg* cfg, const prcr_store_desc* store,
     smem = size_t(2) * T * P * sizeof(float);
     a.lanes = lanes;
     a.tok_per_cta = T;
+    if (kernel == kFused) smem += fused_stage_bytes(block);
 
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return PRCR_ECUDA;

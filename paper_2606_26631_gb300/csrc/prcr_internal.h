@@ -313,6 +313,9 @@ constexpr int kFusedMaxSeqs = 64;
 cudaError_t launch_fused(const FusedArgs& a, dim3 grid, int block, size_t smem,
                          cudaStream_t stream);
 cudaError_t fused_blocks_per_sm(int block, size_t smem, int* out);
+// dynamic shared memory the fused kernel adds to the cos/sin rows: the rows of
+// two layers staged per thread
+size_t fused_stage_bytes(int block);
 cudaError_t launch_plan(const PlanArgs& a, cudaStream_t stream);
 cudaError_t launch_rebind(const RebindArgs& a, dim3 grid, int block, size_t smem,
                           cudaStream_t stream);
