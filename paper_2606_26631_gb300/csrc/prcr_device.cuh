@@ -149,28 +149,26 @@ __device__ __forceinline__ uint64_t pcr_denominator(int64_t K, int64_t span, boo
 __device__ __forceinline__ double pcr_position(int64_t p, int32_t L, int64_t K, int32_t c,
                                                int32_t lo, int32_t hi, bool center,
                                                uint32_t& err) {
+    // The numerator and denominator are selected, not branched on, so that
+    // the lanes of a warp (whose axes may be degenerate or not) share one
+    // float64 division.
     const int64_t span = int64_t(hi) - int64_t(lo);
     const int64_t pl = p - L;
+    const bool deg = span <= 0;  // degenerate axis: u = 0, or u = 1/2 with the centre reading
     const uint64_t Q = pcr_denominator(K, span, center);
-    if (span > 0) {
-        if (exact_ok(pl, L, Q)) {
-            const int64_t tail = int64_t(L + 1) * (span + (K - 1) * (int64_t(c) - lo));
-            return double(pl * int64_t(Q) + tail) / double(Q);
-        }
-        err |= PRCR_ST_POS_RANGE;
-        const double u = double(int64_t(c) - lo) / double(span);
-        return double(pl) + double(L + 1) * (1.0 + double(K - 1) * u) / double(K + 1);
-    }
-    // degenerate axis: u = 0, or u = 1/2 with the centre reading
-    const int64_t tail = center ? int64_t(L + 1) * (K + 1) : int64_t(L + 1);
-    if (exact_ok(pl, L, Q)) return double(pl * int64_t(Q) + tail) / double(Q);
+    const int64_t tail = deg ? (center ? int64_t(L + 1) * (K + 1) : int64_t(L + 1))
+                             : int64_t(L + 1) * (span + (K - 1) * (int64_t(c) - lo));
+    if (exact_ok(pl, L, Q)) return exact_f64(pl * int64_t(Q) + tail) / exact_f64(int64_t(Q));
     err |= PRCR_ST_POS_RANGE;
-    return double(pl) + double(tail) / double(Q);
+    if (deg) return double(pl) + double(tail) / double(Q);
+    const double u = double(int64_t(c) - lo) / double(span);
+    return double(pl) + double(L + 1) * (1.0 + double(K - 1) * u) / double(K + 1);
 }
 
 // p + num / (K + 1), exact while representable (UIR).
 __device__ __forceinline__ double uir_position(int64_t p, int64_t num, int64_t K, uint32_t& err) {
-    if (exact_ok(p, 0, uint64_t(K + 1))) return double(p * (K + 1) + num) / double(K + 1);
+    if (exact_ok(p, 0, uint64_t(K + 1)))
+        return exact_f64(p * (K + 1) + num) / exact_f64(K + 1);
     err |= PRCR_ST_POS_RANGE;
     return double(p) + double(num) / double(K + 1);
 }

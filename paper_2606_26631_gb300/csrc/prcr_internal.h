@@ -45,9 +45,45 @@ inline void fill_turn_freq(const prcr_rope_cfg* cfg, uint64_t* out) {
 // half of the 128-bit product's high word, read as signed) are the angle in
 // [-pi, pi) to 2^-32 of a turn. Needs |pos| < 2^31. Only the final sin/cos
 // runs in float32 (CUDA's sincosf).
-// The position in signed 32.32 fixed point (round to nearest).
+// The position in signed 32.32 fixed point, rounded to nearest (ties to
+// even), formed from the float64 bits with integer instructions only (GB300's
+// float64 pipe is narrow): equal to llrint(pos * 2^32) for |pos| < 2^31, and
+// to -2^63 for pos = -2^31 (+2^31 saturates to 2^63 - 1). A larger magnitude,
+// infinity or NaN gives 0: such positions are reported and their rows
+// skipped wherever they can arise.
 __device__ __forceinline__ long long fixed_32_32(double pos) {
-    return __double2ll_rn(pos * 4294967296.0);
+    const unsigned long long bits = static_cast<unsigned long long>(__double_as_longlong(pos));
+    const int e = int((bits >> 52) & 0x7ff);  // pos * 2^32 = m * 2^(e - 1043)
+    if (e == 0 || e > 1054) return 0;         // zero or subnormal (|pos| < 2^-1022), or |pos| > 2^31
+    const unsigned long long m = (bits & 0xfffffffffffffull) | (1ull << 52);
+    const int sh = e - 1043;
+    unsigned long long r;
+    if (sh >= 0) {
+        r = m << sh;  // < 2^64 (sh <= 11)
+    } else if (-sh > 54) {
+        r = 0;  // below half a unit
+    } else {
+        const int s = -sh;
+        r = m >> s;
+        const unsigned long long rem = m & ((1ull << s) - 1), half = 1ull << (s - 1);
+        if (rem > half || (rem == half && (r & 1))) ++r;
+    }
+    if (bits >> 63) return static_cast<long long>(0ull - r);
+    return r > 0x7fffffffffffffffull ? 0x7fffffffffffffffll : static_cast<long long>(r);
+}
+
+// Exact float64 of an integer of magnitude below 2^53, from integer
+// instructions only.
+__device__ __forceinline__ double exact_f64(long long x) {
+    if (x == 0) return 0.0;
+    const unsigned long long u = x < 0 ? 0ull - static_cast<unsigned long long>(x)
+                                       : static_cast<unsigned long long>(x);
+    const int sh = __clzll(static_cast<long long>(u)) - 11;  // leading one to bit 52
+    const unsigned long long m = u << sh;
+    const unsigned long long bits = (static_cast<unsigned long long>(x < 0) << 63) |
+                                    (static_cast<unsigned long long>(1075 - sh) << 52) |
+                                    (m & 0xfffffffffffffull);
+    return __longlong_as_double(static_cast<long long>(bits));
 }
 
 // sin and cos from a 32.32 fixed-point position (integer arithmetic up to
