@@ -1,8 +1,9 @@
 """Benchmark of the PRCR revisit path (rebind + inject) on GB300.
 
-One step = one call of the whole path over one batch: the plan kernel
-(positions, slots) and the fused gather / M-RoPE rebind / inject kernel, for
-every selected token x layer x KV head of every sequence in the batch.
+One step = one call of the public entry point prcr_rebind_inject over one
+batch: the plan kernel (positions, slots) and the fused gather / M-RoPE
+rebind / inject kernel (one kernel for small batches), for every selected
+token x layer x KV head of every sequence in the batch.
 
 Default workload: the largest one (16-frame 16x32x32 video per sequence,
 4096 revisited tokens per sequence in 3 revisits, batch 32, 36 layers, 8 KV
@@ -44,9 +45,13 @@ SPEC_HBM_GBS = 8000.0
 # workload, from an ncu capture; valid only for the kernel source it was
 # measured on (its sha256 prefix), reported as null otherwise.
 TRAFFIC = {
-    # profiles/rebind_kernel_stress_dram.md: 19,309,795,840 B read + 19,268,509,184 B written
+    # 19,309,795,840 B read + 19,268,509,184 B written
     ("stress", "36f2c98b3efb3176"): 38578305024,
 }
+
+# the Table 3 shapes (Qwen3-VL-8B dimensions, a 768-token image, K = 32 and
+# K = 128), timed after the main workload
+PAPER_SHAPES = ("paper-8b-k32", "paper-8b-k128")
 
 
 def _sha(*paths):
@@ -90,6 +95,8 @@ def parse():
     ap.add_argument("--flush", choices=["auto", "on", "off"], default="auto",
                     help="write a buffer of twice the L2 size before each timed step "
                          "(auto: when a step moves less than 4x the L2 size)")
+    ap.add_argument("--no-paper-shape", action="store_true",
+                    help="skip the Table 3 shape latencies of the revisit path")
     return ap.parse_args()
 
 
@@ -340,6 +347,94 @@ def run_reference(args):
 # ----------------------------------------------------------------------------
 # GPU arm
 # ----------------------------------------------------------------------------
+def selection_manifest(wl, seed: int):
+    """The JSON manifest of the revisits this rank's batch selects (drawn on
+    the host by the workload generator), and whether it equals the committed
+    copy under workloads/manifests/."""
+    from workloads import manifest as MF
+    text = MF.dumps(MF.manifest(wl, seed))
+    path = MF.path_for(wl.name, seed)
+    committed = os.path.exists(path) and open(path).read() == text
+    return dict(path=os.path.relpath(path, ROOT), sha256=MF.sha256_of(text),
+                matches_committed=committed, n_revisits=text.count('"K"'),
+                total_k=MF.manifest(wl, seed)["total_k"])
+
+
+def paper_shape_latency(dev, local, cold_steps: int = 100, inner: int = 20, replays: int = 10):
+    """The revisit of Table 3's shapes (Qwen3-VL-8B dimensions, a 768-token
+    image, one rectangle of K = 32 or 128 tokens, contiguous cache) through
+    the public call prcr_rebind_inject: every output first compared with the
+    oracle; then `cold` = stream launches each after a write of twice the L2
+    size (the raw rows, plan inputs and cache lines not in L2), and `warm` =
+    CUDA-graph replays of `inner` calls back to back (launch overhead gone,
+    working set in L2). Microseconds per call."""
+    import torch
+    sys.path.insert(0, os.path.join(ROOT, "tests"))
+    import parity_util as pu
+    from workloads import get, make_batch
+    out = {}
+    stream = torch.cuda.current_stream()
+    for name in PAPER_SHAPES:
+        batch = make_batch(get(name), device=dev)
+        rv = pu.make_revisit(batch)
+        rv.run()
+        torch.cuda.synchronize()
+        if rv.status_value() != 0:
+            raise RuntimeError(f"{name}: device status {rv.status_value():#x}")
+        err = pu.full_check(batch, rv)
+        launched = kernel_launches(rv.run)
+        nbytes = batch.algorithmic_bytes()
+        flush = L2Flush(dev, "on", nbytes)
+        for _ in range(3):
+            flush()
+            rv.run()
+        torch.cuda.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(cold_steps)]
+        with Clocks(local) as clk:
+            for e0, e1 in ev:
+                flush()
+                e0.record(stream)
+                rv.run()
+                e1.record(stream)
+            torch.cuda.synchronize()
+            cold = [1e3 * e0.elapsed_time(e1) for e0, e1 in ev]
+            g = torch.cuda.CUDAGraph()
+            side = torch.cuda.Stream()
+            side.wait_stream(stream)
+            with torch.cuda.stream(side):
+                rv.run()
+            stream.wait_stream(side)
+            torch.cuda.synchronize()
+            with torch.cuda.graph(g):
+                for _ in range(inner):
+                    rv.run()
+            for _ in range(3):
+                g.replay()
+            torch.cuda.synchronize()
+            evg = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(replays)]
+            for e0, e1 in evg:
+                e0.record(stream)
+                g.replay()
+                e1.record(stream)
+            torch.cuda.synchronize()
+            warm = [1e3 * e0.elapsed_time(e1) / inner for e0, e1 in evg]
+        out[name] = dict(
+            tokens=batch.total_k, bytes=nbytes, kernels=launched or None,
+            cold_us_median=statistics.median(cold), cold_us_mean=statistics.mean(cold),
+            warm_us_median=statistics.median(warm), warm_us_mean=statistics.mean(warm),
+            cold_gbs=nbytes / statistics.median(cold) / 1e3,
+            warm_gbs=nbytes / statistics.median(warm) / 1e3,
+            cold_steps=cold_steps, warm_calls=inner * replays,
+            l2=flush.describe(nbytes) + " (cold); no flush, graph replays (warm)",
+            parity=dict(k_max_err=err["max_err"], positions_slots_v="bit-exact"),
+            clocks=clk.summary())
+        del rv, batch, g
+        torch.cuda.empty_cache()
+    return out
+
+
 def run_gpu(args):
     import torch
     world, rank, local = dist_env()
@@ -383,20 +478,17 @@ def run_gpu(args):
 
     stream = torch.cuda.current_stream()
     # what one public call launches: one fused kernel for small batches, or
-    # the plan kernel then the rebind + inject kernel (timed one by one)
+    # the plan kernel then the rebind + inject kernel
     launched = kernel_launches(rv.run)
     split = launched == ["plan_kernel", "rebind_kernel"] or not launched
     per_step = len(launched) if launched else 2
     for _ in range(args.warmup):
-        if split:
-            rv.run_plan()
-            rv.run_apply()
-        else:
-            rv.run()
+        rv.run()
     torch.cuda.synchronize()
     flush = L2Flush(dev, "off" if args.graph else args.flush, nbytes)
 
     K = args.steps
+    apply_ms = plan_ms = None
     if args.graph:
         # K steps as K / inner replays of a graph holding `inner` steps
         inner = max(1, args.graph_inner)
@@ -426,34 +518,40 @@ def run_gpu(args):
             torch.cuda.synchronize()
         barrier(world)
         step_ms = [e0.elapsed_time(e2) / inner for e0, e2 in ev for _ in range(inner)]
-        apply_ms = None
-        plan_ms = None
     else:
-        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
-               torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+        # the headline: the public call, events around each step
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(K)]
         barrier(world)
         torch.cuda.synchronize()
         with Clocks(local) as clk:
-            for e0, e1, e2 in ev:
+            for e0, e2 in ev:
                 flush()
                 e0.record(stream)
-                if split:
-                    rv.run_plan()
-                    e1.record(stream)
-                    rv.run_apply()
-                else:
-                    rv.run()
-                    e1.record(stream)
+                rv.run()
                 e2.record(stream)
             torch.cuda.synchronize()
         barrier(world)
-        step_ms = [e0.elapsed_time(e2) for e0, _, e2 in ev]
+        step_ms = [e0.elapsed_time(e2) for e0, e2 in ev]
+        # per-kernel durations for the roofline: the same work through the
+        # call's two halves (prcr_plan, prcr_rebind_apply) with an event
+        # between them, after the headline loop
         if split:
-            apply_ms = [e1.elapsed_time(e2) for _, e1, e2 in ev]
-            plan_ms = [e0.elapsed_time(e1) for e0, e1, _ in ev]
+            R = min(K, 20)
+            evk = [tuple(torch.cuda.Event(enable_timing=True) for _ in range(3)) for _ in range(R)]
+            torch.cuda.synchronize()
+            for e0, e1, e2 in evk:
+                flush()
+                e0.record(stream)
+                rv.run_plan()
+                e1.record(stream)
+                rv.run_apply()
+                e2.record(stream)
+            torch.cuda.synchronize()
+            apply_ms = [e1.elapsed_time(e2) for _, e1, e2 in evk]
+            plan_ms = [e0.elapsed_time(e1) for e0, e1, _ in evk]
         else:
             apply_ms = step_ms
-            plan_ms = None
     total_s = sum(step_ms) / 1e3
     total_s = max_over_ranks(total_s, world, dev)
     value = nbytes * world * K / total_s / 1e9
@@ -478,6 +576,10 @@ def run_gpu(args):
     else:  # graph replay: only whole steps are timed
         apply_avg_s = statistics.mean(step_ms) / 1e3
         kernel = " + ".join(launched or ["plan_kernel", "rebind_kernel"]) + " (graph step)"
+    manifest = selection_manifest(wl, rank)
+    shapes = None
+    if rank == 0 and not args.no_paper_shape:
+        shapes = paper_shape_latency(dev, local)
     achieved = nbytes / apply_avg_s / 1e9
     src_sha = _sha(*(os.path.join(ROOT, "paper_2606_26631_gb300", "csrc", f)
                      for f in ("prcr_rebind.cu", "prcr_device.cuh", "prcr_internal.h")))
@@ -506,11 +608,15 @@ def run_gpu(args):
             token_layers_per_s=batch.total_k * wl.n_layers * world * K / total_s,
             plan_us_avg=1e3 * statistics.mean(plan_ms) if plan_ms else None,
             timing="cuda graph, %d steps per replay" % args.graph_inner if args.graph
-            else "stream launches, events around each step and kernel",
-            roofline=roof, cpu_baseline=cpu,
+            else "stream launches of prcr_rebind_inject, events around each step; the "
+                 "roofline kernel timed over %d further steps through prcr_plan + "
+                 "prcr_rebind_apply" % (min(K, 20) if split else 0),
+            roofline=roof, cpu_baseline=cpu, selection_manifest=manifest,
+            paper_shape=shapes,
             e2e=dict(value=e2e_value, unit=UNIT, h2d_bytes_per_step=rv.h2d_bytes(),
                      d2h_bytes_per_step=rv.d2h_bytes(), steps=args.e2e_steps),
-            gpu_launches=per_step * K, kernels_per_step=launched or None,
+            gpu_launches=per_step * K,
+            kernels_per_step=launched or None,
             launches_counted_by="torch.profiler (CUPTI), one call" if launched
             else "two entry points per step, one kernel each",
             clocks=clk.summary(), parity=check)

@@ -8,8 +8,8 @@ CUDA graph those dependencies become graph edges. A replay of the captured
 step must give exactly the results of the same calls made eagerly: the same
 selection, the same cache rows and the same decode output, bit for bit, for
 several trigger queries written into the captured input buffer between
-replays. The stages themselves are checked against the oracle by the
-selection, rebind and decode parity tests."""
+replays. The whole chain is also compared with the oracle's, stage by stage
+and at the final decode output (test_pipeline_matches_oracle_chain)."""
 import pytest
 import torch
 
@@ -90,3 +90,109 @@ def test_pipeline_graph_replay_matches_eager(name):
             assert rv.status_value() == 0 and int(dstat.item()) == 0
             for a, b in zip(snapshot(), eager[i]):
                 assert torch.equal(a, b), (rep, i)
+
+
+def _check_selection(score_b, ref, sel, k, M):
+    """The GPU's set against the oracle's relevance (the selection tests'
+    rule): relevance within 1e-4 relative; the set is the exact top-k of the
+    kernel's own relevance; a valid top-k of the oracle's up to the measured
+    error; the oracle's own set whenever the k-th gap exceeds that error."""
+    import numpy as np
+    from oracle import prcr_oracle as O
+    rel_err = np.abs(score_b - ref) / ref
+    assert rel_err.max() <= 1e-4, rel_err.max()
+    assert len(set(sel.tolist())) == k and np.all(np.diff(sel) > 0)
+    order = np.lexsort((np.arange(M), -score_b.astype(np.float64)))
+    assert np.array_equal(sel, np.sort(order[:k]))
+    tol = 2 * np.abs(score_b - ref).max() + 1e-12
+    chosen = np.zeros(M, dtype=bool)
+    chosen[sel] = True
+    if k < M:
+        assert ref[chosen].min() >= ref[~chosen].max() - tol
+        srt = np.sort(ref)[::-1]
+        if srt[k - 1] - srt[k] > tol:
+            assert np.array_equal(sel, O.ads_select(ref, k))
+
+
+@pytest.mark.parametrize("name", ["paper-8b-k32", "qwen25vl-7b"])
+def test_pipeline_matches_oracle_chain(name):
+    """One revisit through the three entry points, each stage and the final
+    decode output compared with the oracle's chain ads_relevance -> ads_select
+    -> rebind_inject -> decode_attention on the same inputs (the GPU's
+    selected set, once shown to be a valid top-k of the oracle's relevance,
+    is the one the oracle's rebind receives)."""
+    import dataclasses
+    import numpy as np
+    import paper_2606_26631_gb300 as prcr
+    import parity_util as pu
+    from oracle import prcr_oracle as O
+
+    wl = get(name)
+    batch = make_batch(wl, device=DEV, context="random")
+    B, nL, M, H, D = wl.n_seqs, wl.n_layers, wl.n_tokens, wl.n_kv_heads, wl.head_dim
+    sro_h, rto_h = batch.seq_rev_off.cpu().numpy(), batch.rev_tok_off.cpu().numpy()
+    k = int(min(rto_h[sro_h[b + 1]] - rto_h[sro_h[b]] for b in range(B)))
+    Hq = {"paper-8b-k32": 32, "qwen25vl-7b": 28}[name]
+    layer = nL - 1
+    cfg = prcr.rope_cfg(nL, H, D, wl.sections, wl.theta)
+    sd = prcr.store_desc(batch.store_k, batch.store_v, batch.coords)
+    ctx_k, ctx_v = batch.cache_k.clone(), batch.cache_v.clone()
+    g = torch.Generator(device=DEV).manual_seed(31)
+    q_sel = (2.0 * torch.randn((B, Hq, D), device=DEV, generator=g)).to(torch.bfloat16)
+    q_dec = torch.randn((B, nL, Hq, D), device=DEV, generator=g).to(torch.bfloat16)
+
+    # 1. selection
+    idx = torch.empty(B * k, dtype=torch.int32, device=DEV)
+    sro = torch.empty(B + 1, dtype=torch.int32, device=DEV)
+    rto = torch.empty(B + 1, dtype=torch.int32, device=DEV)
+    score = torch.empty((B, M), dtype=torch.float32, device=DEV)
+    ws_sel = torch.empty(prcr.select_workspace_size(B, Hq, M), dtype=torch.uint8, device=DEV)
+    prcr.select_topk(cfg, sd, layer, q_sel, batch.p_txt, k, idx, sro, rto, ws_sel, score)
+    # 2. rebind + inject of the selected set
+    sel = dataclasses.replace(batch, idx=idx, seq_rev_off=sro, rev_tok_off=rto)
+    rv = pu.make_revisit(sel)
+    rv.run()
+    # 3. first decode step over the grown cache
+    max_len = int(batch.cache_len_in.max().item()) + k
+    out = torch.empty(q_dec.shape, dtype=torch.float32, device=DEV)
+    dstat = torch.zeros(1, dtype=torch.int32, device=DEV)
+    ws_dec = torch.empty(max(prcr.decode_workspace_size(cfg, B, Hq, max_len), 16), dtype=torch.uint8,
+                         device=DEV)
+    prcr.decode_attention(cfg, rv.cache, q_dec, rv.next_pos, rv.cache_len_out, max_len, out, dstat,
+                          ws_dec)
+    torch.cuda.synchronize()
+    assert rv.status_value() == 0 and int(dstat.item()) == 0
+
+    # oracle chain, stage by stage
+    sel_h = idx.view(B, k).cpu().numpy()
+    assert np.array_equal(sro.cpu().numpy(), np.arange(B + 1))
+    assert np.array_equal(rto.cpu().numpy(), k * np.arange(B + 1))
+    qv = O.bf16_bits_to_f64(q_sel.view(torch.int16).cpu().numpy())
+    kb = batch.store_k[:, layer].contiguous().view(torch.int16).cpu().numpy()
+    crd = batch.coords.cpu().numpy()
+    p_h = batch.p_txt.cpu().numpy()
+    sc = score.cpu().numpy()
+    for b in range(B):
+        ref = O.ads_relevance(qv[b], int(p_h[b]), kb[b], crd[b], D, wl.sections, wl.theta)
+        _check_selection(sc[b], ref, sel_h[b], k, M)
+    pl = pu.oracle_plan(sel)
+    pu.check_plan(rv, pl)
+    pu.check_rows(sel, rv, pl, range(B * k), range(nL))
+    got = out.cpu().numpy()
+    qd = O.bf16_bits_to_f64(q_dec.view(torch.int16).cpu().numpy())
+    from test_decode_gpu import _cache_rows
+    for b in range(B):
+        n_all = int(pl["cache_len_out"][b])
+        K, V = _cache_rows(ctx_k, ctx_v, batch.block_table, b, n_all, batch.paged)
+        toks = np.arange(b * k, (b + 1) * k)
+        ids = torch.as_tensor(sel_h[b].astype(np.int64), device=DEV)
+        k_raw = pu.bits(batch.store_k[b][:, ids].transpose(0, 1))
+        v_raw = pu.bits(batch.store_v[b][:, ids].transpose(0, 1))
+        K[pl["slot"][toks]] = O.f64_to_bf16_rne(O.rebind_keys(k_raw, pl["pos"][toks], D, wl.sections,
+                                                              wl.theta))
+        V[pl["slot"][toks]] = O.bf16_bits_to_f64(v_raw)
+        for l in range(nL):
+            ref = O.decode_attention(qd[b, l], int(pl["next_pos"][b]), K[:, l], V[:, l], D,
+                                     wl.sections, wl.theta)
+            err = np.abs(got[b, l] - ref).max() / np.abs(V[:, l]).max()
+            assert err <= 1e-3, (name, b, l, err)

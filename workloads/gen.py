@@ -119,16 +119,21 @@ def _disjoint_rects(rng, rows, cols, areas) -> List[Tuple[int, int, int, int]]:
     return rects
 
 
-def selections(wl: Workload, rng) -> List[List[np.ndarray]]:
+def selections(wl: Workload, rng, rects_out: Optional[list] = None) -> List[List[np.ndarray]]:
     """Per sequence, the list of revisited index sets (Eq. 3), each in the
-    order a caller would hand them over (rectangle by rectangle, row-major)."""
+    order a caller would hand them over (rectangle by rectangle, row-major).
+    If ``rects_out`` is a list, it receives per sequence, per revisit, the
+    rectangles as drawn: (grid, first frame, frames, first row, rows, first
+    column, columns) each, or an empty list for scattered tokens."""
     layout = grid_layout(wl)
     out = []
     for _ in range(wl.n_seqs):
         revs = []
+        drawn = []
         if wl.selection == "rect4x4":
             r0 = int(rng.integers(0, 5)); c0 = int(rng.integers(0, 5))
             revs.append(_rect_ids(layout, 0, 0, 1, r0, 4, c0, 4))
+            drawn.append([(0, 0, 1, r0, 4, c0, 4)])
         elif wl.selection in ("rects3_256", "rectset512"):
             _, _, rows, cols, _ = layout[0]
             if wl.selection == "rects3_256":
@@ -138,6 +143,7 @@ def selections(wl: Workload, rng) -> List[List[np.ndarray]]:
                 areas = [512 // n] * n
             rects = _disjoint_rects(rng, rows, cols, areas)
             revs.append(np.concatenate([_rect_ids(layout, 0, 0, 1, *rc) for rc in rects]))
+            drawn.append([(0, 0, 1) + tuple(rc) for rc in rects])
         elif wl.selection == "rev4_256_1024":
             for _ in range(4):
                 g = int(rng.integers(0, len(layout)))
@@ -147,28 +153,35 @@ def selections(wl: Workload, rng) -> List[List[np.ndarray]]:
                 nc = min(cols, max(1, int(round(area / nr))))
                 r0 = int(rng.integers(0, rows - nr + 1)); c0 = int(rng.integers(0, cols - nc + 1))
                 revs.append(_rect_ids(layout, g, 0, 1, r0, nr, c0, nc))
+                drawn.append([(g, 0, 1, r0, nr, c0, nc)])
         elif wl.selection == "video_stress":
             _, frames, rows, cols, _ = layout[0]
             fr = rng.choice(frames, size=2, replace=False)
             for f in fr:
                 revs.append(_rect_ids(layout, 0, int(f), 1, 0, rows, 0, cols))
+                drawn.append([(0, int(f), 1, 0, rows, 0, cols)])
             f0 = int(rng.integers(0, frames - 8 + 1))
             r0 = int(rng.integers(0, rows - 16 + 1)); c0 = int(rng.integers(0, cols - 16 + 1))
             revs.append(_rect_ids(layout, 0, f0, 8, r0, 16, c0, 16))
+            drawn.append([(0, f0, 8, r0, 16, c0, 16)])
         elif wl.selection in ("rect_k32", "rect_k128"):
             nr, nc = (4, 8) if wl.selection == "rect_k32" else (8, 16)
             _, _, rows, cols, _ = layout[0]
             r0 = int(rng.integers(0, rows - nr + 1)); c0 = int(rng.integers(0, cols - nc + 1))
             revs.append(_rect_ids(layout, 0, 0, 1, r0, nr, c0, nc))
+            drawn.append([(0, 0, 1, r0, nr, c0, nc)])
         elif wl.selection == "random":
             # extra = (min revisits, max revisits, min K, max K): distinct random tokens
             rmin, rmax, kmin, kmax = wl.extra
             for _ in range(int(rng.integers(rmin, rmax + 1))):
                 k = min(int(rng.integers(kmin, kmax + 1)), wl.n_tokens)
                 revs.append(rng.choice(wl.n_tokens, size=k, replace=False).astype(np.int32))
+                drawn.append([])
         else:
             raise ValueError(wl.selection)
         out.append(revs)
+        if rects_out is not None:
+            rects_out.append(drawn)
     return out
 
 
