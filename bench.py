@@ -45,8 +45,9 @@ SPEC_HBM_GBS = 8000.0
 # workload, from an ncu capture; valid only for the kernel source it was
 # measured on (its sha256 prefix), reported as null otherwise.
 TRAFFIC = {
-    # 19,309,795,840 B read + 19,268,509,184 B written
-    ("stress", "36f2c98b3efb3176"): 38578305024,
+    # captured on the stress shape cut to 2 sequences (8,192 tokens: 1,194,226,432 B
+    # read + 1,150,181,376 B written) and scaled by the 16x more tokens of a full launch
+    ("stress", "5e0eac633b30788d"): 37510524928,
 }
 
 # the Table 3 shapes (Qwen3-VL-8B dimensions, a 768-token image, K = 32 and
@@ -77,7 +78,8 @@ def parse():
                          "decode: the first decode step over the active cache; select: the "
                          "attention-driven selection of the revisited set; pipeline: select, "
                          "rebind+inject and the first decode step of one revisit, end to end")
-    ap.add_argument("--seqs", type=int, default=0, help="capture/decode: sequences (0 = workload's)")
+    ap.add_argument("--seqs", type=int, default=0,
+                    help="sequences of the workload's batch (0 = the workload's own count)")
     ap.add_argument("--select-source", choices=["raw", "cache"], default="raw",
                     help="select / pipeline: rank from the raw store (prcr_select_topk) or from "
                          "the position-bound cache (prcr_select_topk_cached)")
@@ -352,12 +354,13 @@ def selection_manifest(wl, seed: int):
     the host by the workload generator), and whether it equals the committed
     copy under workloads/manifests/."""
     from workloads import manifest as MF
-    text = MF.dumps(MF.manifest(wl, seed))
+    m = MF.manifest(wl, seed)
+    text = MF.dumps(m)
     path = MF.path_for(wl.name, seed)
     committed = os.path.exists(path) and open(path).read() == text
-    return dict(path=os.path.relpath(path, ROOT), sha256=MF.sha256_of(text),
-                matches_committed=committed, n_revisits=text.count('"K"'),
-                total_k=MF.manifest(wl, seed)["total_k"])
+    return dict(path=os.path.relpath(path, ROOT) if committed else None,
+                sha256=MF.sha256_of(text), matches_committed=committed,
+                n_revisits=m["n_revisits"], total_k=m["total_k"])
 
 
 def paper_shape_latency(dev, local, cold_steps: int = 100, inner: int = 20, replays: int = 10):
@@ -455,6 +458,8 @@ def run_gpu(args):
     from workloads import get, make_batch
 
     wl = get(args.workload)
+    if args.seqs:
+        wl = dataclasses.replace(wl, n_seqs=args.seqs)
     batch = make_batch(wl, device=dev, seed=rank)
     rv = pu.make_revisit(batch)
     nbytes = batch.algorithmic_bytes()
