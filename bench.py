@@ -83,6 +83,9 @@ def parse():
     ap.add_argument("--select-source", choices=["raw", "cache"], default="raw",
                     help="select / pipeline: rank from the raw store (prcr_select_topk) or from "
                          "the position-bound cache (prcr_select_topk_cached)")
+    ap.add_argument("--max-len", type=int, default=8192,
+                    help="decode: the longest sequence (lengths drawn in [1, max-len], the last "
+                         "one at max-len)")
     ap.add_argument("--layers", type=int, default=0,
                     help="select: build the store with this many layers (0 = workload's); "
                          "the selection reads the last one")
@@ -744,7 +747,7 @@ def run_decode_path(args):
     wl = get(args.workload)
     B = args.seqs or wl.n_seqs
     Hq = 4 * wl.n_kv_heads
-    max_len = 8192
+    max_len = args.max_len
     inp = make_decode_inputs(B, wl.n_layers, wl.n_kv_heads, Hq, wl.head_dim, max_len, True,
                              device=dev, seed=1)
     cfg = prcr.rope_cfg(wl.n_layers, wl.n_kv_heads, wl.head_dim, wl.sections, wl.theta)
