@@ -370,8 +370,28 @@ constexpr size_t kDecodeSmem = 46 * 1024;
 // short, with chunks of at least 256 slots (to amortise each CTA's query
 // rotation), a multiple of 32, at most kDecodeMaxChunk, and small enough for
 // the chunk's row offsets to fit beside the rotated queries in shared memory.
-void decode_split(int64_t base_ctas, int64_t max_len, int sms, int64_t q_elems, int* splits,
-                  int* chunk) {
+// A small batch (work for fewer than ~6 waves at 768 slots per chunk) with
+// head_dim 64 or 128 takes the ring kernel instead (*ring = 1): its KV heads
+// are split over CTAs of kDecodeRingWarps warps and the chunk is sized so that
+// the grid is about one wave of kDecodeRingCtasPerSm CTAs per SM, each warp
+// streaming its chunk through a shared-memory ring.
+void decode_split(int64_t base_ctas, int64_t max_len, int sms, int64_t q_elems, int n_kv_heads,
+                  int head_dim, int* splits, int* chunk, int* ring) {
+    const bool small = base_ctas * ((max_len + 767) / 768) < int64_t(sms) * 6;
+    if (small && (head_dim == 64 || head_dim == 128)) {
+        const int64_t units = base_ctas * ((n_kv_heads + kDecodeRingWarps - 1) / kDecodeRingWarps);
+        int64_t want = int64_t(sms) * kDecodeRingCtasPerSm / units;
+        if (want < 1) want = 1;
+        int64_t c = (max_len + want - 1) / want;
+        c = (c + 15) / 16 * 16;
+        if (c > kDecodeMaxChunk) c = kDecodeMaxChunk;
+        *ring = 1;
+        *chunk = int(c);
+        *splits = int((max_len + c - 1) / c);
+        if (*splits < 1) *splits = 1;
+        return;
+    }
+    *ring = 0;
     int64_t want = (int64_t(sms) * 24 + base_ctas - 1) / base_ctas;
     if (want < 1) want = 1;
     int64_t c = (max_len + want - 1) / want;
@@ -379,9 +399,9 @@ void decode_split(int64_t base_ctas, int64_t max_len, int sms, int64_t q_elems, 
     // Below ~768 slots a chunk's prologue and its share of the merge outweigh
     // the better balance when there is work for a few waves anyway (measured:
     // 512 -> 768 slots took the qwen25vl-7b shape from 5032 to 5394 GB/s;
-    // 1184 -> 768 changed qwen3vl-8b by < 1 %). A small batch (one sequence
-    // of ~1k slots) needs the parallelism instead: chunks of 64 slots.
-    const int64_t floor_c = base_ctas * ((max_len + 767) / 768) >= int64_t(sms) * 6 ? 768 : 64;
+    // 1184 -> 768 changed qwen3vl-8b by < 1 %). A small batch at head_dim 256
+    // (the CUDA-core kernel) needs the parallelism instead: chunks of 64 slots.
+    const int64_t floor_c = small ? 64 : 768;
     if (c < floor_c) c = floor_c;
     if (c > kDecodeMaxChunk) c = kDecodeMaxChunk;
     const int64_t cap = (int64_t(kDecodeSmem) - q_elems * int64_t(sizeof(float))) / 8 / 32 * 32;
@@ -589,9 +609,9 @@ size_t prcr_decode_workspace_size(const prcr_rope_cfg* cfg, int32_t n_seqs, int3
     if (check_cfg(cfg) || n_seqs < 1 || max_len < 1 || !decode_shape_ok(cfg, n_q_heads)) return 0;
     int dev = 0, sms = 1;
     if (cudaGetDevice(&dev) == cudaSuccess) sms = sm_count(dev);
-    int splits = 1, chunk = 32;
+    int splits = 1, chunk = 32, ring = 0;
     decode_split(int64_t(n_seqs) * cfg->n_layers, max_len, sms, int64_t(n_q_heads) * cfg->head_dim,
-                 &splits, &chunk);
+                 cfg->n_kv_heads, cfg->head_dim, &splits, &chunk, &ring);
     if (splits == 1) return 0;
     return size_t(n_seqs) * cfg->n_layers * n_q_heads * splits * (cfg->head_dim + 2) * sizeof(float);
 }
@@ -618,7 +638,8 @@ int prcr_decode_attention(const prcr_rope_cfg* cfg, const prcr_cache_desc* cache
     if (cudaGetDevice(&dev) != cudaSuccess) return PRCR_ECUDA;
     DecodeArgs a = {};
     decode_split(int64_t(n_seqs) * cfg->n_layers, max_len, sm_count(dev),
-                 int64_t(n_q_heads) * cfg->head_dim, &a.splits, &a.chunk);
+                 int64_t(n_q_heads) * cfg->head_dim, cfg->n_kv_heads, cfg->head_dim, &a.splits,
+                 &a.chunk, &a.ring);
     if (n_seqs > 65535 || cfg->n_layers > 65535) return PRCR_EINVAL;  // grid z and y
     if (a.splits > 1) {
         const size_t need = size_t(n_seqs) * cfg->n_layers * n_q_heads * a.splits *

@@ -631,6 +631,332 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     if (err) atomicOr(a.status, err);
 }
 
+// Small batches (a grid that would not fill the GPU a few times over): a CTA
+// of kRingWarps warps takes one (sequence, layer, chunk) and up to kRingWarps
+// KV heads, one per warp, and the chunk is sized so that the grid runs as
+// about one wave. Each warp streams its chunk's tiles of 16 slots through a
+// ring of kRingStages stages in shared memory: K and V are both staged by
+// cp.async, kRingStages - 1 tiles ahead of the one being computed, and the
+// first of them are requested before the prologue's barriers (a barrier
+// waits for a thread's plain loads in flight, not for its async copies). The
+// arithmetic is that of decode_mma_kernel (same QK and PV on tensor cores,
+// same online softmax); the key dimensions are permuted per lane group the
+// same way, here with lane group t reading 16-byte chunks t, t + 4, ... of its
+// slot's K row, and chunk c of slot s is stored at c ^ 4 (s & 1) so that
+// those reads are free of bank conflicts.
+constexpr int kRingWarps = kDecodeRingWarps;
+constexpr int kRingStages = 3;
+
+template <int D>
+__global__ void __launch_bounds__(kRingWarps * 32, 2)
+    decode_ring_kernel(const __grid_constant__ DecodeArgs a) {
+    constexpr int KS = D / 16;      // k-steps of QK, m-tiles of PV
+    constexpr int LV = D / 32;      // 16-byte K chunks per lane per slot
+    constexpr int NCH = D / 8;      // 16-byte chunks per row
+    constexpr int PITCH = D + 8;    // bf16 per staged V row (pad: conflict-free ldmatrix)
+    constexpr int KT = 16 * D;      // bf16 per staged K tile
+    constexpr int VT = 16 * PITCH;  // bf16 per staged V tile
+    constexpr int NS = kRingStages;
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    __shared__ __align__(16) float s_cos[kMaxPairs];
+    __shared__ __align__(16) float s_sin[kMaxPairs];
+    __shared__ uint32_t s_mask[kRingWarps][NS];
+    const int P = D / 2;
+    const int g = a.group;
+    const int H = a.n_kv_heads;
+    const int b = blockIdx.z;
+    const int l = blockIdx.y;
+    const int n_hg = (H + kRingWarps - 1) / kRingWarps;
+    const int split = int(blockIdx.x) / n_hg;
+    const int kh0 = (int(blockIdx.x) - split * n_hg) * kRingWarps;
+    const int kh1 = min(H, kh0 + kRingWarps);
+    const int nq = (kh1 - kh0) * g;  // this CTA's query heads
+    float* q_s = reinterpret_cast<float*>(smem_raw);  // [nq][D], rotated and scaled
+    uint16_t* ring = reinterpret_cast<uint16_t*>(smem_raw + size_t(kRingWarps) * g * D * sizeof(float));
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int gid = lane >> 2;
+    const int t = lane & 3;
+    const int kh = kh0 + warp;
+    const bool wact = kh < kh1;
+    const uint16_t* wk = ring + size_t(warp) * NS * (KT + VT);  // NS K stages, then NS V stages
+    const uint32_t wk_s = uint32_t(__cvta_generic_to_shared(wk));
+    const uint32_t wv_s = wk_s + uint32_t(NS * KT * 2);
+    uint32_t err = 0;
+    pdl_allow();
+    {
+        // this CTA's query rows into L2 while the preceding grid drains
+        const char* qrow = reinterpret_cast<const char*>(
+            a.q + ((int64_t(b) * a.n_layers + l) * a.n_q_heads + kh0 * g) * D);
+        for (int o = threadIdx.x * 128; o < nq * D * 2; o += blockDim.x * 128) prefetch_l2(qrow + o);
+    }
+    pdl_wait();
+    const int64_t p = a.q_pos[b];
+    int64_t len = a.seq_len[b];
+    if (len < 0 || len > a.capacity) {
+        err |= PRCR_ST_CAPACITY;
+        len = len < 0 ? 0 : a.capacity;
+    }
+    if (len > int64_t(a.splits) * a.chunk) {  // above the host's max_len: past the split
+        err |= PRCR_ST_CAPACITY;
+        len = int64_t(a.splits) * a.chunk;
+    }
+    // A query position beyond the fixed-point angle reduction (|p| >= 2^31)
+    // is reported and the sequence attends to nothing: its output is zeros.
+    if (p <= -2147483648LL || p >= 2147483648LL) {
+        err |= PRCR_ST_POS_RANGE;
+        len = 0;
+    }
+    const int64_t s_begin = int64_t(split) * a.chunk;
+    const int64_t s_end = min(len, s_begin + a.chunk);
+    const int n_tiles = s_end > s_begin ? int((s_end - s_begin + 15) / 16) : 0;
+    const int64_t lstride = int64_t(l) * a.layer_stride;
+    const uint16_t* kbase = a.cache_k + lstride + int64_t(wact ? kh : kh0) * D;
+    const uint16_t* vbase = a.cache_v + lstride + int64_t(wact ? kh : kh0) * D;
+
+    // block id of this lane's slot (lane & 15) of tile n (paged caches)
+    auto block_id = [&](int n) -> int32_t {
+        const int64_t s = s_begin + 16 * int64_t(n) + (lane & 15);
+        if (a.cache_kind != PRCR_CACHE_PAGED || n >= n_tiles || s >= s_end) return 0;
+        return a.block_table[int64_t(b) * a.bt_stride + s / a.block_size];
+    };
+    // copies of tile n into stage n % NS (one commit group per call, empty
+    // past the last tile or for a warp without a KV head)
+    auto issue = [&](int n, int32_t blk) {
+        if (wact && n < n_tiles) {
+            const int st = n % NS;
+            const int64_t s = s_begin + 16 * int64_t(n) + (lane & 15);
+            int64_t row = -1;
+            if (s < s_end) {
+                if (a.cache_kind == PRCR_CACHE_CONTIGUOUS) {
+                    row = int64_t(b) * a.seq_stride + s * a.slot_stride;
+                } else if (blk < 0 || blk >= a.n_blocks) {
+                    err |= PRCR_ST_NO_BLOCK;
+                } else {
+                    const int64_t lb = s / a.block_size;
+                    row = int64_t(blk) * a.block_stride + (s - lb * a.block_size) * a.slot_stride;
+                }
+            }
+            const uint32_t m = __ballot_sync(kFull, row >= 0) & 0xffffu;
+            if (lane == 0) s_mask[warp][st] = m;
+            const uint32_t ks_ = wk_s + uint32_t(st * KT * 2);
+            const uint32_t vs_ = wv_s + uint32_t(st * VT * 2);
+#pragma unroll
+            for (int i = 0; i < (16 * NCH) / 32; ++i) {
+                const int c = lane + 32 * i;
+                const int slot = c / NCH;
+                const int ch = c - slot * NCH;
+                const int64_t rr = __shfl_sync(kFull, row, slot);
+                const bool ok = rr >= 0;
+                cp_async16(ks_ + uint32_t((slot * D + ((ch ^ ((slot & 1) << 2)) * 8)) * 2),
+                           ok ? kbase + rr + ch * 8 : kbase, ok ? 16 : 0);
+                cp_async16(vs_ + uint32_t((slot * PITCH + ch * 8) * 2),
+                           ok ? vbase + rr + ch * 8 : vbase, ok ? 16 : 0);
+            }
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+
+    // the first NS - 1 tiles are requested now, before the prologue
+    {
+        int32_t blk[NS - 1];
+#pragma unroll
+        for (int i = 0; i < NS - 1; ++i) blk[i] = block_id(i);
+#pragma unroll
+        for (int i = 0; i < NS - 1; ++i) issue(i, blk[i]);
+    }
+    int32_t blk_next = block_id(NS - 1);
+
+    // query heads of this CTA rotated at (p, p, p), scaled by 1/sqrt(D): with
+    // the same position on every axis, pair i turns by p * inv_freq_i
+    // whatever its band, so each pair's cos/sin serves all heads
+    for (int i = threadIdx.x; i < P; i += blockDim.x)
+        sincos_turns(double(p), a.turn_freq[i], &s_sin[i], &s_cos[i]);
+    __syncthreads();
+    const uint16_t* qb = a.q + ((int64_t(b) * a.n_layers + l) * a.n_q_heads + kh0 * g) * D;
+    const bool q16 = (reinterpret_cast<uintptr_t>(a.q) & 15) == 0;
+    for (int e = 8 * threadIdx.x; e < nq * P; e += 8 * blockDim.x) {
+        const int hq = e / P;
+        const int i = e - hq * P;  // a multiple of 8: P is 32 or 64
+        const uint16_t* qx = qb + hq * D + i;
+        uint32_t wx[4], wy[4];
+        if (q16) {
+            const uint4 x4 = __ldg(reinterpret_cast<const uint4*>(qx));
+            const uint4 y4 = __ldg(reinterpret_cast<const uint4*>(qx + P));
+            wx[0] = x4.x; wx[1] = x4.y; wx[2] = x4.z; wx[3] = x4.w;
+            wy[0] = y4.x; wy[1] = y4.y; wy[2] = y4.z; wy[3] = y4.w;
+        } else {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                wx[u] = uint32_t(qx[2 * u]) | (uint32_t(qx[2 * u + 1]) << 16);
+                wy[u] = uint32_t(qx[P + 2 * u]) | (uint32_t(qx[P + 2 * u + 1]) << 16);
+            }
+        }
+        float rx[8], ry[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const float x = __uint_as_float((u & 1) ? (wx[u >> 1] & 0xffff0000u) : (wx[u >> 1] << 16));
+            const float y = __uint_as_float((u & 1) ? (wy[u >> 1] & 0xffff0000u) : (wy[u >> 1] << 16));
+            const float sn = s_sin[i + u], cs = s_cos[i + u];
+            rx[u] = fmaf(x, cs, -y * sn) * a.scale;
+            ry[u] = fmaf(y, cs, x * sn) * a.scale;
+        }
+        float4* ox = reinterpret_cast<float4*>(q_s + hq * D + i);
+        float4* oy = reinterpret_cast<float4*>(q_s + hq * D + i + P);
+        ox[0] = make_float4(rx[0], rx[1], rx[2], rx[3]);
+        ox[1] = make_float4(rx[4], rx[5], rx[6], rx[7]);
+        oy[0] = make_float4(ry[0], ry[1], ry[2], ry[3]);
+        oy[1] = make_float4(ry[4], ry[5], ry[6], ry[7]);
+    }
+    __syncthreads();
+
+    if (wact) {
+        // Q A-fragments (rows = heads of the group; rows >= g and 8..15 are
+        // zero); k-step j of lane group t covers dimensions
+        // 8 (t + 4 (j / 2)) + 4 (j % 2) + 0..3, as the K chunks it reads
+        uint32_t qh[KS][2], ql[KS][2];
+        {
+            const bool hv = gid < g;
+            const float* qr = q_s + ((kh - kh0) * g + (hv ? gid : 0)) * D;
+#pragma unroll
+            for (int j = 0; j < KS; ++j) {
+                const int base = 8 * (t + 4 * (j >> 1)) + 4 * (j & 1);
+                const float x0 = hv ? qr[base] : 0.0f, x1 = hv ? qr[base + 1] : 0.0f;
+                const float x2 = hv ? qr[base + 2] : 0.0f, x3 = hv ? qr[base + 3] : 0.0f;
+                split_bf16x2(x0, x1, qh[j][0], ql[j][0]);
+                split_bf16x2(x2, x3, qh[j][1], ql[j][1]);
+            }
+        }
+        float o[KS][4];
+#pragma unroll
+        for (int mt = 0; mt < KS; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.0f;
+        float m_run = -INFINITY, l_run = 0.0f;
+        const int lslot = (lane & 7) + ((lane >> 4) & 1) * 8;
+        const int ldim = ((lane >> 3) & 1) * 8;
+
+        for (int n = 0; n < n_tiles; ++n) {
+            const int st = n % NS;
+            // this lane's copies of tile n are complete; after the warp
+            // barrier every lane's are visible
+            asm volatile("cp.async.wait_group %0;" ::"n"(NS - 2) : "memory");
+            __syncwarp();
+            // the tile NS - 1 ahead into the stage tile n - 1 used
+            {
+                const int32_t bn = blk_next;
+                blk_next = block_id(n + NS);
+                issue(n + NS - 1, bn);
+            }
+            const uint32_t mask = s_mask[warp][st];
+
+            // S = Q K^T for the two slot tiles (slots gid and 8 + gid)
+            const uint16_t* kt = wk + st * KT;
+            float sc[2][4];
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) {
+                const int slot = nt * 8 + gid;
+                uint4 kv[LV];
+#pragma unroll
+                for (int u = 0; u < LV; ++u)
+                    kv[u] = *reinterpret_cast<const uint4*>(kt + slot * D + (((t + 4 * u) ^ ((slot & 1) << 2)) * 8));
+                sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.0f;
+#pragma unroll
+                for (int j = 0; j < KS; ++j) {
+                    const uint4& w = kv[j >> 1];
+                    const uint32_t b0 = (j & 1) ? w.z : w.x;
+                    const uint32_t b1 = (j & 1) ? w.w : w.y;
+                    mma_16816(sc[nt], qh[j][0], 0u, qh[j][1], 0u, b0, b1);
+                    mma_16816(sc[nt], ql[j][0], 0u, ql[j][1], 0u, b0, b1);
+                }
+            }
+
+            // online softmax of head row gid over the 16 slots
+            float v[4] = {sc[0][0], sc[0][1], sc[1][0], sc[1][1]};
+            const int sl[4] = {2 * t, 2 * t + 1, 8 + 2 * t, 9 + 2 * t};
+            float mx = -INFINITY;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                if (!((mask >> sl[i]) & 1u)) v[i] = -INFINITY;
+                mx = fmaxf(mx, v[i]);
+            }
+            mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 1));
+            mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 2));
+            const float m_new = fmaxf(m_run, mx);
+            // arguments are <= 0: __expf's error (a few ulp) is far inside
+            // the float32 accumulation's
+            const float alpha = m_new == -INFINITY ? 1.0f : __expf(m_run - m_new);
+            float ps = 0.0f;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                v[i] = v[i] == -INFINITY ? 0.0f : __expf(v[i] - m_new);
+                ps += v[i];
+            }
+            ps += __shfl_xor_sync(kFull, ps, 1);
+            ps += __shfl_xor_sync(kFull, ps, 2);
+            l_run = l_run * alpha + ps;
+            m_run = m_new;
+            // O^T columns are heads 2t, 2t+1: their rescale factors live in rows 2t, 2t+1
+            const float a0 = __shfl_sync(kFull, alpha, (2 * t) * 4);
+            const float a1 = __shfl_sync(kFull, alpha, (2 * t + 1) * 4);
+#pragma unroll
+            for (int mt = 0; mt < KS; ++mt) {
+                o[mt][0] *= a0; o[mt][1] *= a1; o[mt][2] *= a0; o[mt][3] *= a1;
+            }
+            uint32_t pb0h, pb0l, pb1h, pb1l;
+            split_bf16x2(v[0], v[1], pb0h, pb0l);
+            split_bf16x2(v[2], v[3], pb1h, pb1l);
+
+            // O^T += V^T P^T
+#pragma unroll
+            for (int mt = 0; mt < KS; ++mt) {
+                uint32_t r0, r1, r2, r3;
+                const uint32_t addr = wv_s + uint32_t((st * VT + lslot * PITCH + mt * 16 + ldim) * 2);
+                asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                             : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                             : "r"(addr));
+                mma_16816(o[mt], r0, r1, r2, r3, pb0h, pb1h);
+                mma_16816(o[mt], r0, r1, r2, r3, pb0l, pb1l);
+            }
+            __syncwarp();  // stage st is refilled at the next iteration
+        }
+
+        // heads 2t, 2t+1 of this lane's O^T columns
+        const float l0 = __shfl_sync(kFull, l_run, (2 * t) * 4);
+        const float l1 = __shfl_sync(kFull, l_run, (2 * t + 1) * 4);
+        const float m0 = __shfl_sync(kFull, m_run, (2 * t) * 4);
+        const float m1 = __shfl_sync(kFull, m_run, (2 * t + 1) * 4);
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int h = 2 * t + hh;
+            if (h >= g) continue;
+            const int64_t o_idx = (int64_t(b) * a.n_layers + l) * a.n_q_heads + kh * g + h;
+            const float lh = hh ? l1 : l0;
+            if (a.splits == 1) {
+                const float inv = lh > 0.0f ? 1.0f / lh : 0.0f;
+                float* out = a.out + o_idx * D;
+#pragma unroll
+                for (int mt = 0; mt < KS; ++mt) {
+                    out[mt * 16 + gid] = o[mt][hh] * inv;
+                    out[mt * 16 + gid + 8] = o[mt][2 + hh] * inv;
+                }
+            } else {
+                float* part = a.partial + (o_idx * a.splits + split) * (D + 2);
+#pragma unroll
+                for (int mt = 0; mt < KS; ++mt) {
+                    part[mt * 16 + gid] = o[mt][hh];
+                    part[mt * 16 + gid + 8] = o[mt][2 + hh];
+                }
+                if (gid == 0) {
+                    part[D] = hh ? m1 : m0;
+                    part[D + 1] = lh;
+                }
+            }
+        }
+    }
+    // every copy this thread issued has landed before the CTA may end
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    if (err) atomicOr(a.status, err);
+}
+
 // Merge the chunks of one (sequence, layer, query head). The chunks' maxima
 // and sums are reduced by the whole CTA, their weights exp(m_s - M) staged in
 // shared memory 256 at a time, and thread d accumulates dimension d over the
@@ -756,28 +1082,25 @@ cudaError_t launch_gp(const DecodeArgs& a, dim3 grid, size_t smem, cudaStream_t 
 cudaError_t launch_decode(const DecodeArgs& a, int gp, dim3 grid, size_t smem,
                           cudaStream_t stream) {
     cudaError_t e;
-    if (a.head_dim == 64 || a.head_dim == 128) {
+    if (a.ring) {
+        // small batch: KV heads split over CTAs, K and V streamed through a
+        // shared-memory ring per warp
+        const int n_hg = (a.n_kv_heads + kRingWarps - 1) / kRingWarps;
+        const int D = a.head_dim;
+        const size_t sm = size_t(kRingWarps) * a.group * D * sizeof(float) +
+                          size_t(kRingWarps) * kRingStages * 16 * (D + D + 8) * sizeof(uint16_t);
+        dim3 g2 = grid;
+        g2.x *= unsigned(n_hg);
+        auto k = D == 64 ? decode_ring_kernel<64> : decode_ring_kernel<128>;
+        e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
+        if (e == cudaSuccess) e = launch_pdl(k, g2, dim3(kRingWarps * 32), sm, stream, a);
+    } else if (a.head_dim == 64 || a.head_dim == 128) {
         // tensor-core kernel: rotated queries + two staged V tiles per warp
         const size_t sm = size_t(a.n_q_heads) * a.head_dim * sizeof(float) +
                           size_t(kDecodeThreads / 32) * 2 * 16 * (a.head_dim + 8) * sizeof(uint16_t);
-        // a batch that fills under ~2 waves of resident CTAs splits its KV
-        // heads over more CTAs (a shorter chain per CTA)
-        const int n_hg = (a.n_kv_heads + kDecodeThreads / 32 - 1) / (kDecodeThreads / 32);
-        int dev = 0, sms = 148;
-        if (cudaGetDevice(&dev) == cudaSuccess)
-            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        const bool hg = n_hg > 1 && int64_t(grid.x) * grid.y * grid.z < int64_t(sms) * 6;
-        dim3 g2 = grid;
-        if (hg) g2.x *= unsigned(n_hg);
-        if (a.head_dim == 64) {
-            auto k = hg ? decode_mma_kernel<64, true> : decode_mma_kernel<64, false>;
-            e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
-            if (e == cudaSuccess) e = launch_pdl(k, g2, dim3(kDecodeThreads), sm, stream, a);
-        } else {
-            auto k = hg ? decode_mma_kernel<128, true> : decode_mma_kernel<128, false>;
-            e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
-            if (e == cudaSuccess) e = launch_pdl(k, g2, dim3(kDecodeThreads), sm, stream, a);
-        }
+        auto k = a.head_dim == 64 ? decode_mma_kernel<64, false> : decode_mma_kernel<128, false>;
+        e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
+        if (e == cudaSuccess) e = launch_pdl(k, grid, dim3(kDecodeThreads), sm, stream, a);
     } else {
         // groups of 1, 2 and 4 query heads run as 4 (padded) heads x 8 slots per
         // warp iteration, groups of 5..8 as 8 heads x 4 slots

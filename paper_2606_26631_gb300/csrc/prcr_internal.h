@@ -256,11 +256,14 @@ struct DecodeArgs {
     int32_t group;
     int32_t splits;
     int32_t chunk;
+    int32_t ring;               // small batch: the ring-staged kernel (head_dim 64, 128)
     float scale;
     uint64_t turn_freq[kMaxPairs];  // pair i: round(inv_freq_i / (2 pi) * 2^64)
 };
 
 constexpr int kDecodeMaxChunk = 4096;
+constexpr int kDecodeRingWarps = 4;   // KV heads (one per warp) per CTA of the ring kernel
+constexpr int kDecodeRingCtasPerSm = 2;
 
 constexpr int kSelectMaxQHeads = 128;
 constexpr int kSelectTokTile = 16;   // smallest tile of the logits kernel (sizes the workspace)
