@@ -130,24 +130,32 @@ def kernel_launches(fn):
 
 
 class L2Flush:
-    """Evicts L2 between timed steps by writing a buffer of twice its size."""
+    """Evicts L2 between timed steps: writes a buffer of twice its size, then
+    reads another of twice its size, so that the next step finds none of its
+    inputs in L2 and no dirty lines whose write-back would land inside its
+    timed region (a write alone leaves ~one L2 of dirty lines behind)."""
 
     def __init__(self, dev, mode, nbytes):
         import torch
         self.l2 = int(getattr(torch.cuda.get_device_properties(dev), "L2_cache_size", 0)) or (129 << 20)
         self.enabled = mode == "on" or (mode == "auto" and nbytes < 4 * self.l2)
         self.buf = torch.empty(2 * self.l2, dtype=torch.uint8, device=dev) if self.enabled else None
+        self.rbuf = (torch.zeros(2 * self.l2 // 4, dtype=torch.int32, device=dev)
+                     if self.enabled else None)
+        self.sink = torch.zeros((), dtype=torch.int64, device=dev) if self.enabled else None
         self.i = 0
 
     def __call__(self):
         if self.enabled:
             self.i += 1
             self.buf.fill_(self.i & 0xFF)
+            self.sink.add_(self.rbuf.sum())
 
     def describe(self, nbytes):
         if self.enabled:
-            return ("L2 flushed before each step (%d MB written); each step moves %.2f GB"
-                    % (2 * self.l2 >> 20, nbytes / 1e9))
+            return ("L2 flushed before each step (%d MB written, then %d MB of another buffer "
+                    "read); each step moves %.2f GB" % (2 * self.l2 >> 20, 2 * self.l2 >> 20,
+                                                      nbytes / 1e9))
         if nbytes >= 4 * self.l2:
             return "inputs larger than L2 (no flush): each step moves %.2f GB" % (nbytes / 1e9)
         return ("warm: no flush between steps, %.2f GB per step against a %d MB L2"

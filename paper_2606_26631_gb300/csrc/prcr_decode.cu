@@ -29,9 +29,6 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kDecodeThreads = 128;
-// slots of its chunk a CTA of the head-split (small batch) variant requests
-// into L2 before its tile loop: 4 KV heads x 64 slots x 512 B = 128 KB
-constexpr int kDecodeHgPrefetch = 64;
 
 
 // EPL consecutive bf16 of a row as EPL / 2 packed words.
@@ -299,9 +296,9 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int sr
                  : "memory");
 }
 
-// HG: the CTAs of a (sequence, layer, chunk) split its KV heads, one per warp
-// (small batches: more, shorter CTAs); else one CTA takes all of them.
-template <int D, bool HG>
+// One CTA per (sequence, layer, chunk) takes all KV heads of the layer, its
+// warps looping over them (small batches take decode_ring_kernel below).
+template <int D>
 __global__ void __launch_bounds__(kDecodeThreads, 3)
     decode_mma_kernel(const __grid_constant__ DecodeArgs a) {
     constexpr int KS = D / 16;     // k-steps of QK, m-tiles of PV
@@ -315,14 +312,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     uint16_t* vbuf = reinterpret_cast<uint16_t*>(smem_raw + size_t(Hq) * D * sizeof(float));
     const int b = blockIdx.z;
     const int l = blockIdx.y;
-    constexpr int NWARP = kDecodeThreads / 32;
-    int split = blockIdx.x, kh0 = 0, kh1 = a.n_kv_heads;
-    if constexpr (HG) {
-        const int n_hg = (a.n_kv_heads + NWARP - 1) / NWARP;
-        split = int(blockIdx.x) / n_hg;
-        kh0 = (int(blockIdx.x) - split * n_hg) * NWARP;
-        kh1 = min(a.n_kv_heads, kh0 + NWARP);
-    }
+    const int split = blockIdx.x, kh0 = 0, kh1 = a.n_kv_heads;
     uint32_t err = 0;
     pdl_allow();
 
@@ -366,35 +356,6 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     }
     const int64_t s_begin = int64_t(split) * a.chunk;
     const int64_t s_end = min(len, s_begin + a.chunk);
-    if constexpr (HG) {
-        // A small batch gives each warp a few tiles only, and a chain of a
-        // few DRAM round trips per warp is most of the CTA's life: the chunk's
-        // rows (its first kDecodeHgPrefetch slots) are all requested into L2
-        // now, so that the tile loop waits on L2. Slot s's KV heads kh0..kh1
-        // are one contiguous span of its K (and of its V) row.
-        const int64_t s_lo = a.cache_kind == PRCR_CACHE_CONTIGUOUS ? s_begin + 16 : s_begin;
-        const int64_t s_hi = min(s_end, s_begin + kDecodeHgPrefetch);
-        const int span = (kh1 - kh0) * D * 2;  // bytes
-        for (int64_t s = s_lo + threadIdx.x; s < s_hi; s += blockDim.x) {
-            int64_t row;
-            if (a.cache_kind == PRCR_CACHE_CONTIGUOUS) {
-                row = int64_t(b) * a.seq_stride + s * a.slot_stride;
-            } else {
-                const int64_t lb = s / a.block_size;
-                const int32_t blk = a.block_table[int64_t(b) * a.bt_stride + lb];
-                if (blk < 0 || blk >= a.n_blocks) continue;  // reported by the tile loop
-                row = int64_t(blk) * a.block_stride + (s - lb * a.block_size) * a.slot_stride;
-            }
-            const int64_t off = row + int64_t(l) * a.layer_stride + int64_t(kh0) * D;
-            const char* kp = reinterpret_cast<const char*>(a.cache_k + off);
-            const char* vp = reinterpret_cast<const char*>(a.cache_v + off);
-            for (int o = 0; o < span; o += 128) {
-                prefetch_l2(kp + o);
-                prefetch_l2(vp + o);
-            }
-        }
-    }
-
     __shared__ __align__(16) float s_cos[kMaxPairs];
     __shared__ __align__(16) float s_sin[kMaxPairs];
     for (int i = threadIdx.x; i < P; i += blockDim.x) {
@@ -404,7 +365,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     const uint16_t* qb = a.q + (int64_t(b) * a.n_layers + l) * Hq * D;
     // the query heads of this CTA's KV heads, eight rotation pairs per thread
     // (two 16-byte loads when the query rows are 16-byte aligned)
-    const int e_beg = HG ? kh0 * a.group * P : 0, e_end = HG ? kh1 * a.group * P : Hq * P;
+    const int e_beg = 0, e_end = Hq * P;
     const bool q16 = (reinterpret_cast<uintptr_t>(a.q) & 15) == 0;
     for (int e = e_beg + 8 * threadIdx.x; e < e_end; e += 8 * blockDim.x) {
         const int hq = e / P;
@@ -1098,7 +1059,7 @@ cudaError_t launch_decode(const DecodeArgs& a, int gp, dim3 grid, size_t smem,
         // tensor-core kernel: rotated queries + two staged V tiles per warp
         const size_t sm = size_t(a.n_q_heads) * a.head_dim * sizeof(float) +
                           size_t(kDecodeThreads / 32) * 2 * 16 * (a.head_dim + 8) * sizeof(uint16_t);
-        auto k = a.head_dim == 64 ? decode_mma_kernel<64, false> : decode_mma_kernel<128, false>;
+        auto k = a.head_dim == 64 ? decode_mma_kernel<64> : decode_mma_kernel<128>;
         e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
         if (e == cudaSuccess) e = launch_pdl(k, grid, dim3(kDecodeThreads), sm, stream, a);
     } else {
