@@ -607,6 +607,9 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
 // those reads are free of bank conflicts.
 constexpr int kRingWarps = kDecodeRingWarps;
 constexpr int kRingStages = 3;
+// rounds of eight query pairs per thread: the CTA's query heads are at most
+// kRingWarps * 8 (a GQA group of 8), i.e. kRingWarps * 8 * D / 2 pairs
+constexpr int kRingQRounds = 2;
 
 template <int D>
 __global__ void __launch_bounds__(kRingWarps * 32, 2)
@@ -654,6 +657,32 @@ __global__ void __launch_bounds__(kRingWarps * 32, 2)
     pdl_wait();
     const int64_t p = a.q_pos[b];
     int64_t len = a.seq_len[b];
+    // this thread's query words (eight rotation pairs of a head per round,
+    // at most kRingQRounds rounds), requested with the length so that they
+    // do not queue behind the ring's first copies
+    const uint16_t* qb = a.q + ((int64_t(b) * a.n_layers + l) * a.n_q_heads + kh0 * g) * D;
+    const bool q16 = (reinterpret_cast<uintptr_t>(a.q) & 15) == 0;
+    uint32_t wx[kRingQRounds][4], wy[kRingQRounds][4];
+#pragma unroll
+    for (int r = 0; r < kRingQRounds; ++r) {
+        const int e = 8 * (threadIdx.x + r * kRingWarps * 32);
+        if (e < nq * P) {
+            const int hq = e / P;
+            const uint16_t* qx = qb + hq * D + (e - hq * P);
+            if (q16) {
+                const uint4 x4 = __ldg(reinterpret_cast<const uint4*>(qx));
+                const uint4 y4 = __ldg(reinterpret_cast<const uint4*>(qx + P));
+                wx[r][0] = x4.x; wx[r][1] = x4.y; wx[r][2] = x4.z; wx[r][3] = x4.w;
+                wy[r][0] = y4.x; wy[r][1] = y4.y; wy[r][2] = y4.z; wy[r][3] = y4.w;
+            } else {
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    wx[r][u] = uint32_t(qx[2 * u]) | (uint32_t(qx[2 * u + 1]) << 16);
+                    wy[r][u] = uint32_t(qx[P + 2 * u]) | (uint32_t(qx[P + 2 * u + 1]) << 16);
+                }
+            }
+        }
+    }
     if (len < 0 || len > a.capacity) {
         err |= PRCR_ST_CAPACITY;
         len = len < 0 ? 0 : a.capacity;
@@ -734,30 +763,17 @@ __global__ void __launch_bounds__(kRingWarps * 32, 2)
     for (int i = threadIdx.x; i < P; i += blockDim.x)
         sincos_turns(double(p), a.turn_freq[i], &s_sin[i], &s_cos[i]);
     __syncthreads();
-    const uint16_t* qb = a.q + ((int64_t(b) * a.n_layers + l) * a.n_q_heads + kh0 * g) * D;
-    const bool q16 = (reinterpret_cast<uintptr_t>(a.q) & 15) == 0;
-    for (int e = 8 * threadIdx.x; e < nq * P; e += 8 * blockDim.x) {
+#pragma unroll
+    for (int r = 0; r < kRingQRounds; ++r) {
+        const int e = 8 * (threadIdx.x + r * kRingWarps * 32);
+        if (e >= nq * P) break;
         const int hq = e / P;
         const int i = e - hq * P;  // a multiple of 8: P is 32 or 64
-        const uint16_t* qx = qb + hq * D + i;
-        uint32_t wx[4], wy[4];
-        if (q16) {
-            const uint4 x4 = __ldg(reinterpret_cast<const uint4*>(qx));
-            const uint4 y4 = __ldg(reinterpret_cast<const uint4*>(qx + P));
-            wx[0] = x4.x; wx[1] = x4.y; wx[2] = x4.z; wx[3] = x4.w;
-            wy[0] = y4.x; wy[1] = y4.y; wy[2] = y4.z; wy[3] = y4.w;
-        } else {
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                wx[u] = uint32_t(qx[2 * u]) | (uint32_t(qx[2 * u + 1]) << 16);
-                wy[u] = uint32_t(qx[P + 2 * u]) | (uint32_t(qx[P + 2 * u + 1]) << 16);
-            }
-        }
         float rx[8], ry[8];
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
-            const float x = __uint_as_float((u & 1) ? (wx[u >> 1] & 0xffff0000u) : (wx[u >> 1] << 16));
-            const float y = __uint_as_float((u & 1) ? (wy[u >> 1] & 0xffff0000u) : (wy[u >> 1] << 16));
+            const float x = __uint_as_float((u & 1) ? (wx[r][u >> 1] & 0xffff0000u) : (wx[r][u >> 1] << 16));
+            const float y = __uint_as_float((u & 1) ? (wy[r][u >> 1] & 0xffff0000u) : (wy[r][u >> 1] << 16));
             const float sn = s_sin[i + u], cs = s_cos[i + u];
             rx[u] = fmaf(x, cs, -y * sn) * a.scale;
             ry[u] = fmaf(y, cs, x * sn) * a.scale;
