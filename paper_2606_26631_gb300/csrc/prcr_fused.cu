@@ -131,8 +131,8 @@ __global__ void __launch_bounds__(512) fused_kernel(const __grid_constant__ Fuse
     // are known to be well formed), and their range slots
     const int ra = last_at_or_before(s_rto, n_rev, tok0);
     const int rz = last_at_or_before(s_rto, n_rev, tok1 - 1);
-    if (tid < 6 * (rz - ra + 1) && tid < 6 * kFusedMaxRevisits)
-        s_mm[tid / 6][tid % 6] = (tid % 6) < 3 ? INT_MAX : INT_MIN;
+    for (int i = tid; i < 6 * min(rz - ra + 1, kFusedMaxRevisits); i += bd)
+        s_mm[i / 6][i % 6] = (i % 6) < 3 ? INT_MAX : INT_MIN;
     if (__syncthreads_or(bad)) {
         if (lead && tid == 0) atomicOr(a.status, PRCR_ST_CSR);
         return;

@@ -93,6 +93,24 @@ EDGE = [
 ]
 
 
+def test_one_tile_touching_64_revisits():
+    """One-kernel path where a single CTA's tile (256 tokens at one thread per
+    token: one KV head of head_dim 16) spans all 64 revisits of the batch, so
+    that the CTA reduces 64 coordinate ranges at once (more range slots than
+    it has threads); every output against the oracle."""
+    import parity_util as pu
+    wl = Workload(name="edge-manyrev", n_layers=2, n_kv_heads=1, head_dim=16, sections=(2, 3, 3),
+                  n_seqs=4, grids=((2, 8, 8),), selection="random", cache="contiguous",
+                  cur_pos=("uniform", 50, 5000), extra=(16, 16, 1, 4))
+    batch = make_batch(wl, device=DEV, seed=9)
+    assert batch.n_revisits == 64 and batch.total_k <= 256
+    rv = pu.make_revisit(batch)
+    assert _kernel_names(rv.run) == ["fused_kernel"]
+    torch.cuda.synchronize()
+    assert rv.status_value() == 0
+    pu.full_check(batch, rv)
+
+
 @pytest.mark.parametrize("wl", EDGE, ids=[w.name for w in EDGE])
 def test_edge_shapes(wl):
     import parity_util as pu
