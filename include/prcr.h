@@ -39,10 +39,12 @@
  *  - State: the outputs of a call depend only on its arguments. The library
  *    keeps process-wide caches that are filled on first use and read-only
  *    afterwards (guarded by a mutex): the turn rates per (theta, head_dim),
- *    the SM count and kernel occupancies per device, and, for
- *    prcr_rebind_inject_static only, a fixed scratch array per device and its
- *    address. Every entry point except prcr_rebind_inject_static may be
- *    called from several host threads at once.
+ *    the SM count, kernel occupancies and the one-kernel revisit path's
+ *    shared-memory limit per device, and, for prcr_rebind_inject_static only,
+ *    a fixed scratch array per device and its address. The per-device entries
+ *    assume the device is not reset while the process uses the library.
+ *    Every entry point except prcr_rebind_inject_static may be called from
+ *    several host threads at once.
  */
 #ifndef PRCR_H_
 #define PRCR_H_
