@@ -198,3 +198,48 @@ def test_select_interleaved_layout():
                                   wl.theta, O.LAYOUT_INTERLEAVED)
             assert (np.abs(sc[b] - ref) / ref).max() <= 1e-4, wl.name
             assert np.array_equal(sel[b], _topk_by(sc[b].astype(np.float64), k))
+
+
+# Coordinate structures beyond one image per sequence: two images of widths
+# 4 and 16 in one sequence, a 24-wide video with a t section that ends inside
+# an 8-pair group, head_dim 64 with a GQA group of 8, and a sequence whose
+# coordinates are shuffled (no token shares a row or column with its index
+# neighbours). The relevance must not depend on any grid regularity.
+GRID_SHAPES = {
+    "rot-w4-w16": (Workload(name="rot-w4-w16", n_layers=1, n_kv_heads=2, head_dim=128,
+                            sections=(24, 20, 20), n_seqs=2, grids=((2, 6, 4), (1, 9, 16)),
+                            selection="random", cache="contiguous", cur_pos=("uniform", 300, 5000),
+                            extra=(1, 1, 1, 20)), 8, False),
+    "rot-t20": (Workload(name="rot-t20", n_layers=1, n_kv_heads=4, head_dim=128,
+                         sections=(20, 20, 24), n_seqs=2, grids=((3, 11, 24),), selection="random",
+                         cache="contiguous", cur_pos=("uniform", 300, 5000), extra=(1, 1, 1, 20)),
+                16, False),
+    "rot-d64-g8": (Workload(name="rot-d64-g8", n_layers=1, n_kv_heads=2, head_dim=64,
+                            sections=(8, 12, 12), n_seqs=2, grids=((1, 20, 24),), selection="random",
+                            cache="contiguous", cur_pos=("uniform", 300, 5000), extra=(1, 1, 1, 20)),
+                   16, False),
+    "rot-shuffled": (get("qwen2vl-2b"), 8, True),
+}
+
+
+@pytest.mark.parametrize("name", sorted(GRID_SHAPES))
+def test_select_coordinate_structures(name):
+    wl, Hq, shuffle = GRID_SHAPES[name]
+    batch = make_batch(wl, device=DEV)
+    B, M, D = wl.n_seqs, wl.n_tokens, wl.head_dim
+    if shuffle:
+        perm = torch.randperm(M, generator=torch.Generator().manual_seed(5)).to(DEV)
+        batch.coords[0] = batch.coords[0][perm].clone()
+    k = min(40, M - 1)
+    g = torch.Generator(device=DEV)
+    g.manual_seed(29)
+    q = (3.0 * torch.randn((B, Hq, D), generator=g, device=DEV)).to(torch.bfloat16)
+    idx, sro, rto, score = _select(batch, 0, Hq, k, q, batch.p_txt)
+    qv = O.bf16_bits_to_f64(q.view(torch.int16).cpu().numpy())
+    coords = batch.coords.cpu().numpy()
+    for b in range(B):
+        k_raw = batch.store_k[b, 0].view(torch.int16).cpu().numpy()
+        ref = O.ads_relevance(qv[b], int(batch.p_txt[b]), k_raw, coords[b], D, wl.sections, wl.theta)
+        rel_err = np.abs(score[b] - ref) / ref
+        assert rel_err.max() <= 1e-4, (b, rel_err.max())
+        assert np.array_equal(idx[b], _topk_by(score[b].astype(np.float64), k))
