@@ -696,11 +696,14 @@ int prcr_select_topk(const prcr_rope_cfg* cfg, const prcr_store_desc* store, int
     if ((rc = check_store(cfg, store))) return rc;
     if (n_seqs > store->n_seqs) return PRCR_EINVAL;
     SelectArgs a = {};
-    // token tiles of the logits kernel: 64 tokens (32 at head_dim 256, whose
-    // cos/sin rows are twice as long)
+    // token tiles of the softmax statistics: 16 tokens (one warp's MMA rows)
+    // for the tensor-core logits kernel (head_dim 64, 128); else the CUDA-core
+    // kernel's tiles, 64 tokens (32 at head_dim 256, whose cos/sin rows are
+    // twice as long)
+    const int D = cfg->head_dim;
     rc = select_common(cfg, n_seqs, layer, n_q_heads, store->n_tokens, q, q_pos, k, idx_out,
                        seq_rev_off, rev_tok_off, score_out, workspace, workspace_bytes,
-                       cfg->head_dim > 128 ? 32 : 64, a);
+                       D == 64 || D == 128 ? 16 : (D > 128 ? 32 : 64), a);
     if (rc || n_seqs == 0) return rc;
     a.store_k = static_cast<const uint16_t*>(store->k);
     a.store_seq_stride = store->seq_stride;

@@ -248,169 +248,212 @@ __global__ void __launch_bounds__(256, 3) ads_logits_kernel(const __grid_constan
 }
 
 // D += A B on tensor cores: mma.sync m16n8k8 with tf32 operands (the upper
-// 19 bits of each float32 register), float32 accumulate.
-__device__ __forceinline__ void mma_1688_tf32(float (&c)[4], uint32_t a0, uint32_t a2, uint32_t b0,
-                                              uint32_t b1) {
+// 19 bits of each float32 register), float32 accumulate. Fragments as the
+// PTX ISA lays them out for this shape: a0 (row g, col t), a1 (row g + 8,
+// col t), a2 (row g, col t + 4), a3 (row g + 8, col t + 4); b0 (row t, col
+// g), b1 (row t + 4, col g); lane = 4 g + t.
+__device__ __forceinline__ void mma_1688_tf32(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                              uint32_t a3, uint32_t b0, uint32_t b1) {
     asm volatile(
         "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
         "{%8,%9}, {%0,%1,%2,%3};"
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-        : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// Tensor-core logits (head_dim 64 and 128). Persistent over token tiles like
-// the kernel above; a tile is 64 tokens, one octet of 8 per warp, and a warp
-// takes its octet through all KV heads:
-//   S (16 rows = the group's query heads, rows >= g zero; 8 tokens)
-//     = Q (16 x D) K_rot^T (D x 8), D / 8 k-steps of mma.sync m16n8k8 (tf32),
-//   K_rot the keys turned by the offsets of their coordinates from p.
-// The dot product does not depend on the order of the dimensions, so k-step j
-// of lane group t (= lane & 3) takes pair t * P/4 + j: k-slot t holds its
-// first-half dimension and k-slot t + 4 its rotate-half partner. A lane then
-// owns P/4 whole pairs of its token (= lane >> 2), loads them as two
-// contiguous runs and rotates them itself with its own cos/sin, computed once
-// per octet and reused for every KV head. The raw bf16 queries are exact
-// tf32 operands; each rotated key is split into a tf32 head (truncation) and
-// its float32 remainder (< 2^-10 of the value, itself truncated by the MMA),
-// and both products are summed (float32 accumulate): each keeps ~20
-// significant bits (float32-level logits) over float32's range.
-// The accumulator of lane (g, t) holds head g at tokens 2t, 2t+1 of the octet.
-// SPLIT: work items cover a group of KV heads (small batches); else every
-// item covers all of them.
-template <int D, bool SPLIT>
-__global__ void __launch_bounds__(256, 2) ads_logits_mma_kernel(const __grid_constant__ SelectArgs a) {
+__device__ __forceinline__ uint32_t word_of(const uint4& v, int i) {
+    return i == 0 ? v.x : (i == 1 ? v.y : (i == 2 ? v.z : v.w));
+}
+
+// Tensor-core logits (head_dim 64 and 128). Persistent over work items
+// (sequence, group of at most 8 KV heads, 16 NW tokens); warp w of a CTA
+// takes tokens 16 w .. 16 w + 15 of the item through the group's KV heads:
+//   S (16 rows = the warp's tokens; 8 columns = the GQA group's query heads,
+//      columns >= g zero) = K_rot Q^T, D / 8 k-steps of mma.sync m16n8k8 (tf32),
+//   K_rot the raw keys turned by the offsets of their coordinates from p.
+// The dot product does not depend on the order of the dimensions, so the
+// k-slots are permuted: at k-step s, lane group t (= lane & 3) holds pair
+// 32 (s / 8) + 8 t + s % 8 of its two tokens (rows g and g + 8), the
+// first-half dimension in k-slot t and its rotate-half partner in k-slot
+// t + 4. A lane then loads each half of its two rows as 16-byte runs (the
+// four lanes of a token cover 64 contiguous bytes) and rotates the two
+// tokens' pairs together in packed float2 arithmetic. The cos/sin of a
+// lane's (token, pair) are computed once per item into the warp's
+// shared-memory table and read back for every KV head. The raw bf16 queries
+// are exact tf32 operands (B, kept in shared memory in fragment order per
+// (sequence, head group)); each rotated key is split into a tf32 head
+// (truncation, one bit operation) and its float32 remainder (< 2^-10 of the
+// value, itself truncated by the MMA), and both products are summed in
+// float32: ~20 significant bits per product over float32's range. Runs of
+// 16-byte loads are double-buffered: the run two ahead is requested as soon
+// as a buffer's words are used. Each KV head's logits go straight from the
+// accumulators to global memory; the softmax statistics are left to the
+// normaliser kernel.
+template <int D, int NW>
+__global__ void __launch_bounds__(NW * 32, 2) ads_logits_mma_kernel(const __grid_constant__ SelectArgs a) {
     pdl_allow();
     pdl_wait();
-    constexpr int P = D / 2, PL = P / 4, T = 64;
-    constexpr int NW = PL / 8;  // 16-byte loads per half row per lane
+    constexpr int P = D / 2, KS = D / 8, NR = KS / 8;  // k-steps; 16-byte runs per half row
+    constexpr int T = 16 * NW;                         // tokens per work item
+    static_assert(NR == 1 || NR == 2, "head_dim 64 or 128");
     extern __shared__ __align__(16) float sm[];
     const int Hq = a.n_q_heads, H = a.n_kv_heads, g = Hq / H, M = a.n_tokens;
-    // a work item is (sequence, group of KPI KV heads, token tile), tiles fastest
-    const int KPI = SPLIT ? a.kh_per_item : H, n_khg = SPLIT ? (H + KPI - 1) / KPI : 1;
-    uint2* qa_s = reinterpret_cast<uint2*>(sm);                  // [KPI][PL][32]: (a0, a2), raw queries
-    float* lg_s = reinterpret_cast<float*>(qa_s + KPI * PL * 32);  // [Hq][T + 1]
+    const int KPI = a.kh_per_item, n_khg = (H + KPI - 1) / KPI;
+    const int n_it = (M + T - 1) / T;  // work items per (sequence, head group)
+    uint4* qf_s = reinterpret_cast<uint4*>(sm);  // [KPI][KS / 2][32] B fragments
+    float4* tr_s = reinterpret_cast<float4*>(qf_s + KPI * (KS / 2) * 32);  // [NW][KS][32]
+    uint64_t* tf_s = reinterpret_cast<uint64_t*>(tr_s + NW * KS * 32);      // [P] turn rates
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int gid = lane >> 2, tq = lane & 3;
-    const int64_t total = int64_t(a.n_seqs) * n_khg * a.n_tiles;
-    const int64_t t_beg = total * blockIdx.x / gridDim.x, t_end = total * (blockIdx.x + 1) / gridDim.x;
-    // axis of each of this lane's pairs, two bits each
+    for (int i = tid; i < P; i += NW * 32) tf_s[i] = a.turn_freq[i];
+    __syncthreads();
+    // axis of this lane's pair at each k-step, two bits each
     uint32_t axes = 0u;
 #pragma unroll
-    for (int p = 0; p < PL; ++p)
-        axes |= uint32_t(pair_axis(tq * PL + p, a.layout, a.sec_t, a.sec_h, a.sec_w)) << (2 * p);
+    for (int s = 0; s < KS; ++s)
+        axes |= uint32_t(pair_axis(32 * (s / 8) + 8 * tq + s % 8, a.layout, a.sec_t, a.sec_h,
+                                   a.sec_w)) << (2 * s);
+    const int64_t total = int64_t(a.n_seqs) * n_khg * n_it;
+    const int64_t i_beg = total * blockIdx.x / gridDim.x, i_end = total * (blockIdx.x + 1) / gridDim.x;
     int64_t cur_bg = -1;
+    float4* tr_w = tr_s + warp * KS * 32 + lane;
+    const int64_t layer_off = int64_t(a.layer) * a.store_layer_stride + 8 * tq;
 
-    for (int64_t item = t_beg; item < t_end; ++item) {
-        const int64_t bg = item / a.n_tiles;  // (sequence, KV-head group)
-        const int b = SPLIT ? int(bg / n_khg) : int(bg), j = int(item - bg * a.n_tiles);
-        const int kh_a = SPLIT ? int(bg - int64_t(b) * n_khg) * KPI : 0;
-        const int kh_b = SPLIT ? min(H, kh_a + KPI) : H;
-        const int m0 = j * T, nt = min(T, M - m0);
+    for (int64_t item = i_beg; item < i_end; ++item) {
+        const int64_t bg = item / n_it;  // (sequence, KV-head group)
+        const int b = int(bg / n_khg), it = int(item - bg * n_it);
+        const int kh_a = int(bg - int64_t(b) * n_khg) * KPI, nkh = min(KPI, H - kh_a);
+        const int j = it * NW + warp;  // the warp's 16-token tile
+        const int m0 = 16 * j, ntw = min(16, M - m0);
+        // this lane's two tokens (rows g and g + 8 of the warp's MMA tile); a
+        // token past the end reads the tile's last token (its logits are
+        // never written out)
+        const int ta = gid, tb = gid + 8;
+        const int ma = m0 + min(ta, ntw - 1), mb = m0 + min(tb, ntw - 1);
+        const uint16_t* kb = a.store_k + int64_t(b) * a.store_seq_stride + layer_off;
+        const uint16_t* ra = kb + int64_t(ma) * a.store_token_stride;
+        const uint16_t* rb = kb + int64_t(mb) * a.store_token_stride;
+        const int n_runs = nkh * NR;
+        // run r = (KV head kh_a + r / NR, 16-byte run r % NR): first-half x and
+        // second-half y words of tokens a and b
+        uint4 buf0[4], buf1[4];
+        auto fetch = [&](uint4 (&k)[4], int r) {
+            const int off = (kh_a + r / NR) * D + 32 * (r % NR);
+            k[0] = ld_stream(ra + off);
+            k[1] = ld_stream(ra + off + P);
+            k[2] = ld_stream(rb + off);
+            k[3] = ld_stream(rb + off + P);
+        };
+        if (ntw > 0) {
+            fetch(buf0, 0);
+            if (n_runs > 1) fetch(buf1, 1);
+        }
         if (bg != cur_bg) {
-            // the group's raw queries as A fragments (a bf16 value is an exact
-            // tf32 operand)
+            // the group's raw queries as B fragments (a bf16 value is an exact
+            // tf32 operand): entry (kh, s / 2, lane) holds k-steps s and s + 1
+            __syncthreads();  // every warp is done with the previous group's
             const uint16_t* qs = a.q + int64_t(b) * Hq * D;
-            for (int e = tid; e < (kh_b - kh_a) * PL * 32; e += blockDim.x) {
-                const int kh = kh_a + e / (PL * 32), ks = (e / 32) % PL, ln = e & 31;
-                const int h = ln >> 2, tt = ln & 3;
-                uint2 f = make_uint2(0u, 0u);
+            for (int e = tid; e < nkh * (KS / 2) * 32; e += NW * 32) {
+                const int kk = e / ((KS / 2) * 32), s2 = (e / 32) % (KS / 2), ln = e & 31;
+                const int h = ln >> 2, t4 = ln & 3;
+                uint4 f = make_uint4(0u, 0u, 0u, 0u);
                 if (h < g) {
-                    const uint16_t* qr = qs + (kh * g + h) * D + tt * PL + ks;
-                    f.x = uint32_t(qr[0]) << 16;
-                    f.y = uint32_t(qr[P]) << 16;
+                    const uint16_t* qr = qs + ((kh_a + kk) * g + h) * D;
+                    const int i0 = 32 * ((2 * s2) / 8) + 8 * t4 + (2 * s2) % 8;  // pair of k-step 2 s2
+                    f.x = uint32_t(qr[i0]) << 16;
+                    f.y = uint32_t(qr[i0 + P]) << 16;
+                    f.z = uint32_t(qr[i0 + 1]) << 16;
+                    f.w = uint32_t(qr[i0 + 1 + P]) << 16;
                 }
-                qa_s[e] = f;
+                qf_s[e] = f;
             }
             cur_bg = bg;
+            __syncthreads();
         }
-        __syncthreads();
+        if (ntw <= 0) continue;  // past the sequence's last token
 
-        // this warp's octet: the lane's token and its cos/sin for pairs tq * PL ..
-        const int to = 8 * warp + gid;  // token within the tile
-        const bool live = to < nt;
-        const int m = m0 + (live ? to : 0);
-        float cs[PL], sn[PL];
+        // cos/sin of the lane's (token, pair) at each k-step, at the offsets
+        // of the tokens' coordinates from the trigger position
         {
-            // angles at the offsets from the trigger position
-            const int32_t* crd = a.coords + int64_t(b) * a.coord_seq_stride + 3 * int64_t(m);
+            const int32_t* crd = a.coords + int64_t(b) * a.coord_seq_stride;
             const int64_t p = a.q_pos[b];
-            const int64_t c0 = crd[0] - p, c1 = crd[1] - p, c2 = crd[2] - p;
+            const int64_t oa[3] = {crd[3 * ma] - p, crd[3 * ma + 1] - p, crd[3 * ma + 2] - p};
+            const int64_t ob[3] = {crd[3 * mb] - p, crd[3 * mb + 1] - p, crd[3 * mb + 2] - p};
 #pragma unroll
-            for (int p = 0; p < PL; ++p) {
-                const uint32_t ax = (axes >> (2 * p)) & 3u;
-                sincos_coord(ax == 0 ? c0 : (ax == 1 ? c1 : c2), a.turn_freq[tq * PL + p], &sn[p], &cs[p]);
+            for (int s = 0; s < KS; ++s) {
+                const uint32_t ax = (axes >> (2 * s)) & 3u;
+                const uint64_t rate = tf_s[32 * (s / 8) + 8 * tq + s % 8];
+                float4 t;
+                sincos_coord(ax == 0 ? oa[0] : (ax == 1 ? oa[1] : oa[2]), rate, &t.z, &t.x);
+                sincos_coord(ax == 0 ? ob[0] : (ax == 1 ? ob[1] : ob[2]), rate, &t.w, &t.y);
+                tr_w[s * 32] = t;
             }
         }
-        const uint16_t* krow = a.store_k + int64_t(b) * a.store_seq_stride +
-                               int64_t(a.layer) * a.store_layer_stride +
-                               int64_t(m) * a.store_token_stride + tq * PL;
-        // a dead lane (token past the tile's end) reads its octet's first
-        // token: its logits are never written out, so its data need not be zero
-        uint4 xn[NW], yn[NW];
+        __syncwarp();
+
+        float acc[4];
+        auto clear = [&]() { acc[0] = acc[1] = acc[2] = acc[3] = 0.0f; };
+        clear();
+        // the eight k-steps of run u of KV head kk (words in k)
+        auto run = [&](const uint4 (&k)[4], int kk, int u) {
+            const uint4* qf = qf_s + (kk * (KS / 2) + 4 * u) * 32 + lane;
 #pragma unroll
-        for (int u = 0; u < NW; ++u) {
-            xn[u] = ld_stream(krow + kh_a * D + 8 * u);
-            yn[u] = ld_stream(krow + kh_a * D + P + 8 * u);
-        }
-        for (int kh = kh_a; kh < kh_b; ++kh) {
-            uint32_t xw[4 * NW], yw[4 * NW];
-#pragma unroll
-            for (int u = 0; u < NW; ++u) {
-                xw[4 * u] = xn[u].x; xw[4 * u + 1] = xn[u].y; xw[4 * u + 2] = xn[u].z; xw[4 * u + 3] = xn[u].w;
-                yw[4 * u] = yn[u].x; yw[4 * u + 1] = yn[u].y; yw[4 * u + 2] = yn[u].z; yw[4 * u + 3] = yn[u].w;
+            for (int s8 = 0; s8 < 8; ++s8) {
+                const int s = 8 * u + s8, w = s8 / 2;
+                const bool up = s8 & 1;  // upper bf16 of the word
+                const uint32_t wxa = word_of(k[0], w), wya = word_of(k[1], w);
+                const uint32_t wxb = word_of(k[2], w), wyb = word_of(k[3], w);
+                const float2 X = up ? make_float2(hi_f32(wxa), hi_f32(wxb))
+                                    : make_float2(lo_f32(wxa), lo_f32(wxb));
+                const float2 Y = up ? make_float2(hi_f32(wya), hi_f32(wyb))
+                                    : make_float2(lo_f32(wya), lo_f32(wyb));
+                const float4 t = tr_w[s * 32];
+                const float2 C = make_float2(t.x, t.y), S = make_float2(t.z, t.w);
+                const float2 ys = __fmul2_rn(Y, S), xs = __fmul2_rn(X, S);
+                const float2 Xr = __ffma2_rn(X, C, make_float2(-ys.x, -ys.y));
+                const float2 Yr = __ffma2_rn(Y, C, xs);
+                // tf32 heads by truncation, float32 remainders
+                const uint32_t hxa = __float_as_uint(Xr.x) & 0xffffe000u;
+                const uint32_t hxb = __float_as_uint(Xr.y) & 0xffffe000u;
+                const uint32_t hya = __float_as_uint(Yr.x) & 0xffffe000u;
+                const uint32_t hyb = __float_as_uint(Yr.y) & 0xffffe000u;
+                // remainders v - head, two per packed FMA with (-1, -1)
+                const float2 lx = __ffma2_rn(make_float2(__uint_as_float(hxa), __uint_as_float(hxb)),
+                                             make_float2(-1.0f, -1.0f), Xr);
+                const float2 ly = __ffma2_rn(make_float2(__uint_as_float(hya), __uint_as_float(hyb)),
+                                             make_float2(-1.0f, -1.0f), Yr);
+                const float lxa = lx.x, lxb = lx.y, lya = ly.x, lyb = ly.y;
+                const uint4 q2 = qf[(s8 / 2) * 32];
+                const uint32_t b0 = up ? q2.z : q2.x, b1 = up ? q2.w : q2.y;
+                mma_1688_tf32(acc, hxa, hxb, hya, hyb, b0, b1);
+                mma_1688_tf32(acc, __float_as_uint(lxa), __float_as_uint(lxb),
+                              __float_as_uint(lya), __float_as_uint(lyb), b0, b1);
             }
-            if (kh + 1 < kh_b) {  // the next head's pairs, in flight during this head's MMAs
+        };
+        // KV head kk done: its logits out (the softmax statistics come from
+        // the normaliser kernel, one pass over the logits)
+        const bool va = ta < ntw, vb = tb < ntw;
+        auto finish = [&](int kk) {
+            const int h0 = 2 * tq;  // columns 2t, 2t + 1
+            float* lg = a.logits + (int64_t(b) * Hq + (kh_a + kk) * g + h0) * M + m0;
 #pragma unroll
-                for (int u = 0; u < NW; ++u) {
-                    xn[u] = ld_stream(krow + (kh + 1) * D + 8 * u);
-                    yn[u] = ld_stream(krow + (kh + 1) * D + P + 8 * u);
+            for (int c = 0; c < 2; ++c) {
+                if (h0 + c < g) {
+                    if (va) lg[int64_t(c) * M + ta] = acc[c] * a.scale;
+                    if (vb) lg[int64_t(c) * M + tb] = acc[2 + c] * a.scale;
                 }
             }
-            float c[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-            const uint2* qa = qa_s + (kh - kh_a) * PL * 32 + lane;
-#pragma unroll
-            for (int ks = 0; ks < PL; ++ks) {
-                // pair ks of this lane: element ks of each half
-                const float x = (ks & 1) ? hi_f32(xw[ks >> 1]) : lo_f32(xw[ks >> 1]);
-                const float y = (ks & 1) ? hi_f32(yw[ks >> 1]) : lo_f32(yw[ks >> 1]);
-                const float kx = fmaf(x, cs[ks], -y * sn[ks]);
-                const float ky = fmaf(y, cs[ks], x * sn[ks]);
-                // keys: tf32 head by truncation (one bit operation), exact
-                // float32 remainder < 2^-10 |k|, truncated in turn by the MMA
-                const uint32_t bxh = __float_as_uint(kx) & 0xffffe000u;
-                const uint32_t byh = __float_as_uint(ky) & 0xffffe000u;
-                const uint32_t bxl = __float_as_uint(kx - __uint_as_float(bxh));
-                const uint32_t byl = __float_as_uint(ky - __uint_as_float(byh));
-                const uint2 f = qa[ks * 32];
-                mma_1688_tf32(c, f.x, f.y, bxh, byh);
-                mma_1688_tf32(c, f.x, f.y, bxl, byl);
-            }
-            if (gid < g) {  // (rows are T + 1 floats apart: 4-byte stores)
-                float* dst = lg_s + (kh * g + gid) * (T + 1) + 8 * warp + 2 * tq;
-                dst[0] = c[0] * a.scale;
-                dst[1] = c[1] * a.scale;
-            }
-        }
-        __syncthreads();
-
-        for (int hq = kh_a * g + warp; hq < kh_b * g; hq += blockDim.x >> 5) {
-            const float* row = lg_s + hq * (T + 1);
-            float mx = -INFINITY;
-            for (int t = lane; t < nt; t += 32) mx = fmaxf(mx, row[t]);
-#pragma unroll
-            for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-            float z = 0.0f;
-            float* dst = a.logits + (int64_t(b) * Hq + hq) * M + m0;
-            for (int t = lane; t < nt; t += 32) {
-                z += expf(row[t] - mx);
-                dst[t] = row[t];
-            }
-#pragma unroll
-            for (int o = 16; o; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
-            if (lane == 0) {
-                float* ts = a.tile_stats + ((int64_t(b) * Hq + hq) * a.n_tiles + j) * 2;
-                ts[0] = mx;
-                ts[1] = z;
+            clear();
+        };
+        // run r in buffer r % 2; once its words are used, run r + 2 is requested into it
+        for (int r = 0; r < n_runs; r += 2) {
+            run(buf0, r / NR, r % NR);
+            if (NR == 1) finish(r);
+            if (r + 2 < n_runs) fetch(buf0, r + 2);
+            if (r + 1 < n_runs) {
+                run(buf1, (r + 1) / NR, (r + 1) % NR);
+                finish((r + 1) / NR);
+                if (r + 3 < n_runs) fetch(buf1, r + 3);
             }
         }
     }
@@ -687,7 +730,76 @@ __global__ void __launch_bounds__(256) ads_norm_kernel(const __grid_constant__ S
     }
 }
 
+// Softmax normaliser of each (sequence, query head) straight from its logits
+// (the tensor-core logits kernel writes no tile statistics): every thread
+// keeps a running (max, sum of exp) over sixteen logits at a time (four
+// 16-byte loads when the row is 16-byte aligned), and the block merges them.
+__device__ __forceinline__ void merge_max_sum(float& m, float& s, float m2, float s2) {
+    const float mn = fmaxf(m, m2);
+    if (mn == -INFINITY) return;
+    s = (m == -INFINITY ? 0.0f : s * __expf(m - mn)) + (m2 == -INFINITY ? 0.0f : s2 * __expf(m2 - mn));
+    m = mn;
+}
+
+__global__ void __launch_bounds__(256) ads_norm_logits_kernel(const __grid_constant__ SelectArgs a) {
+    pdl_allow();
+    pdl_wait();
+    __shared__ float s_m[8], s_z[8];
+    const int hq = blockIdx.x, b = blockIdx.y, M = a.n_tokens;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const float* lg = a.logits + (int64_t(b) * a.n_q_heads + hq) * M;
+    float mx = -INFINITY, z = 0.0f;
+    auto chunk = [&](const float (&x)[16]) {
+        float cm = mx;
+#pragma unroll
+        for (int u = 0; u < 16; ++u) cm = fmaxf(cm, x[u]);
+        float cz = 0.0f;
+#pragma unroll
+        for (int u = 0; u < 16; ++u) cz += __expf(x[u] - cm);
+        z = (mx == -INFINITY ? 0.0f : z * __expf(mx - cm)) + cz;
+        mx = cm;
+    };
+    int i = 0;  // logits [0, i) done
+    if ((M & 3) == 0) {
+        const float4* l4 = reinterpret_cast<const float4*>(lg);
+        for (; i + 4096 <= M; i += 4096) {  // 256 threads x 16 logits
+            float x[16];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const float4 v = l4[(i >> 2) + u * 256 + threadIdx.x];
+                x[4 * u] = v.x; x[4 * u + 1] = v.y; x[4 * u + 2] = v.z; x[4 * u + 3] = v.w;
+            }
+            chunk(x);
+        }
+    }
+    for (; i + 4096 <= M; i += 4096) {
+        float x[16];
+#pragma unroll
+        for (int u = 0; u < 16; ++u) x[u] = lg[i + u * 256 + threadIdx.x];
+        chunk(x);
+    }
+    for (int t = i + threadIdx.x; t < M; t += 256) merge_max_sum(mx, z, lg[t], 1.0f);
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        const float m2 = __shfl_xor_sync(0xffffffffu, mx, o), z2 = __shfl_xor_sync(0xffffffffu, z, o);
+        merge_max_sum(mx, z, m2, z2);
+    }
+    if (lane == 0) {
+        s_m[warp] = mx;
+        s_z[warp] = z;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (int w = 1; w < 8; ++w) merge_max_sum(mx, z, s_m[w], s_z[w]);
+        float* nrm = a.norm + (int64_t(b) * a.n_q_heads + hq) * 2;
+        nrm[0] = mx == -INFINITY ? 0.0f : mx;
+        nrm[1] = mx == -INFINITY ? 0.0f : 1.0f / (z * float(a.n_q_heads));
+    }
+}
+
 // Relevance of every token: mean over the query heads of its softmax weight.
+// A thread takes four consecutive tokens (16-byte loads when the rows are
+// 16-byte aligned), eight heads' logits requested together.
 __global__ void __launch_bounds__(256) ads_relevance_kernel(const __grid_constant__ SelectArgs a) {
     pdl_allow();
     pdl_wait();
@@ -696,21 +808,50 @@ __global__ void __launch_bounds__(256) ads_relevance_kernel(const __grid_constan
     const int Hq = a.n_q_heads, M = a.n_tokens;
     for (int i = threadIdx.x; i < 2 * Hq; i += blockDim.x) s_n[i] = a.norm[int64_t(b) * Hq * 2 + i];
     __syncthreads();
-    const int m = blockIdx.x * blockDim.x + threadIdx.x;
+    const int m = 4 * (blockIdx.x * blockDim.x + threadIdx.x);
     if (m >= M) return;
     const float* lg = a.logits + int64_t(b) * Hq * M + m;
-    float r = 0.0f;
-    int h = 0;
-    for (; h + 8 <= Hq; h += 8) {  // eight heads' logits requested together
-        float x[8];
+    float r[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    if ((M & 3) == 0) {
+        int h = 0;
+        for (; h + 8 <= Hq; h += 8) {
+            float4 x[8];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) x[u] = lg[int64_t(h + u) * M];
+            for (int u = 0; u < 8; ++u) x[u] = *reinterpret_cast<const float4*>(lg + int64_t(h + u) * M);
 #pragma unroll
-        for (int u = 0; u < 8; ++u) r = fmaf(expf(x[u] - s_n[2 * (h + u)]), s_n[2 * (h + u) + 1], r);
+            for (int u = 0; u < 8; ++u) {
+                const float mh = s_n[2 * (h + u)], wh = s_n[2 * (h + u) + 1];
+                r[0] = fmaf(expf(x[u].x - mh), wh, r[0]);
+                r[1] = fmaf(expf(x[u].y - mh), wh, r[1]);
+                r[2] = fmaf(expf(x[u].z - mh), wh, r[2]);
+                r[3] = fmaf(expf(x[u].w - mh), wh, r[3]);
+            }
+        }
+        for (; h < Hq; ++h) {
+            const float4 x = *reinterpret_cast<const float4*>(lg + int64_t(h) * M);
+            const float mh = s_n[2 * h], wh = s_n[2 * h + 1];
+            r[0] = fmaf(expf(x.x - mh), wh, r[0]);
+            r[1] = fmaf(expf(x.y - mh), wh, r[1]);
+            r[2] = fmaf(expf(x.z - mh), wh, r[2]);
+            r[3] = fmaf(expf(x.w - mh), wh, r[3]);
+        }
+    } else {
+        const int n = min(4, M - m);
+        for (int h = 0; h < Hq; ++h) {
+            const float mh = s_n[2 * h], wh = s_n[2 * h + 1];
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                if (u < n) r[u] = fmaf(expf(lg[int64_t(h) * M + u] - mh), wh, r[u]);
+        }
     }
-    for (; h < Hq; ++h) r = fmaf(expf(lg[int64_t(h) * M] - s_n[2 * h]), s_n[2 * h + 1], r);
-    a.rel[int64_t(b) * M + m] = r;
-    if (a.score_out) a.score_out[int64_t(b) * M + m] = r;
+    const int n = min(4, M - m);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        if (u < n) {
+            a.rel[int64_t(b) * M + m + u] = r[u];
+            if (a.score_out) a.score_out[int64_t(b) * M + m + u] = r[u];
+        }
+    }
 }
 
 // Block-wide exclusive scan of one int per thread; returns the total.
@@ -767,8 +908,11 @@ __global__ void __launch_bounds__(1024) ads_select_kernel(const __grid_constant_
     // candidate is >= 1, so the padding never counts). Counting against
     // thresholds needs no histogram, hence no atomics on the few bins that
     // relevances sharing their high bits would all fall into.
+    // The search also stops as soon as exactly K keys reach X: the selection
+    // is then every key >= X (the compaction below takes all keys above X
+    // and, of those equal to X, exactly the K - above that remain).
     const unsigned int K = unsigned(a.k);
-    unsigned int X = 0u;
+    unsigned int X = 0u, cX = 0u;  // cX: keys >= X, once X > 0
     for (int bit = 30; bit >= 0; bit -= 2) {
         const unsigned int x1 = X | (1u << bit), x2 = X | (2u << bit), x3 = X | (3u << bit);
         unsigned int c1 = 0u, c2 = 0u, c3 = 0u;
@@ -791,8 +935,10 @@ __global__ void __launch_bounds__(1024) ads_select_kernel(const __grid_constant_
         const unsigned int t1 = __reduce_add_sync(0xffffffffu, wl ? s_cnt[lane] : 0u);
         const unsigned int t2 = __reduce_add_sync(0xffffffffu, wl ? s_cnt[32 + lane] : 0u);
         const unsigned int t3 = __reduce_add_sync(0xffffffffu, wl ? s_cnt[64 + lane] : 0u);
+        cX = t3 >= K ? t3 : (t2 >= K ? t2 : (t1 >= K ? t1 : cX));
         X = t3 >= K ? x3 : (t2 >= K ? x2 : (t1 >= K ? x1 : X));
         __syncthreads();
+        if (X != 0u && cX == K) break;  // uniform: every thread read the same counts
     }
     // keys strictly above X: all taken; of the keys equal to X, the first ones
     unsigned int above = 0u, n_eq = 0u;
@@ -873,41 +1019,46 @@ cudaError_t launch_logits(const SelectArgs& a, int n_seqs, int sms, cudaStream_t
     return launch_logits_g<L, 8>(a, n_seqs, sms, stream);
 }
 
+constexpr int kMmaWarps = 8;  // warps per CTA of the tensor-core logits kernel (16 tokens each)
+
+template <int D>
+size_t logits_mma_smem(int kpi) {
+    return size_t(kpi) * (D / 16) * 32 * 16 + size_t(kMmaWarps) * (D / 8) * 32 * 16 +
+           size_t(D / 2) * 8;
+}
+
 template <int D>
 cudaError_t launch_logits_mma(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream) {
-    const size_t smem = size_t(a.n_kv_heads) * (D / 8) * 32 * 8 +
-                        size_t(a.n_q_heads) * (a.tok_tile + 1) * 4;
-    cudaError_t e = cudaFuncSetAttribute(ads_logits_mma_kernel<D, false>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(ads_logits_mma_kernel<D, true>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    auto kern = ads_logits_mma_kernel<D, kMmaWarps>;
+    const int H = a.n_kv_heads;
+    SelectArgs b = a;
+    b.kh_per_item = H < 8 ? H : 8;  // KV heads per work item (sizes the query fragments)
+    const size_t smem_max = logits_mma_smem<D>(b.kh_per_item);
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem_max));
     if (e != cudaSuccess) return e;
     int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ads_logits_mma_kernel<D, false>, 256,
-                                                      smem);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kMmaWarps * 32, smem_max);
     if (e != cudaSuccess) return e;
     const int64_t resident = int64_t(sms) * (per_sm > 0 ? per_sm : 1);
-    // Few tiles (a small batch): split the KV heads over work items until
-    // there are two per resident CTA, so that short chains run side by side.
-    SelectArgs b = a;
-    const int H = a.n_kv_heads;
-    b.kh_per_item = H;
-    while (b.kh_per_item > 1 &&
-           int64_t(n_seqs) * a.n_tiles * ((H + b.kh_per_item - 1) / b.kh_per_item) < 2 * resident)
+    // Few tokens (a small batch): fewer KV heads per item until there are two
+    // items per resident CTA, so that short chains run side by side.
+    const int64_t n_it = (a.n_tokens + 16 * kMmaWarps - 1) / (16 * kMmaWarps);
+    auto items = [&](int kpi) { return int64_t(n_seqs) * n_it * ((H + kpi - 1) / kpi); };
+    while (b.kh_per_item > 1 && items(b.kh_per_item) < 2 * resident)
         b.kh_per_item = (b.kh_per_item + 1) / 2;
-    const int64_t items = int64_t(n_seqs) * a.n_tiles * ((H + b.kh_per_item - 1) / b.kh_per_item);
-    const unsigned grid = unsigned(items < resident ? items : resident);
-    return b.kh_per_item < H
-               ? launch_pdl(ads_logits_mma_kernel<D, true>, dim3(grid), dim3(256), smem, stream, b)
-               : launch_pdl(ads_logits_mma_kernel<D, false>, dim3(grid), dim3(256), smem, stream, b);
+    const int64_t n = items(b.kh_per_item);
+    const unsigned grid = unsigned(n < resident ? n : resident);
+    return launch_pdl(kern, dim3(grid), dim3(kMmaWarps * 32), logits_mma_smem<D>(b.kh_per_item),
+                      stream, b);
 }
 
 // The normalisers, relevances and selection after a logits kernel.
-static cudaError_t launch_select_tail(const SelectArgs& a, int n_seqs, cudaStream_t stream) {
-    cudaError_t e = launch_pdl(ads_norm_kernel, dim3(a.n_q_heads, n_seqs, 1), dim3(256), 0, stream, a);
+static cudaError_t launch_select_tail(const SelectArgs& a, int n_seqs, cudaStream_t stream,
+                                      bool norm_from_logits = false) {
+    cudaError_t e = launch_pdl(norm_from_logits ? ads_norm_logits_kernel : ads_norm_kernel,
+                               dim3(a.n_q_heads, n_seqs, 1), dim3(256), 0, stream, a);
     if (e != cudaSuccess) return e;
-    e = launch_pdl(ads_relevance_kernel, dim3((a.n_tokens + 255) / 256, n_seqs, 1), dim3(256), 0,
+    e = launch_pdl(ads_relevance_kernel, dim3((a.n_tokens + 1023) / 1024, n_seqs, 1), dim3(256), 0,
                    stream, a);
     if (e != cudaSuccess) return e;
     const int M = a.n_tokens;
@@ -922,9 +1073,10 @@ static cudaError_t launch_select_tail(const SelectArgs& a, int n_seqs, cudaStrea
 
 cudaError_t launch_select(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream) {
     cudaError_t e;
-    if (a.head_dim == 128 && a.tok_tile == 64) {
+    const bool mma = (a.head_dim == 128 || a.head_dim == 64) && a.tok_tile == 16;
+    if (a.head_dim == 128 && mma) {
         e = launch_logits_mma<128>(a, n_seqs, sms, stream);
-    } else if (a.head_dim == 64 && a.tok_tile == 64) {
+    } else if (a.head_dim == 64 && mma) {
         e = launch_logits_mma<64>(a, n_seqs, sms, stream);
     } else {
         const int L = a.head_dim <= 64 ? 4 : (a.head_dim <= 128 ? 8 : 16);
@@ -933,7 +1085,7 @@ cudaError_t launch_select(const SelectArgs& a, int n_seqs, int sms, cudaStream_t
                              : launch_logits<16>(a, n_seqs, sms, stream));
     }
     if (e != cudaSuccess) return e;
-    return launch_select_tail(a, n_seqs, stream);
+    return launch_select_tail(a, n_seqs, stream, mma);
 }
 
 cudaError_t launch_select_cached(const SelectArgs& a, int n_seqs, int sms, cudaStream_t stream) {
