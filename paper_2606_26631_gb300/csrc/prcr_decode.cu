@@ -827,24 +827,34 @@ __global__ void __launch_bounds__(kRingWarps * 32, 2)
 
             // S = Q K^T for the two slot tiles (slots gid and 8 + gid)
             const uint16_t* kt = wk + st * KT;
-            float sc[2][4];
+            // four independent accumulation chains (two slot tiles x the
+            // query's head and remainder), summed at the end
+            float sc[2][4], sl_[2][4];
+            uint4 kv[2][LV];
 #pragma unroll
             for (int nt = 0; nt < 2; ++nt) {
                 const int slot = nt * 8 + gid;
-                uint4 kv[LV];
 #pragma unroll
                 for (int u = 0; u < LV; ++u)
-                    kv[u] = *reinterpret_cast<const uint4*>(kt + slot * D + (((t + 4 * u) ^ ((slot & 1) << 2)) * 8));
+                    kv[nt][u] = *reinterpret_cast<const uint4*>(kt + slot * D + (((t + 4 * u) ^ ((slot & 1) << 2)) * 8));
                 sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.0f;
+                sl_[nt][0] = sl_[nt][1] = sl_[nt][2] = sl_[nt][3] = 0.0f;
+            }
 #pragma unroll
-                for (int j = 0; j < KS; ++j) {
-                    const uint4& w = kv[j >> 1];
+            for (int j = 0; j < KS; ++j) {
+#pragma unroll
+                for (int nt = 0; nt < 2; ++nt) {
+                    const uint4& w = kv[nt][j >> 1];
                     const uint32_t b0 = (j & 1) ? w.z : w.x;
                     const uint32_t b1 = (j & 1) ? w.w : w.y;
                     mma_16816(sc[nt], qh[j][0], 0u, qh[j][1], 0u, b0, b1);
-                    mma_16816(sc[nt], ql[j][0], 0u, ql[j][1], 0u, b0, b1);
+                    mma_16816(sl_[nt], ql[j][0], 0u, ql[j][1], 0u, b0, b1);
                 }
             }
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int r = 0; r < 4; ++r) sc[nt][r] += sl_[nt][r];
 
             // online softmax of head row gid over the 16 slots
             float v[4] = {sc[0][0], sc[0][1], sc[1][0], sc[1][1]};

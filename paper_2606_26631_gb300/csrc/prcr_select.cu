@@ -749,10 +749,12 @@ __global__ void __launch_bounds__(256) ads_norm_logits_kernel(const __grid_const
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const float* lg = a.logits + (int64_t(b) * a.n_q_heads + hq) * M;
     float mx = -INFINITY, z = 0.0f;
+    // sixteen logits (-inf past the end) into the running (max, sum of exp)
     auto chunk = [&](const float (&x)[16]) {
         float cm = mx;
 #pragma unroll
         for (int u = 0; u < 16; ++u) cm = fmaxf(cm, x[u]);
+        if (cm == -INFINITY) return;
         float cz = 0.0f;
 #pragma unroll
         for (int u = 0; u < 16; ++u) cz += __expf(x[u] - cm);
@@ -772,13 +774,15 @@ __global__ void __launch_bounds__(256) ads_norm_logits_kernel(const __grid_const
             chunk(x);
         }
     }
-    for (; i + 4096 <= M; i += 4096) {
+    for (; i < M; i += 4096) {
         float x[16];
 #pragma unroll
-        for (int u = 0; u < 16; ++u) x[u] = lg[i + u * 256 + threadIdx.x];
+        for (int u = 0; u < 16; ++u) {
+            const int t = i + u * 256 + threadIdx.x;
+            x[u] = t < M ? lg[t] : -INFINITY;
+        }
         chunk(x);
     }
-    for (int t = i + threadIdx.x; t < M; t += 256) merge_max_sum(mx, z, lg[t], 1.0f);
 #pragma unroll
     for (int o = 16; o; o >>= 1) {
         const float m2 = __shfl_xor_sync(0xffffffffu, mx, o), z2 = __shfl_xor_sync(0xffffffffu, z, o);
@@ -797,9 +801,12 @@ __global__ void __launch_bounds__(256) ads_norm_logits_kernel(const __grid_const
     }
 }
 
-// Relevance of every token: mean over the query heads of its softmax weight.
-// A thread takes four consecutive tokens (16-byte loads when the rows are
-// 16-byte aligned), eight heads' logits requested together.
+// Relevance of every token: mean over the query heads of its softmax weight,
+// the heads accumulated in ascending order. TPT consecutive tokens per thread:
+// four (16-byte loads, eight heads' logits requested together) for large
+// batches, one (sixteen heads requested together) where the grid would
+// otherwise be a few CTAs.
+template <int TPT>
 __global__ void __launch_bounds__(256) ads_relevance_kernel(const __grid_constant__ SelectArgs a) {
     pdl_allow();
     pdl_wait();
@@ -808,11 +815,23 @@ __global__ void __launch_bounds__(256) ads_relevance_kernel(const __grid_constan
     const int Hq = a.n_q_heads, M = a.n_tokens;
     for (int i = threadIdx.x; i < 2 * Hq; i += blockDim.x) s_n[i] = a.norm[int64_t(b) * Hq * 2 + i];
     __syncthreads();
-    const int m = 4 * (blockIdx.x * blockDim.x + threadIdx.x);
+    const int m = TPT * (blockIdx.x * blockDim.x + threadIdx.x);
     if (m >= M) return;
     const float* lg = a.logits + int64_t(b) * Hq * M + m;
-    float r[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-    if ((M & 3) == 0) {
+    float r[TPT];
+#pragma unroll
+    for (int u = 0; u < TPT; ++u) r[u] = 0.0f;
+    if (TPT == 1) {
+        int h = 0;
+        for (; h + 16 <= Hq; h += 16) {
+            float x[16];
+#pragma unroll
+            for (int u = 0; u < 16; ++u) x[u] = lg[int64_t(h + u) * M];
+#pragma unroll
+            for (int u = 0; u < 16; ++u) r[0] = fmaf(expf(x[u] - s_n[2 * (h + u)]), s_n[2 * (h + u) + 1], r[0]);
+        }
+        for (; h < Hq; ++h) r[0] = fmaf(expf(lg[int64_t(h) * M] - s_n[2 * h]), s_n[2 * h + 1], r[0]);
+    } else if ((M & 3) == 0) {
         int h = 0;
         for (; h + 8 <= Hq; h += 8) {
             float4 x[8];
@@ -822,31 +841,31 @@ __global__ void __launch_bounds__(256) ads_relevance_kernel(const __grid_constan
             for (int u = 0; u < 8; ++u) {
                 const float mh = s_n[2 * (h + u)], wh = s_n[2 * (h + u) + 1];
                 r[0] = fmaf(expf(x[u].x - mh), wh, r[0]);
-                r[1] = fmaf(expf(x[u].y - mh), wh, r[1]);
-                r[2] = fmaf(expf(x[u].z - mh), wh, r[2]);
-                r[3] = fmaf(expf(x[u].w - mh), wh, r[3]);
+                r[1 % TPT] = fmaf(expf(x[u].y - mh), wh, r[1 % TPT]);
+                r[2 % TPT] = fmaf(expf(x[u].z - mh), wh, r[2 % TPT]);
+                r[3 % TPT] = fmaf(expf(x[u].w - mh), wh, r[3 % TPT]);
             }
         }
         for (; h < Hq; ++h) {
             const float4 x = *reinterpret_cast<const float4*>(lg + int64_t(h) * M);
             const float mh = s_n[2 * h], wh = s_n[2 * h + 1];
             r[0] = fmaf(expf(x.x - mh), wh, r[0]);
-            r[1] = fmaf(expf(x.y - mh), wh, r[1]);
-            r[2] = fmaf(expf(x.z - mh), wh, r[2]);
-            r[3] = fmaf(expf(x.w - mh), wh, r[3]);
+            r[1 % TPT] = fmaf(expf(x.y - mh), wh, r[1 % TPT]);
+            r[2 % TPT] = fmaf(expf(x.z - mh), wh, r[2 % TPT]);
+            r[3 % TPT] = fmaf(expf(x.w - mh), wh, r[3 % TPT]);
         }
     } else {
-        const int n = min(4, M - m);
+        const int n = min(TPT, M - m);
         for (int h = 0; h < Hq; ++h) {
             const float mh = s_n[2 * h], wh = s_n[2 * h + 1];
 #pragma unroll
-            for (int u = 0; u < 4; ++u)
+            for (int u = 0; u < TPT; ++u)
                 if (u < n) r[u] = fmaf(expf(lg[int64_t(h) * M + u] - mh), wh, r[u]);
         }
     }
-    const int n = min(4, M - m);
+    const int n = min(TPT, M - m);
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < TPT; ++u) {
         if (u < n) {
             a.rel[int64_t(b) * M + m + u] = r[u];
             if (a.score_out) a.score_out[int64_t(b) * M + m + u] = r[u];
@@ -1058,8 +1077,13 @@ static cudaError_t launch_select_tail(const SelectArgs& a, int n_seqs, cudaStrea
     cudaError_t e = launch_pdl(norm_from_logits ? ads_norm_logits_kernel : ads_norm_kernel,
                                dim3(a.n_q_heads, n_seqs, 1), dim3(256), 0, stream, a);
     if (e != cudaSuccess) return e;
-    e = launch_pdl(ads_relevance_kernel, dim3((a.n_tokens + 1023) / 1024, n_seqs, 1), dim3(256), 0,
-                   stream, a);
+    // four tokens per thread once the grid fills the GPU a few times over
+    if (int64_t(n_seqs) * a.n_tokens >= (int64_t(1) << 19))
+        e = launch_pdl(ads_relevance_kernel<4>, dim3((a.n_tokens + 1023) / 1024, n_seqs, 1), dim3(256),
+                       0, stream, a);
+    else
+        e = launch_pdl(ads_relevance_kernel<1>, dim3((a.n_tokens + 255) / 256, n_seqs, 1), dim3(256), 0,
+                       stream, a);
     if (e != cudaSuccess) return e;
     const int M = a.n_tokens;
     // just enough warps for PER tokens per thread: fewer warps, cheaper rounds
