@@ -313,16 +313,32 @@ __global__ void __launch_bounds__(NW * 32, 2) ads_logits_mma_kernel(const __grid
     for (int s = 0; s < KS; ++s)
         axes |= uint32_t(pair_axis(32 * (s / 8) + 8 * tq + s % 8, a.layout, a.sec_t, a.sec_h,
                                    a.sec_w)) << (2 * s);
+    // Schedule: q = total / grid whole items per CTA, a contiguous run. The
+    // R = total - q * grid items left over would make R CTAs run q + 1 items;
+    // when 2 R <= grid they are split instead into halves by KV heads, one
+    // half per CTA, so that no CTA runs more than q + 1/2 items.
     const int64_t total = int64_t(a.n_seqs) * n_khg * n_it;
-    const int64_t i_beg = total * blockIdx.x / gridDim.x, i_end = total * (blockIdx.x + 1) / gridDim.x;
-    int64_t cur_bg = -1;
+    const int64_t G = gridDim.x, q = total / G, R = total - q * G;
+    const bool halves = R > 0 && 2 * R <= G && KPI > 1;
+    const int64_t c = blockIdx.x;
+    const int64_t i_beg = halves ? c * q : total * c / G;
+    const int64_t i_end = halves ? i_beg + q : total * (c + 1) / G;
+    const int n_work = int(i_end - i_beg) + (halves && c < 2 * R ? 1 : 0);
+    int cur_b = -1, cur_kh = -1;
     float4* tr_w = tr_s + warp * KS * 32 + lane;
     const int64_t layer_off = int64_t(a.layer) * a.store_layer_stride + 8 * tq;
 
-    for (int64_t item = i_beg; item < i_end; ++item) {
+    for (int w = 0; w < n_work; ++w) {
+        const bool half = i_beg + w >= i_end;
+        const int64_t item = half ? q * G + c / 2 : i_beg + w;
         const int64_t bg = item / n_it;  // (sequence, KV-head group)
         const int b = int(bg / n_khg), it = int(item - bg * n_it);
-        const int kh_a = int(bg - int64_t(b) * n_khg) * KPI, nkh = min(KPI, H - kh_a);
+        int kh_a = int(bg - int64_t(b) * n_khg) * KPI, nkh = min(KPI, H - kh_a);
+        if (half) {  // the first or second half of the group's KV heads
+            const int h1 = (nkh + 1) / 2;
+            kh_a += (c & 1) ? h1 : 0;
+            nkh = (c & 1) ? nkh - h1 : h1;
+        }
         const int j = it * NW + warp;  // the warp's 16-token tile
         const int m0 = 16 * j, ntw = min(16, M - m0);
         // this lane's two tokens (rows g and g + 8 of the warp's MMA tile); a
@@ -344,11 +360,11 @@ __global__ void __launch_bounds__(NW * 32, 2) ads_logits_mma_kernel(const __grid
             k[2] = ld_stream(rb + off);
             k[3] = ld_stream(rb + off + P);
         };
-        if (ntw > 0) {
+        if (ntw > 0 && n_runs > 0) {
             fetch(buf0, 0);
             if (n_runs > 1) fetch(buf1, 1);
         }
-        if (bg != cur_bg) {
+        if (b != cur_b || kh_a != cur_kh) {
             // the group's raw queries as B fragments (a bf16 value is an exact
             // tf32 operand): entry (kh, s / 2, lane) holds k-steps s and s + 1
             __syncthreads();  // every warp is done with the previous group's
@@ -367,10 +383,11 @@ __global__ void __launch_bounds__(NW * 32, 2) ads_logits_mma_kernel(const __grid
                 }
                 qf_s[e] = f;
             }
-            cur_bg = bg;
+            cur_b = b;
+            cur_kh = kh_a;
             __syncthreads();
         }
-        if (ntw <= 0) continue;  // past the sequence's last token
+        if (ntw <= 0 || nkh <= 0) continue;  // past the sequence's last token, or no KV head
 
         // cos/sin of the lane's (token, pair) at each k-step, at the offsets
         // of the tokens' coordinates from the trigger position
