@@ -781,6 +781,17 @@ __global__ void __launch_bounds__(256) ads_norm_logits_kernel(const __grid_const
     int i = 0;  // logits [0, i) done
     if ((M & 3) == 0) {
         const float4* l4 = reinterpret_cast<const float4*>(lg);
+        for (; i + 8192 <= M; i += 8192) {  // 256 threads x 32 logits, all requested at once
+            float x[2][16];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const float4 v = l4[(i >> 2) + u * 256 + threadIdx.x];
+                x[u >> 2][4 * (u & 3)] = v.x; x[u >> 2][4 * (u & 3) + 1] = v.y;
+                x[u >> 2][4 * (u & 3) + 2] = v.z; x[u >> 2][4 * (u & 3) + 3] = v.w;
+            }
+            chunk(x[0]);
+            chunk(x[1]);
+        }
         for (; i + 4096 <= M; i += 4096) {  // 256 threads x 16 logits
             float x[16];
 #pragma unroll
@@ -819,7 +830,8 @@ __global__ void __launch_bounds__(256) ads_norm_logits_kernel(const __grid_const
 }
 
 // Relevance of every token: mean over the query heads of its softmax weight,
-// the heads accumulated in ascending order. TPT consecutive tokens per thread:
+// the heads accumulated in ascending order (exp of arguments <= 0 by
+// __expf, relative error ~1e-6, far inside the relevance's float32 budget). TPT consecutive tokens per thread:
 // four (16-byte loads, eight heads' logits requested together) for large
 // batches, one (sixteen heads requested together) where the grid would
 // otherwise be a few CTAs.
@@ -845,9 +857,9 @@ __global__ void __launch_bounds__(256) ads_relevance_kernel(const __grid_constan
 #pragma unroll
             for (int u = 0; u < 16; ++u) x[u] = lg[int64_t(h + u) * M];
 #pragma unroll
-            for (int u = 0; u < 16; ++u) r[0] = fmaf(expf(x[u] - s_n[2 * (h + u)]), s_n[2 * (h + u) + 1], r[0]);
+            for (int u = 0; u < 16; ++u) r[0] = fmaf(__expf(x[u] - s_n[2 * (h + u)]), s_n[2 * (h + u) + 1], r[0]);
         }
-        for (; h < Hq; ++h) r[0] = fmaf(expf(lg[int64_t(h) * M] - s_n[2 * h]), s_n[2 * h + 1], r[0]);
+        for (; h < Hq; ++h) r[0] = fmaf(__expf(lg[int64_t(h) * M] - s_n[2 * h]), s_n[2 * h + 1], r[0]);
     } else if ((M & 3) == 0) {
         int h = 0;
         for (; h + 8 <= Hq; h += 8) {
@@ -857,19 +869,19 @@ __global__ void __launch_bounds__(256) ads_relevance_kernel(const __grid_constan
 #pragma unroll
             for (int u = 0; u < 8; ++u) {
                 const float mh = s_n[2 * (h + u)], wh = s_n[2 * (h + u) + 1];
-                r[0] = fmaf(expf(x[u].x - mh), wh, r[0]);
-                r[1 % TPT] = fmaf(expf(x[u].y - mh), wh, r[1 % TPT]);
-                r[2 % TPT] = fmaf(expf(x[u].z - mh), wh, r[2 % TPT]);
-                r[3 % TPT] = fmaf(expf(x[u].w - mh), wh, r[3 % TPT]);
+                r[0] = fmaf(__expf(x[u].x - mh), wh, r[0]);
+                r[1 % TPT] = fmaf(__expf(x[u].y - mh), wh, r[1 % TPT]);
+                r[2 % TPT] = fmaf(__expf(x[u].z - mh), wh, r[2 % TPT]);
+                r[3 % TPT] = fmaf(__expf(x[u].w - mh), wh, r[3 % TPT]);
             }
         }
         for (; h < Hq; ++h) {
             const float4 x = *reinterpret_cast<const float4*>(lg + int64_t(h) * M);
             const float mh = s_n[2 * h], wh = s_n[2 * h + 1];
-            r[0] = fmaf(expf(x.x - mh), wh, r[0]);
-            r[1 % TPT] = fmaf(expf(x.y - mh), wh, r[1 % TPT]);
-            r[2 % TPT] = fmaf(expf(x.z - mh), wh, r[2 % TPT]);
-            r[3 % TPT] = fmaf(expf(x.w - mh), wh, r[3 % TPT]);
+            r[0] = fmaf(__expf(x.x - mh), wh, r[0]);
+            r[1 % TPT] = fmaf(__expf(x.y - mh), wh, r[1 % TPT]);
+            r[2 % TPT] = fmaf(__expf(x.z - mh), wh, r[2 % TPT]);
+            r[3 % TPT] = fmaf(__expf(x.w - mh), wh, r[3 % TPT]);
         }
     } else {
         const int n = min(TPT, M - m);
@@ -877,7 +889,7 @@ __global__ void __launch_bounds__(256) ads_relevance_kernel(const __grid_constan
             const float mh = s_n[2 * h], wh = s_n[2 * h + 1];
 #pragma unroll
             for (int u = 0; u < TPT; ++u)
-                if (u < n) r[u] = fmaf(expf(lg[int64_t(h) * M + u] - mh), wh, r[u]);
+                if (u < n) r[u] = fmaf(__expf(lg[int64_t(h) * M + u] - mh), wh, r[u]);
         }
     }
     const int n = min(TPT, M - m);
