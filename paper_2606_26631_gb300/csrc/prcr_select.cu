@@ -353,16 +353,20 @@ __global__ void __launch_bounds__(NW * 32, 2) ads_logits_mma_kernel(const __grid
         // run r = (KV head kh_a + r / NR, 16-byte run r % NR): first-half x and
         // second-half y words of tokens a and b
         uint4 buf0[4], buf1[4];
-        auto fetch = [&](uint4 (&k)[4], int r) {
-            const int off = (kh_a + r / NR) * D + 32 * (r % NR);
-            k[0] = ld_stream(ra + off);
-            k[1] = ld_stream(ra + off + P);
-            k[2] = ld_stream(rb + off);
-            k[3] = ld_stream(rb + off + P);
+        // run u of the KV head whose rows start at pa (token a) and pb (token
+        // b): compile-time offsets from two pointers advanced by D per head
+        const uint16_t* pa = ra + kh_a * D;
+        const uint16_t* pb = rb + kh_a * D;
+        auto fetch = [&](uint4 (&k)[4], const uint16_t* xa, const uint16_t* xb, int u) {
+            k[0] = ld_stream(xa + 32 * u);
+            k[1] = ld_stream(xa + 32 * u + P);
+            k[2] = ld_stream(xb + 32 * u);
+            k[3] = ld_stream(xb + 32 * u + P);
         };
         if (ntw > 0 && n_runs > 0) {
-            fetch(buf0, 0);
-            if (n_runs > 1) fetch(buf1, 1);
+            fetch(buf0, pa, pb, 0);
+            if (NR == 2) fetch(buf1, pa, pb, 1);
+            else if (n_runs > 1) fetch(buf1, pa + D, pb + D, 0);
         }
         if (b != cur_b || kh_a != cur_kh) {
             // the group's raw queries as B fragments (a bf16 value is an exact
@@ -450,9 +454,11 @@ __global__ void __launch_bounds__(NW * 32, 2) ads_logits_mma_kernel(const __grid
         // KV head kk done: its logits out (the softmax statistics come from
         // the normaliser kernel, one pass over the logits)
         const bool va = ta < ntw, vb = tb < ntw;
-        auto finish = [&](int kk) {
-            const int h0 = 2 * tq;  // columns 2t, 2t + 1
-            float* lg = a.logits + (int64_t(b) * Hq + (kh_a + kk) * g + h0) * M + m0;
+        // columns 2t, 2t + 1 of each KV head's logits; lg advances by g rows per head
+        const int h0 = 2 * tq;
+        float* lg = a.logits + (int64_t(b) * Hq + kh_a * g + h0) * M + m0;
+        const int64_t lg_step = int64_t(g) * M;
+        auto finish = [&]() {
 #pragma unroll
             for (int c = 0; c < 2; ++c) {
                 if (h0 + c < g) {
@@ -460,17 +466,34 @@ __global__ void __launch_bounds__(NW * 32, 2) ads_logits_mma_kernel(const __grid
                     if (vb) lg[int64_t(c) * M + tb] = acc[2 + c] * a.scale;
                 }
             }
+            lg += lg_step;
             clear();
         };
-        // run r in buffer r % 2; once its words are used, run r + 2 is requested into it
-        for (int r = 0; r < n_runs; r += 2) {
-            run(buf0, r / NR, r % NR);
-            if (NR == 1) finish(r);
-            if (r + 2 < n_runs) fetch(buf0, r + 2);
-            if (r + 1 < n_runs) {
-                run(buf1, (r + 1) / NR, (r + 1) % NR);
-                finish((r + 1) / NR);
-                if (r + 3 < n_runs) fetch(buf1, r + 3);
+        // Each buffer's next run is requested as soon as its words are used:
+        // head dim 128, buffer u holds run u of the current KV head; head dim
+        // 64 (one run per head), buffers take alternate heads.
+        if (NR == 2) {
+            for (int kk = 0; kk < nkh; ++kk) {
+                run(buf0, kk, 0);
+                pa += D;
+                pb += D;
+                if (kk + 1 < nkh) fetch(buf0, pa, pb, 0);
+                run(buf1, kk, 1);
+                finish();
+                if (kk + 1 < nkh) fetch(buf1, pa, pb, 1);
+            }
+        } else {
+            for (int kk = 0; kk < nkh; kk += 2) {
+                run(buf0, kk, 0);
+                finish();
+                if (kk + 2 < nkh) fetch(buf0, pa + 2 * D, pb + 2 * D, 0);
+                if (kk + 1 < nkh) {
+                    run(buf1, kk + 1, 0);
+                    finish();
+                    if (kk + 3 < nkh) fetch(buf1, pa + 3 * D, pb + 3 * D, 0);
+                }
+                pa += 2 * D;
+                pb += 2 * D;
             }
         }
     }
