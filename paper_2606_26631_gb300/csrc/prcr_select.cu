@@ -303,9 +303,15 @@ __global__ void __launch_bounds__(NW * 32, 2) ads_logits_mma_kernel(const __grid
     uint4* qf_s = reinterpret_cast<uint4*>(sm);  // [KPI][KS / 2][32] B fragments
     float4* tr_s = reinterpret_cast<float4*>(qf_s + KPI * (KS / 2) * 32);  // [NW][KS][32]
     uint64_t* tf_s = reinterpret_cast<uint64_t*>(tr_s + NW * KS * 32);      // [P] turn rates
+    float2* r8_s = reinterpret_cast<float2*>(tf_s + P);  // [P] turn of 8 w-steps; (1, 0) off the w band
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int gid = lane >> 2, tq = lane & 3;
-    for (int i = tid; i < P; i += NW * 32) tf_s[i] = a.turn_freq[i];
+    for (int i = tid; i < P; i += NW * 32) {
+        tf_s[i] = a.turn_freq[i];
+        float2 r = make_float2(1.0f, 0.0f);
+        if (pair_axis(i, a.layout, a.sec_t, a.sec_h, a.sec_w) == 2) sincos_coord(8, a.turn_freq[i], &r.y, &r.x);
+        r8_s[i] = r;
+    }
     __syncthreads();
     // axis of this lane's pair at each k-step, two bits each
     uint32_t axes = 0u;
@@ -398,16 +404,35 @@ __global__ void __launch_bounds__(NW * 32, 2) ads_logits_mma_kernel(const __grid
         {
             const int32_t* crd = a.coords + int64_t(b) * a.coord_seq_stride;
             const int64_t p = a.q_pos[b];
-            const int64_t oa[3] = {crd[3 * ma] - p, crd[3 * ma + 1] - p, crd[3 * ma + 2] - p};
-            const int64_t ob[3] = {crd[3 * mb] - p, crd[3 * mb + 1] - p, crd[3 * mb + 2] - p};
+            const int ca[3] = {crd[3 * ma], crd[3 * ma + 1], crd[3 * ma + 2]};
+            const int cb[3] = {crd[3 * mb], crd[3 * mb + 1], crd[3 * mb + 2]};
+            const int64_t oa[3] = {ca[0] - p, ca[1] - p, ca[2] - p};
+            // Every lane's two tokens on one image row, 8 columns apart (a
+            // 16-token tile within a row): token b's angles are token a's
+            // turned by 8 w-steps on the w pairs and equal on the others.
+            const bool row8 = __all_sync(0xffffffffu, cb[0] == ca[0] && cb[1] == ca[1] &&
+                                                          int64_t(cb[2]) == int64_t(ca[2]) + 8);
+            if (row8) {
 #pragma unroll
-            for (int s = 0; s < KS; ++s) {
-                const uint32_t ax = (axes >> (2 * s)) & 3u;
-                const uint64_t rate = tf_s[32 * (s / 8) + 8 * tq + s % 8];
-                float4 t;
-                sincos_coord(ax == 0 ? oa[0] : (ax == 1 ? oa[1] : oa[2]), rate, &t.z, &t.x);
-                sincos_coord(ax == 0 ? ob[0] : (ax == 1 ? ob[1] : ob[2]), rate, &t.w, &t.y);
-                tr_w[s * 32] = t;
+                for (int s = 0; s < KS; ++s) {
+                    const uint32_t ax = (axes >> (2 * s)) & 3u;
+                    const int i = 32 * (s / 8) + 8 * tq + s % 8;
+                    float sn, cs;
+                    sincos_coord(ax == 0 ? oa[0] : (ax == 1 ? oa[1] : oa[2]), tf_s[i], &sn, &cs);
+                    const float2 r = r8_s[i];
+                    tr_w[s * 32] = make_float4(cs, fmaf(cs, r.x, -sn * r.y), sn, fmaf(sn, r.x, cs * r.y));
+                }
+            } else {
+                const int64_t ob[3] = {cb[0] - p, cb[1] - p, cb[2] - p};
+#pragma unroll
+                for (int s = 0; s < KS; ++s) {
+                    const uint32_t ax = (axes >> (2 * s)) & 3u;
+                    const uint64_t rate = tf_s[32 * (s / 8) + 8 * tq + s % 8];
+                    float4 t;
+                    sincos_coord(ax == 0 ? oa[0] : (ax == 1 ? oa[1] : oa[2]), rate, &t.z, &t.x);
+                    sincos_coord(ax == 0 ? ob[0] : (ax == 1 ? ob[1] : ob[2]), rate, &t.w, &t.y);
+                    tr_w[s * 32] = t;
+                }
             }
         }
         __syncwarp();
@@ -1095,7 +1120,7 @@ constexpr int kMmaWarps = 8;  // warps per CTA of the tensor-core logits kernel 
 template <int D>
 size_t logits_mma_smem(int kpi) {
     return size_t(kpi) * (D / 16) * 32 * 16 + size_t(kMmaWarps) * (D / 8) * 32 * 16 +
-           size_t(D / 2) * 8;
+           size_t(D / 2) * 16;
 }
 
 template <int D>
