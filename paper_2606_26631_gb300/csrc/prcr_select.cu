@@ -538,8 +538,9 @@ __global__ void __launch_bounds__(NW * 32, 2) ads_logits_mma_kernel(const __grid
 // permuted per lane group so that a lane loads its two tokens' 64 contiguous
 // bytes each straight into A fragments. The next item's rows are loaded
 // right after this item's MMAs, the rows of the one after that requested
-// into L2. An item writes its 16 logits per head and the tile's (max, sum of
-// exp) per head; a token without a readable row gets logit -inf.
+// into L2. An item writes its 16 logits per head (the softmax statistics
+// are left to the normaliser kernel); a token without a readable row gets
+// logit -inf.
 template <int D>
 __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
     ads_logits_cache_kernel(const __grid_constant__ SelectArgs a) {
@@ -634,7 +635,6 @@ __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
 
     uint32_t qh[KS][2], ql[KS][2];
     float* lg_base[2] = {nullptr, nullptr};
-    float* ts_base[2] = {nullptr, nullptr};
     int cur_b = -1, cur_kh = -1;
     bool q_ok = true;  // the sequence's query position is within the angle range
     Item cur, nxt, pf;
@@ -691,7 +691,6 @@ __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
             for (int hh = 0; hh < 2; ++hh) {  // rows of this lane's heads 2t, 2t + 1
                 const int64_t r = int64_t(b) * Hq + kh * g + min(2 * t + hh, g - 1);
                 lg_base[hh] = a.logits + r * M;
-                ts_base[hh] = a.tile_stats + r * NT * 2;
             }
         }
         // S^T (16 tokens x 8 columns = the group's query heads, columns >= g
@@ -715,25 +714,11 @@ __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
         }
 
         // token gid: heads 2t, 2t + 1 in c[0], c[1]; token gid + 8 in c[2], c[3]
+        // (the softmax statistics come from the normaliser kernel, one pass
+        // over the logits)
         const bool ok0 = (mask >> gid) & 1u, ok1 = (mask >> (gid + 8)) & 1u;
         float v[4] = {ok0 ? c[0] : -INFINITY, ok0 ? c[1] : -INFINITY, ok1 ? c[2] : -INFINITY,
                       ok1 ? c[3] : -INFINITY};
-        // per head (column): max and sum of exp over the 16 tokens (the eight
-        // lanes of one t hold them)
-        float mx0 = fmaxf(v[0], v[2]), mx1 = fmaxf(v[1], v[3]);
-#pragma unroll
-        for (int o = 4; o < 32; o <<= 1) {
-            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
-            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
-        }
-        // arguments <= 0: __expf's few-ulp error is far below the relevance bar
-        float z0 = (v[0] == -INFINITY ? 0.0f : __expf(v[0] - mx0)) + (v[2] == -INFINITY ? 0.0f : __expf(v[2] - mx0));
-        float z1 = (v[1] == -INFINITY ? 0.0f : __expf(v[1] - mx1)) + (v[3] == -INFINITY ? 0.0f : __expf(v[3] - mx1));
-#pragma unroll
-        for (int o = 4; o < 32; o <<= 1) {
-            z0 += __shfl_xor_sync(0xffffffffu, z0, o);
-            z1 += __shfl_xor_sync(0xffffffffu, z1, o);
-        }
         const int m0 = 16 * j;
         const bool full = m0 + 16 <= M;
 #pragma unroll
@@ -746,12 +731,6 @@ __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
             } else {
                 if (m0 + gid < M) lg[gid] = v[hh];
                 if (m0 + gid + 8 < M) lg[gid + 8] = v[2 + hh];
-            }
-            if (gid == 0) {
-                const float mxh = hh ? mx1 : mx0;
-                float* ts = ts_base[hh] + 2 * j;
-                ts[0] = mxh;
-                ts[1] = mxh == -INFINITY ? 0.0f : (hh ? z1 : z0);
             }
         }
         cur = nxt;
@@ -1204,7 +1183,7 @@ cudaError_t launch_select_cached(const SelectArgs& a, int n_seqs, int sms, cudaS
     const int64_t resident = int64_t(sms) * (per_sm > 0 ? per_sm : 1);
     e = launch_pdl(k, dim3(unsigned(ctas < resident ? ctas : resident)), dim3(256), smem, stream, a);
     if (e != cudaSuccess) return e;
-    return launch_select_tail(a, n_seqs, stream);
+    return launch_select_tail(a, n_seqs, stream, true);
 }
 
 }  // namespace prcr
