@@ -595,24 +595,40 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
 // Small batches (a grid that would not fill the GPU a few times over): a CTA
 // of kRingWarps warps takes one (sequence, layer, chunk) and up to kRingWarps
 // KV heads, one per warp, and the chunk is sized so that the grid runs as
-// about one wave. Each warp streams its chunk's tiles of 16 slots through a
-// ring of kRingStages stages in shared memory: K and V are both staged by
-// cp.async, kRingStages - 1 tiles ahead of the one being computed, and the
-// first of them are requested before the prologue's barriers (a barrier
-// waits for a thread's plain loads in flight, not for its async copies). The
-// arithmetic is that of decode_mma_kernel (same QK and PV on tensor cores,
-// same online softmax); the key dimensions are permuted per lane group the
-// same way, here with lane group t reading 16-byte chunks t, t + 4, ... of its
-// slot's K row, and chunk c of slot s is stored at c ^ 4 (s & 1) so that
-// those reads are free of bank conflicts.
+// about one wave of kDecodeRingCtasPerSm CTAs per SM. Each warp streams its
+// chunk's tiles of 16 slots through a ring of kRingStages stages in shared
+// memory: K and V are both staged by cp.async, kRingStages - 1 tiles ahead
+// of the one being computed, and the first of them are requested before the
+// prologue's barriers (a barrier waits for a thread's plain loads in flight,
+// not for its async copies). Two stages keep the CTA's shared memory at
+// 66 KB (three CTAs, twelve warps per SM); more warps per SM hide more of
+// each warp's latency chain than a deeper ring would.
+// QK is S^T = K Q^T (the tile's 16 slots as the MMA rows, the GQA group's
+// query heads as the 8 columns: one MMA per k-step and query piece, half of
+// what Q K^T with the heads as rows takes), and PV is O^T += V^T P^T as in
+// decode_mma_kernel, P^T's fragments transposed from S^T's in registers
+// (movmatrix); each lane keeps the online-softmax state of the two heads
+// whose O^T columns it holds. The key dimensions are permuted per lane group
+// as in decode_mma_kernel, here with lane group t reading 16-byte chunks t,
+// t + 4, ... of its slot's K row, and chunk c of slot s is stored at
+// c ^ 4 (s & 1) so that those reads are free of bank conflicts.
+// Transpose of an 8 x 8 matrix of 16-bit values held as mma fragments
+// (lane 4 r + c holds row r, columns 2c and 2c + 1): afterwards the lane holds
+// row r, columns 2c and 2c + 1 of the transpose.
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x) {
+    uint32_t y;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+    return y;
+}
+
 constexpr int kRingWarps = kDecodeRingWarps;
-constexpr int kRingStages = 3;
+constexpr int kRingStages = 2;
 // rounds of eight query pairs per thread: the CTA's query heads are at most
 // kRingWarps * 8 (a GQA group of 8), i.e. kRingWarps * 8 * D / 2 pairs
 constexpr int kRingQRounds = 2;
 
 template <int D>
-__global__ void __launch_bounds__(kRingWarps * 32, 2)
+__global__ void __launch_bounds__(kRingWarps * 32, kDecodeRingCtasPerSm)
     decode_ring_kernel(const __grid_constant__ DecodeArgs a) {
     constexpr int KS = D / 16;      // k-steps of QK, m-tiles of PV
     constexpr int LV = D / 32;      // 16-byte K chunks per lane per slot
@@ -635,17 +651,22 @@ __global__ void __launch_bounds__(kRingWarps * 32, 2)
     const int kh0 = (int(blockIdx.x) - split * n_hg) * kRingWarps;
     const int kh1 = min(H, kh0 + kRingWarps);
     const int nq = (kh1 - kh0) * g;  // this CTA's query heads
-    float* q_s = reinterpret_cast<float*>(smem_raw);  // [nq][D], rotated and scaled
-    uint16_t* ring = reinterpret_cast<uint16_t*>(smem_raw + size_t(kRingWarps) * g * D * sizeof(float));
+    // the ring, stage-major: stage st of warp w holds a K tile then a V tile
+    // at ring + (st * kRingWarps + w) * (KT + VT); the rotated queries
+    // ([nq][D] float32, needed only until every warp holds its fragments)
+    // share the last stage, which is first filled after that
+    uint16_t* ring = reinterpret_cast<uint16_t*>(smem_raw);
+    float* q_s = reinterpret_cast<float*>(ring + size_t(NS - 1) * kRingWarps * (KT + VT));
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int gid = lane >> 2;
     const int t = lane & 3;
     const int kh = kh0 + warp;
     const bool wact = kh < kh1;
-    const uint16_t* wk = ring + size_t(warp) * NS * (KT + VT);  // NS K stages, then NS V stages
+    const uint16_t* wk = ring + size_t(warp) * (KT + VT);  // this warp's stage 0
     const uint32_t wk_s = uint32_t(__cvta_generic_to_shared(wk));
-    const uint32_t wv_s = wk_s + uint32_t(NS * KT * 2);
+    const uint32_t wv_s = wk_s + uint32_t(KT * 2);
+    constexpr uint32_t kStageBytes = uint32_t(kRingWarps * (KT + VT) * 2);  // one stage of all warps
     uint32_t err = 0;
     pdl_allow();
     {
@@ -729,8 +750,8 @@ __global__ void __launch_bounds__(kRingWarps * 32, 2)
             }
             const uint32_t m = __ballot_sync(kFull, row >= 0) & 0xffffu;
             if (lane == 0) s_mask[warp][st] = m;
-            const uint32_t ks_ = wk_s + uint32_t(st * KT * 2);
-            const uint32_t vs_ = wv_s + uint32_t(st * VT * 2);
+            const uint32_t ks_ = wk_s + uint32_t(st) * kStageBytes;
+            const uint32_t vs_ = wv_s + uint32_t(st) * kStageBytes;
 #pragma unroll
             for (int i = 0; i < (16 * NCH) / 32; ++i) {
                 const int c = lane + 32 * i;
@@ -787,27 +808,29 @@ __global__ void __launch_bounds__(kRingWarps * 32, 2)
     }
     __syncthreads();
 
-    if (wact) {
-        // Q A-fragments (rows = heads of the group; rows >= g and 8..15 are
-        // zero); k-step j of lane group t covers dimensions
-        // 8 (t + 4 (j / 2)) + 4 (j % 2) + 0..3, as the K chunks it reads
-        uint32_t qh[KS][2], ql[KS][2];
-        {
-            const bool hv = gid < g;
-            const float* qr = q_s + ((kh - kh0) * g + (hv ? gid : 0)) * D;
+    // the query B fragments (columns = heads of the group; columns >= g are
+    // zero); k-step j of lane group t covers dimensions
+    // 8 (t + 4 (j / 2)) + 4 (j % 2) + 0..3, as the K chunks it reads
+    uint32_t qh[KS][2], ql[KS][2];
+    {
+        const bool hv = wact && gid < g;
+        const float* qr = q_s + (hv ? (kh - kh0) * g + gid : 0) * D;
 #pragma unroll
-            for (int j = 0; j < KS; ++j) {
-                const int base = 8 * (t + 4 * (j >> 1)) + 4 * (j & 1);
-                const float x0 = hv ? qr[base] : 0.0f, x1 = hv ? qr[base + 1] : 0.0f;
-                const float x2 = hv ? qr[base + 2] : 0.0f, x3 = hv ? qr[base + 3] : 0.0f;
-                split_bf16x2(x0, x1, qh[j][0], ql[j][0]);
-                split_bf16x2(x2, x3, qh[j][1], ql[j][1]);
-            }
+        for (int j = 0; j < KS; ++j) {
+            const int base = 8 * (t + 4 * (j >> 1)) + 4 * (j & 1);
+            const float x0 = hv ? qr[base] : 0.0f, x1 = hv ? qr[base + 1] : 0.0f;
+            const float x2 = hv ? qr[base + 2] : 0.0f, x3 = hv ? qr[base + 3] : 0.0f;
+            split_bf16x2(x0, x1, qh[j][0], ql[j][0]);
+            split_bf16x2(x2, x3, qh[j][1], ql[j][1]);
         }
+    }
+    __syncthreads();  // the queries' stage may now be filled
+
+    if (wact) {
         float o[KS][4];
 #pragma unroll
         for (int mt = 0; mt < KS; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.0f;
-        float m_run = -INFINITY, l_run = 0.0f;
+        float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.0f, 0.0f};  // heads 2t, 2t + 1
         const int lslot = (lane & 7) + ((lane >> 4) & 1) * 8;
         const int ldim = ((lane >> 3) & 1) * 8;
 
@@ -825,11 +848,11 @@ __global__ void __launch_bounds__(kRingWarps * 32, 2)
             }
             const uint32_t mask = s_mask[warp][st];
 
-            // S = Q K^T for the two slot tiles (slots gid and 8 + gid)
-            const uint16_t* kt = wk + st * KT;
-            // four independent accumulation chains (two slot tiles x the
-            // query's head and remainder), summed at the end
-            float sc[2][4], sl_[2][4];
+            const uint16_t* kt = wk + size_t(st) * kRingWarps * (KT + VT);
+            // S^T (16 slots x 8 columns = the group's query heads, columns >= g
+            // zero) = K Q^T: this lane's slots gid (kv[0]) and 8 + gid (kv[1])
+            // are the A rows, the query fragments the B operand unchanged; the
+            // query's head and remainder products in two chains
             uint4 kv[2][LV];
 #pragma unroll
             for (int nt = 0; nt < 2; ++nt) {
@@ -837,66 +860,61 @@ __global__ void __launch_bounds__(kRingWarps * 32, 2)
 #pragma unroll
                 for (int u = 0; u < LV; ++u)
                     kv[nt][u] = *reinterpret_cast<const uint4*>(kt + slot * D + (((t + 4 * u) ^ ((slot & 1) << 2)) * 8));
-                sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.0f;
-                sl_[nt][0] = sl_[nt][1] = sl_[nt][2] = sl_[nt][3] = 0.0f;
             }
+            float sh[4] = {0.0f, 0.0f, 0.0f, 0.0f}, sl_[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
             for (int j = 0; j < KS; ++j) {
-#pragma unroll
-                for (int nt = 0; nt < 2; ++nt) {
-                    const uint4& w = kv[nt][j >> 1];
-                    const uint32_t b0 = (j & 1) ? w.z : w.x;
-                    const uint32_t b1 = (j & 1) ? w.w : w.y;
-                    mma_16816(sc[nt], qh[j][0], 0u, qh[j][1], 0u, b0, b1);
-                    mma_16816(sl_[nt], ql[j][0], 0u, ql[j][1], 0u, b0, b1);
-                }
+                const uint4& w0 = kv[0][j >> 1];
+                const uint4& w1 = kv[1][j >> 1];
+                const uint32_t a0 = (j & 1) ? w0.z : w0.x, a2 = (j & 1) ? w0.w : w0.y;
+                const uint32_t a1 = (j & 1) ? w1.z : w1.x, a3 = (j & 1) ? w1.w : w1.y;
+                mma_16816(sh, a0, a1, a2, a3, qh[j][0], qh[j][1]);
+                mma_16816(sl_, a0, a1, a2, a3, ql[j][0], ql[j][1]);
             }
-#pragma unroll
-            for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-                for (int r = 0; r < 4; ++r) sc[nt][r] += sl_[nt][r];
 
-            // online softmax of head row gid over the 16 slots
-            float v[4] = {sc[0][0], sc[0][1], sc[1][0], sc[1][1]};
-            const int sl[4] = {2 * t, 2 * t + 1, 8 + 2 * t, 9 + 2 * t};
-            float mx = -INFINITY;
+            // online softmax of this lane's heads 2t, 2t + 1 (columns) over the
+            // 16 slots: the eight lanes of one t hold them, two slots each
+            const bool oka = (mask >> gid) & 1u, okb = (mask >> (8 + gid)) & 1u;
+            float pa[2], pb[2], alpha[2];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                if (!((mask >> sl[i]) & 1u)) v[i] = -INFINITY;
-                mx = fmaxf(mx, v[i]);
+            for (int hh = 0; hh < 2; ++hh) {
+                const float va = oka ? sh[hh] + sl_[hh] : -INFINITY;
+                const float vb = okb ? sh[2 + hh] + sl_[2 + hh] : -INFINITY;
+                float mx = fmaxf(va, vb);
+                mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 4));
+                mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 8));
+                mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 16));
+                const float m_new = fmaxf(m_run[hh], mx);
+                // arguments are <= 0: __expf's error (a few ulp) is far inside
+                // the float32 accumulation's
+                alpha[hh] = m_new == -INFINITY ? 1.0f : __expf(m_run[hh] - m_new);
+                pa[hh] = va == -INFINITY ? 0.0f : __expf(va - m_new);
+                pb[hh] = vb == -INFINITY ? 0.0f : __expf(vb - m_new);
+                float ps = pa[hh] + pb[hh];
+                ps += __shfl_xor_sync(kFull, ps, 4);
+                ps += __shfl_xor_sync(kFull, ps, 8);
+                ps += __shfl_xor_sync(kFull, ps, 16);
+                l_run[hh] = l_run[hh] * alpha[hh] + ps;
+                m_run[hh] = m_new;
             }
-            mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 1));
-            mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 2));
-            const float m_new = fmaxf(m_run, mx);
-            // arguments are <= 0: __expf's error (a few ulp) is far inside
-            // the float32 accumulation's
-            const float alpha = m_new == -INFINITY ? 1.0f : __expf(m_run - m_new);
-            float ps = 0.0f;
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                v[i] = v[i] == -INFINITY ? 0.0f : __expf(v[i] - m_new);
-                ps += v[i];
-            }
-            ps += __shfl_xor_sync(kFull, ps, 1);
-            ps += __shfl_xor_sync(kFull, ps, 2);
-            l_run = l_run * alpha + ps;
-            m_run = m_new;
-            // O^T columns are heads 2t, 2t+1: their rescale factors live in rows 2t, 2t+1
-            const float a0 = __shfl_sync(kFull, alpha, (2 * t) * 4);
-            const float a1 = __shfl_sync(kFull, alpha, (2 * t + 1) * 4);
+            // O^T columns are heads 2t, 2t + 1: this lane's own factors
 #pragma unroll
             for (int mt = 0; mt < KS; ++mt) {
-                o[mt][0] *= a0; o[mt][1] *= a1; o[mt][2] *= a0; o[mt][3] *= a1;
+                o[mt][0] *= alpha[0]; o[mt][1] *= alpha[1]; o[mt][2] *= alpha[0]; o[mt][3] *= alpha[1];
             }
-            uint32_t pb0h, pb0l, pb1h, pb1l;
-            split_bf16x2(v[0], v[1], pb0h, pb0l);
-            split_bf16x2(v[2], v[3], pb1h, pb1l);
+            // P^T as B fragments: the 8 x 8 blocks (slots 0..7 | 8..15) x heads
+            // held as (slot gid; heads 2t, 2t + 1) are transposed in registers
+            uint32_t m1h, m1l, m2h, m2l;
+            split_bf16x2(pa[0], pa[1], m1h, m1l);
+            split_bf16x2(pb[0], pb[1], m2h, m2l);
+            const uint32_t pb0h = movmatrix_trans(m1h), pb1h = movmatrix_trans(m2h);
+            const uint32_t pb0l = movmatrix_trans(m1l), pb1l = movmatrix_trans(m2l);
 
             // O^T += V^T P^T
 #pragma unroll
             for (int mt = 0; mt < KS; ++mt) {
                 uint32_t r0, r1, r2, r3;
-                const uint32_t addr = wv_s + uint32_t((st * VT + lslot * PITCH + mt * 16 + ldim) * 2);
+                const uint32_t addr = wv_s + uint32_t(st) * kStageBytes + uint32_t((lslot * PITCH + mt * 16 + ldim) * 2);
                 asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
                              : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
                              : "r"(addr));
@@ -907,10 +925,7 @@ __global__ void __launch_bounds__(kRingWarps * 32, 2)
         }
 
         // heads 2t, 2t+1 of this lane's O^T columns
-        const float l0 = __shfl_sync(kFull, l_run, (2 * t) * 4);
-        const float l1 = __shfl_sync(kFull, l_run, (2 * t + 1) * 4);
-        const float m0 = __shfl_sync(kFull, m_run, (2 * t) * 4);
-        const float m1 = __shfl_sync(kFull, m_run, (2 * t + 1) * 4);
+        const float l0 = l_run[0], l1 = l_run[1], m0 = m_run[0], m1 = m_run[1];
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
             const int h = 2 * t + hh;
@@ -1074,8 +1089,11 @@ cudaError_t launch_decode(const DecodeArgs& a, int gp, dim3 grid, size_t smem,
         // shared-memory ring per warp
         const int n_hg = (a.n_kv_heads + kRingWarps - 1) / kRingWarps;
         const int D = a.head_dim;
-        const size_t sm = size_t(kRingWarps) * a.group * D * sizeof(float) +
-                          size_t(kRingWarps) * kRingStages * 16 * (D + D + 8) * sizeof(uint16_t);
+        // the ring (the rotated queries share its last stage)
+        const size_t sm = size_t(kRingWarps) * kRingStages * 16 * (D + D + 8) * sizeof(uint16_t);
+        static_assert(8 * 128 * sizeof(float) <= 16 * (2 * 128 + 8) * sizeof(uint16_t) &&
+                          8 * 64 * sizeof(float) <= 16 * (2 * 64 + 8) * sizeof(uint16_t),
+                      "a GQA group's rotated queries fit in one warp's share of a ring stage");
         dim3 g2 = grid;
         g2.x *= unsigned(n_hg);
         auto k = D == 64 ? decode_ring_kernel<64> : decode_ring_kernel<128>;

@@ -263,7 +263,7 @@ struct DecodeArgs {
 
 constexpr int kDecodeMaxChunk = 4096;
 constexpr int kDecodeRingWarps = 4;   // KV heads (one per warp) per CTA of the ring kernel
-constexpr int kDecodeRingCtasPerSm = 2;
+constexpr int kDecodeRingCtasPerSm = 3;
 
 constexpr int kSelectMaxQHeads = 128;
 constexpr int kSelectTokTile = 16;   // smallest tile of the logits kernel (sizes the workspace)
