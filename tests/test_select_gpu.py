@@ -243,3 +243,37 @@ def test_select_coordinate_structures(name):
         rel_err = np.abs(score[b] - ref) / ref
         assert rel_err.max() <= 1e-4, (b, rel_err.max())
         assert np.array_equal(idx[b], _topk_by(score[b].astype(np.float64), k))
+
+
+# Shapes whose logits work divides unevenly over the persistent grid of a
+# 152-SM GB300 (two CTAs per SM): the last items are split in halves by KV
+# heads, here over groups of 3 KV heads (halves of 2 and 1) and 5 (3 and 2,
+# then 2 and 1 for the group of 2). The split items are the last ones, i.e.
+# the last sequences', which the test checks against the oracle.
+HALVES = {
+    "halves-h6": (Workload(name="halves-h6", n_layers=1, n_kv_heads=6, head_dim=128,
+                           sections=(16, 24, 24), n_seqs=24, grids=((1, 40, 40),), selection="random",
+                           cache="contiguous", cur_pos=("uniform", 2000, 9000), extra=(1, 1, 1, 40)), 12),
+    "halves-h5-d64": (Workload(name="halves-h5-d64", n_layers=1, n_kv_heads=5, head_dim=64,
+                               sections=(8, 12, 12), n_seqs=20, grids=((1, 40, 50),), selection="random",
+                               cache="contiguous", cur_pos=("uniform", 2000, 9000), extra=(1, 1, 1, 40)), 15),
+}
+
+
+@pytest.mark.parametrize("name", sorted(HALVES))
+def test_select_leftover_halves(name):
+    wl, Hq = HALVES[name]
+    batch = make_batch(wl, device=DEV)
+    B, M, D = wl.n_seqs, wl.n_tokens, wl.head_dim
+    k = 100
+    g = torch.Generator(device=DEV)
+    g.manual_seed(29)
+    q = (3.0 * torch.randn((B, Hq, D), generator=g, device=DEV)).to(torch.bfloat16)
+    idx, _, _, score = _select(batch, 0, Hq, k, q, batch.p_txt)
+    qv = O.bf16_bits_to_f64(q.view(torch.int16).cpu().numpy())
+    coords = batch.coords.cpu().numpy()
+    for b in (0, B - 3, B - 2, B - 1):
+        k_raw = batch.store_k[b, 0].view(torch.int16).cpu().numpy()
+        ref = O.ads_relevance(qv[b], int(batch.p_txt[b]), k_raw, coords[b], D, wl.sections, wl.theta)
+        assert (np.abs(score[b] - ref) / ref).max() <= 1e-4, b
+        assert np.array_equal(idx[b], _topk_by(score[b].astype(np.float64), k))
