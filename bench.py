@@ -102,6 +102,9 @@ def parse():
                          "(auto: when a step moves less than 4x the L2 size)")
     ap.add_argument("--no-paper-shape", action="store_true",
                     help="skip the Table 3 shape latencies of the revisit path")
+    ap.add_argument("--no-next-rows", action="store_true",
+                    help="skip the NEXT rows' numbers (selection, small-batch decode, one "
+                         "revisit end to end) in the revisit path's line")
     return ap.parse_args()
 
 
@@ -607,6 +610,9 @@ def run_gpu(args):
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(wl, wl.n_layers, n_samples=args.cpu_samples, device=dev)
+    rows = None
+    if rank == 0 and world == 1 and not args.no_next_rows:
+        rows = next_rows(args)
 
     if rank == 0:
         R = batch.n_revisits
@@ -628,7 +634,7 @@ def run_gpu(args):
                  "roofline kernel timed over %d further steps through prcr_plan + "
                  "prcr_rebind_apply" % (min(K, 20) if split else 0),
             roofline=roof, cpu_baseline=cpu, selection_manifest=manifest,
-            paper_shape=shapes,
+            paper_shape=shapes, next_rows=rows,
             e2e=dict(value=e2e_value, unit=UNIT, h2d_bytes_per_step=rv.h2d_bytes(),
                      d2h_bytes_per_step=rv.d2h_bytes(), steps=args.e2e_steps),
             gpu_launches=per_step * K,
@@ -640,6 +646,51 @@ def run_gpu(args):
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def next_rows(args):
+    """The NEXT rows' headline numbers, measured inside the default run (one
+    GPU, rank 0) by the same code as their own --path lines, whose JSON
+    lines are captured rather than printed: the attention-driven selection on
+    the workload's shape (one layer of the store; the selection reads one
+    layer), from the raw store and from the position-bound cache, the
+    small-batch first decode step (paper 8B shape: one sequence of 933 slots
+    x 36 layers) and one whole revisit (select, rebind + inject, decode) of
+    the paper 8B shape at K = 32 replayed as a CUDA graph."""
+    import contextlib
+    import io
+
+    def run(fn, **kw):
+        ns = argparse.Namespace(**vars(args))
+        ns.__dict__.update(dict(no_cpu_baseline=True, seqs=0, layers=0, graph=False,
+                                flush="auto", select_source="raw"))
+        ns.__dict__.update(kw)
+        buf = io.StringIO()
+        with contextlib.redirect_stdout(buf):
+            fn(ns)
+        for line in buf.getvalue().splitlines():
+            if line.startswith("{"):
+                return json.loads(line)
+        return None
+
+    out = {}
+    for src in ("raw", "cache"):
+        d = run(run_select_path, path="select", layers=1, steps=50, warmup=5, select_source=src)
+        out[f"select_{src}"] = dict(workload=d["config"]["workload"], ms=d["ms_per_step"],
+                                    gbs=d["value"], frac=d["roofline"]["frac"],
+                                    l2=d["config"]["l2"])
+    d = run(run_decode_path, path="decode", workload="paper-8b-k32", seqs=1, max_len=933,
+            steps=200, warmup=10)
+    out["decode_1x933"] = dict(us=1e3 * d["ms_per_step"], gbs=d["value"], frac=d["roofline"]["frac"],
+                               l2=d["config"].get("l2"))
+    d = run(run_pipeline_path, path="pipeline", workload="paper-8b-k32", steps=200, warmup=10,
+            graph=True)
+    out["revisit_k32_graph"] = dict(us=1e3 * d["ms_per_step"], timing="one CUDA graph per %d steps"
+                                    % args.graph_inner)
+    out["measured_by"] = ("bench.py's select / decode / pipeline paths, run inside this call "
+                          "(parity: tests/test_select*_gpu.py, test_decode_gpu.py, "
+                          "test_pipeline_gpu.py)")
+    return out
 
 
 def _timed(fn, steps, warmup, local, flush):

@@ -53,6 +53,11 @@ def test_gpu_arm_line():
     for k in ("sm_mhz", "sm_max_mhz", "reasons"):
         assert k in d["clocks"], k
     assert d["config"]["workload"] == "tiny"
+    rows = d["next_rows"]
+    for k in ("select_raw", "select_cache", "decode_1x933", "revisit_k32_graph"):
+        assert k in rows, k
+    assert rows["select_raw"]["ms"] > 0 and rows["select_cache"]["gbs"] > 0
+    assert rows["decode_1x933"]["us"] > 0 and rows["revisit_k32_graph"]["us"] > 0
 
 
 @pytest.mark.gpu
