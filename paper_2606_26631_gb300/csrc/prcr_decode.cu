@@ -276,16 +276,21 @@ __global__ void __launch_bounds__(kDecodeThreads, 3) decode_kernel(const __grid_
 // per iteration; the next 16 slots' K rows (registers) and V rows (shared
 // memory) are requested right after the current QK, so they are in flight
 // during the softmax and P V of the current slots.
-//   QK:  S (16 heads x 8 slots, rows >= g zero) = Q (16 x 16 dims) x K^T, two
-//        n-tiles of 8 slots, D/16 k-steps. The dot product does not depend on
-//        the order of the dimensions, so k-step j of lane group t uses the four
-//        dimensions t*D/4 + 4j .. +3: each lane then loads its slot's 64
-//        contiguous bytes (D = 128) straight into B fragments.
+//   QK:  S^T (16 slots x 8 heads, columns >= g zero) = K (16 slots x 16 dims)
+//        x Q^T, D/16 k-steps: the slots fill all 16 MMA rows (with the heads
+//        as rows only g of 16 would be used, and two n-tiles of 8 slots take
+//        twice the MMAs). The dot product does not depend on the order of the
+//        dimensions, so k-step j of lane group t uses the four dimensions
+//        t*D/4 + 4j .. +3: each lane then loads its two slots' (g and g + 8)
+//        64 contiguous bytes (D = 128) straight into A fragments, and the
+//        query's fragments are the B operand. Lane (g, t) holds slots g and
+//        g + 8 of heads 2t, 2t+1, so it keeps those two heads' online-softmax
+//        state (reduced over the eight lanes of one t).
 //   PV:  O^T (16 dims x 8 heads) += V^T (16 dims x 16 slots) x P^T (16 slots x
-//        8 heads). The QK accumulator of lane (g, t) holds head g at slots 2t,
-//        2t+1 (tile 0) and 2t+8, 2t+9 (tile 1): exactly the P^T B fragment.
-//        V tiles are staged in shared memory with cp.async (double-buffered)
-//        and read as A fragments with ldmatrix.trans.
+//        8 heads): P^T's B fragments are S^T's 8 x 8 blocks transposed in
+//        registers (movmatrix); O^T's columns are the lane's own heads 2t,
+//        2t+1. V tiles are staged in shared memory with cp.async
+//        (double-buffered) and read as A fragments with ldmatrix.trans.
 // bf16 operands hold only 8 significant bits, so the float32 query and the
 // float32 probabilities are each split into a bf16 head and a bf16 remainder
 // (two MMAs each): products stay exact and the result keeps ~16 bits per
@@ -294,6 +299,15 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int sr
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
                  "r"(src_bytes)
                  : "memory");
+}
+
+// Transpose of an 8 x 8 matrix of 16-bit values held as mma fragments
+// (lane 4 r + c holds row r, columns 2c and 2c + 1): afterwards the lane holds
+// row r, columns 2c and 2c + 1 of the transpose.
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x) {
+    uint32_t y;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+    return y;
 }
 
 // One CTA per (sequence, layer, chunk) takes all KV heads of the layer, its
@@ -413,7 +427,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
     const uint32_t wv_s = uint32_t(__cvta_generic_to_shared(wv));
 
     for (int kh = kh0 + warp; kh < kh1; kh += nwarps) {
-        // Q A-fragments (rows = heads of the group; rows >= g and 8..15 are zero)
+        // the query B fragments (columns = heads of the group; columns >= g are zero)
         uint32_t qh[KS][2], ql[KS][2];
         {
             const bool hv = gid < g;
@@ -429,7 +443,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
         float o[KS][4];
 #pragma unroll
         for (int mt = 0; mt < KS; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.0f;
-        float m_run = -INFINITY, l_run = 0.0f;
+        float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.0f, 0.0f};  // heads 2t, 2t + 1
         const uint16_t* kbase = a.cache_k + lstride + int64_t(kh) * D;
         const uint16_t* vbase = a.cache_v + lstride + int64_t(kh) * D;
 
@@ -484,58 +498,60 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
             const bool more = s0 + 16 < s_end;
             const int32_t blk_next = more ? block_of(s0 + 16) : 0;
 
-            // S = Q K^T for the two slot tiles
-            float sc[2][4];
+            // S^T (16 slots x 8 columns = the group's query heads, columns >= g
+            // zero) = K Q^T: this lane's slots gid (kn[0]) and 8 + gid (kn[1])
+            // are the A rows, the query fragments the B operand unchanged; the
+            // query's head and remainder products in two chains
+            float sh[4] = {0.0f, 0.0f, 0.0f, 0.0f}, sl_[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-            for (int nt = 0; nt < 2; ++nt) {
-                sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.0f;
-#pragma unroll
-                for (int j = 0; j < KS; ++j) {
-                    const uint4& w = kn[nt][j >> 1];
-                    const uint32_t b0 = (j & 1) ? w.z : w.x;
-                    const uint32_t b1 = (j & 1) ? w.w : w.y;
-                    mma_16816(sc[nt], qh[j][0], 0u, qh[j][1], 0u, b0, b1);
-                    mma_16816(sc[nt], ql[j][0], 0u, ql[j][1], 0u, b0, b1);
-                }
+            for (int j = 0; j < KS; ++j) {
+                const uint4& w0 = kn[0][j >> 1];
+                const uint4& w1 = kn[1][j >> 1];
+                const uint32_t a0 = (j & 1) ? w0.z : w0.x, a2 = (j & 1) ? w0.w : w0.y;
+                const uint32_t a1 = (j & 1) ? w1.z : w1.x, a3 = (j & 1) ? w1.w : w1.y;
+                mma_16816(sh, a0, a1, a2, a3, qh[j][0], qh[j][1]);
+                mma_16816(sl_, a0, a1, a2, a3, ql[j][0], ql[j][1]);
             }
             // the next tile's K and V are in flight during the softmax and P V
             if (more) fetch(s0 + 16, st ^ 1, blk_next);
 
-            // online softmax of head row gid over the 16 slots
-            float v[4] = {sc[0][0], sc[0][1], sc[1][0], sc[1][1]};
-            const int sl[4] = {2 * t, 2 * t + 1, 8 + 2 * t, 9 + 2 * t};
-            float mx = -INFINITY;
+            // online softmax of this lane's heads 2t, 2t + 1 (columns) over the
+            // 16 slots: the eight lanes of one t hold them, two slots each
+            const bool oka = (mask >> gid) & 1u, okb = (mask >> (8 + gid)) & 1u;
+            float pa[2], pb[2], alpha[2];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                if (!((mask >> sl[i]) & 1u)) v[i] = -INFINITY;
-                mx = fmaxf(mx, v[i]);
+            for (int hh = 0; hh < 2; ++hh) {
+                const float va = oka ? sh[hh] + sl_[hh] : -INFINITY;
+                const float vb = okb ? sh[2 + hh] + sl_[2 + hh] : -INFINITY;
+                float mx = fmaxf(va, vb);
+                mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 4));
+                mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 8));
+                mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 16));
+                const float m_new = fmaxf(m_run[hh], mx);
+                // arguments are <= 0: __expf's error (a few ulp) is far inside
+                // the float32 accumulation's
+                alpha[hh] = m_new == -INFINITY ? 1.0f : __expf(m_run[hh] - m_new);
+                pa[hh] = va == -INFINITY ? 0.0f : __expf(va - m_new);
+                pb[hh] = vb == -INFINITY ? 0.0f : __expf(vb - m_new);
+                float ps = pa[hh] + pb[hh];
+                ps += __shfl_xor_sync(kFull, ps, 4);
+                ps += __shfl_xor_sync(kFull, ps, 8);
+                ps += __shfl_xor_sync(kFull, ps, 16);
+                l_run[hh] = l_run[hh] * alpha[hh] + ps;
+                m_run[hh] = m_new;
             }
-            mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 1));
-            mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 2));
-            const float m_new = fmaxf(m_run, mx);
-            // arguments are <= 0: __expf's error (a few ulp) is far inside
-            // the float32 accumulation's
-            const float alpha = m_new == -INFINITY ? 1.0f : __expf(m_run - m_new);
-            float ps = 0.0f;
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                v[i] = v[i] == -INFINITY ? 0.0f : __expf(v[i] - m_new);
-                ps += v[i];
-            }
-            ps += __shfl_xor_sync(kFull, ps, 1);
-            ps += __shfl_xor_sync(kFull, ps, 2);
-            l_run = l_run * alpha + ps;
-            m_run = m_new;
-            // O^T columns are heads 2t, 2t+1: their rescale factors live in rows 2t, 2t+1
-            const float a0 = __shfl_sync(kFull, alpha, (2 * t) * 4);
-            const float a1 = __shfl_sync(kFull, alpha, (2 * t + 1) * 4);
+            // O^T columns are heads 2t, 2t + 1: this lane's own factors
 #pragma unroll
             for (int mt = 0; mt < KS; ++mt) {
-                o[mt][0] *= a0; o[mt][1] *= a1; o[mt][2] *= a0; o[mt][3] *= a1;
+                o[mt][0] *= alpha[0]; o[mt][1] *= alpha[1]; o[mt][2] *= alpha[0]; o[mt][3] *= alpha[1];
             }
-            uint32_t pb0h, pb0l, pb1h, pb1l;
-            split_bf16x2(v[0], v[1], pb0h, pb0l);
-            split_bf16x2(v[2], v[3], pb1h, pb1l);
+            // P^T as B fragments: the 8 x 8 blocks (slots 0..7 | 8..15) x heads
+            // held as (slot gid; heads 2t, 2t + 1) are transposed in registers
+            uint32_t m1h, m1l, m2h, m2l;
+            split_bf16x2(pa[0], pa[1], m1h, m1l);
+            split_bf16x2(pb[0], pb[1], m2h, m2l);
+            const uint32_t pb0h = movmatrix_trans(m1h), pb1h = movmatrix_trans(m2h);
+            const uint32_t pb0l = movmatrix_trans(m1l), pb1l = movmatrix_trans(m2l);
 
             // O^T += V^T P^T
             if (more) asm volatile("cp.async.wait_group 1;" ::: "memory");
@@ -557,10 +573,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
         }
 
         // heads 2t, 2t+1 of this lane's O^T columns
-        const float l0 = __shfl_sync(kFull, l_run, (2 * t) * 4);
-        const float l1 = __shfl_sync(kFull, l_run, (2 * t + 1) * 4);
-        const float m0 = __shfl_sync(kFull, m_run, (2 * t) * 4);
-        const float m1 = __shfl_sync(kFull, m_run, (2 * t + 1) * 4);
+        const float l0 = l_run[0], l1 = l_run[1], m0 = m_run[0], m1 = m_run[1];
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
             const int h = 2 * t + hh;
@@ -603,24 +616,11 @@ __global__ void __launch_bounds__(kDecodeThreads, 3)
 // not for its async copies). Two stages keep the CTA's shared memory at
 // 66 KB (three CTAs, twelve warps per SM); more warps per SM hide more of
 // each warp's latency chain than a deeper ring would.
-// QK is S^T = K Q^T (the tile's 16 slots as the MMA rows, the GQA group's
-// query heads as the 8 columns: one MMA per k-step and query piece, half of
-// what Q K^T with the heads as rows takes), and PV is O^T += V^T P^T as in
-// decode_mma_kernel, P^T's fragments transposed from S^T's in registers
-// (movmatrix); each lane keeps the online-softmax state of the two heads
-// whose O^T columns it holds. The key dimensions are permuted per lane group
-// as in decode_mma_kernel, here with lane group t reading 16-byte chunks t,
-// t + 4, ... of its slot's K row, and chunk c of slot s is stored at
-// c ^ 4 (s & 1) so that those reads are free of bank conflicts.
-// Transpose of an 8 x 8 matrix of 16-bit values held as mma fragments
-// (lane 4 r + c holds row r, columns 2c and 2c + 1): afterwards the lane holds
-// row r, columns 2c and 2c + 1 of the transpose.
-__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x) {
-    uint32_t y;
-    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
-    return y;
-}
-
+// The arithmetic is that of decode_mma_kernel (S^T = K Q^T, O^T += V^T P^T,
+// the same online softmax); the key dimensions are permuted per lane group as
+// there, here with lane group t reading 16-byte chunks t, t + 4, ... of its
+// slot's K row, and chunk c of slot s is stored at c ^ 4 (s & 1) so that
+// those reads are free of bank conflicts.
 constexpr int kRingWarps = kDecodeRingWarps;
 constexpr int kRingStages = 2;
 // rounds of eight query pairs per thread: the CTA's query heads are at most
