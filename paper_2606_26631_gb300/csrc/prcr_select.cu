@@ -537,10 +537,10 @@ __global__ void __launch_bounds__(NW * 32, 2) ads_logits_mma_kernel(const __grid
 // head and a bf16 remainder (two MMAs per k-step). The key dimensions are
 // permuted per lane group so that a lane loads its two tokens' 64 contiguous
 // bytes each straight into A fragments. The next item's rows are loaded
-// right after this item's MMAs, the rows of the one after that requested
-// into L2. An item writes its 16 logits per head (the softmax statistics
-// are left to the normaliser kernel); a token without a readable row gets
-// logit -inf.
+// during this item's MMAs (each 16-byte run as soon as the register it goes
+// into is used), the rows of the one after that requested into L2. An item
+// writes its 16 logits per head (the softmax statistics are left to the
+// normaliser kernel); a token without a readable row gets logit -inf.
 template <int D>
 __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
     ads_logits_cache_kernel(const __grid_constant__ SelectArgs a) {
@@ -575,52 +575,84 @@ __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
     // token 16 j + (lane & 15) of sequence b, or -1 (past the end, or no
     // readable row). Computed once per item, when its rows are requested.
     const int64_t layer_off = int64_t(a.layer) * a.cache_layer_stride;
-    auto row_of = [&](const Item& x) -> int64_t {
+    // The row lookup in two halves, one item apart: start() forms the slot of
+    // this lane's token and issues its block-table load (paged caches), whose
+    // value finish() uses an item later, when the lookup's dependent loads
+    // have long returned. The sequence's first image slot is kept per
+    // sequence (items run sequence-major).
+    struct RowReq {
+        int64_t slot;  // -1: no row
+        int32_t blk;
+    };
+    int s0_b = -1;
+    int32_t s0_v = 0;
+    auto row_start = [&](const Item& x, RowReq& q) {
+        q.slot = -1;
+        q.blk = 0;
         const int m = 16 * x.j + (lane & 15);
-        if (m >= M) return -1;
-        const int64_t slot = int64_t(a.img_slot0[x.b]) + m;
+        if (m >= M) return;
+        if (x.b != s0_b) {
+            s0_b = x.b;
+            s0_v = a.img_slot0[x.b];
+        }
+        const int64_t slot = int64_t(s0_v) + m;
         if (slot < 0 || slot >= a.cache_capacity) {
             err |= PRCR_ST_CAPACITY;
-            return -1;
+            return;
         }
+        q.slot = slot;
+        if (a.cache_kind != PRCR_CACHE_CONTIGUOUS) {
+            // block index by a 32-bit division when the slot fits in 31 bits
+            // (a 64-bit division costs several times as many instructions as
+            // the rest of a row lookup)
+            const int64_t lb = slot <= INT32_MAX ? int64_t(uint32_t(slot) / uint32_t(a.block_size))
+                                                 : slot / a.block_size;
+            q.blk = a.block_table[int64_t(x.b) * a.bt_stride + lb];
+        }
+    };
+    auto row_finish = [&](const Item& x, const RowReq& q) -> int64_t {
+        if (q.slot < 0) return -1;
         int64_t row;
         if (a.cache_kind == PRCR_CACHE_CONTIGUOUS) {
-            row = int64_t(x.b) * a.cache_seq_stride + slot * a.cache_slot_stride;
+            row = int64_t(x.b) * a.cache_seq_stride + q.slot * a.cache_slot_stride;
         } else {
-            // block index and offset by a 32-bit division when the slot fits
-            // in 31 bits (a 64-bit division costs several times as many
-            // instructions as the rest of a row lookup)
-            int64_t lb, off;
-            if (slot <= INT32_MAX) {
-                const uint32_t us = uint32_t(slot), ubs = uint32_t(a.block_size);
-                lb = us / ubs;
-                off = us - uint32_t(lb) * ubs;
-            } else {
-                lb = slot / a.block_size;
-                off = slot - lb * a.block_size;
-            }
-            const int32_t blk = a.block_table[int64_t(x.b) * a.bt_stride + lb];
-            if (blk < 0 || blk >= a.n_blocks) {
+            if (q.blk < 0 || q.blk >= a.n_blocks) {
                 err |= PRCR_ST_NO_BLOCK;
                 return -1;
             }
-            row = int64_t(blk) * a.cache_block_stride + off * a.cache_slot_stride;
+            const int64_t off = q.slot <= INT32_MAX ? int64_t(uint32_t(q.slot) % uint32_t(a.block_size))
+                                                    : q.slot % a.block_size;
+            row = int64_t(q.blk) * a.cache_block_stride + off * a.cache_slot_stride;
         }
         return row + layer_off;
+    };
+    auto row_of = [&](const Item& x) -> int64_t {
+        RowReq q;
+        row_start(x, q);
+        return row_finish(x, q);
     };
     uint4 kn[2][LV];
     uint32_t mask_n = 0u;
     // loads an item's 16 key rows (row: this lane's token, from row_of). A
     // token without a row reads the cache's first row instead: its logit is
     // set to -inf whatever the row holds (tokens are separate MMA rows).
-    auto fetch = [&](int64_t row, int kh) {
-        mask_n = __ballot_sync(0xffffffffu, row >= 0) & 0xffffu;
+    // this lane's two token rows (tokens gid and gid + 8) of an item, and the
+    // item's row mask
+    auto rows_of = [&](int64_t row, int kh, const uint16_t* (&kp)[2]) -> uint32_t {
+        const uint32_t m = __ballot_sync(0xffffffffu, row >= 0) & 0xffffu;
         const int64_t r0 = (row >= 0 ? row : 0) + int64_t(kh) * D;
 #pragma unroll
-        for (int nt = 0; nt < 2; ++nt) {
-            const uint16_t* kp = a.cache_k + __shfl_sync(0xffffffffu, r0, nt * 8 + gid) + t * (D / 4);
+        for (int nt = 0; nt < 2; ++nt)
+            kp[nt] = a.cache_k + __shfl_sync(0xffffffffu, r0, nt * 8 + gid) + t * (D / 4);
+        return m;
+    };
+    auto fetch = [&](int64_t row, int kh) {
+        const uint16_t* kp[2];
+        mask_n = rows_of(row, kh, kp);
 #pragma unroll
-            for (int u = 0; u < LV; ++u) kn[nt][u] = ld_stream(kp + 8 * u);
+        for (int nt = 0; nt < 2; ++nt) {
+#pragma unroll
+            for (int u = 0; u < LV; ++u) kn[nt][u] = ld_stream(kp[nt] + 8 * u);
         }
     };
     // the rows of the item after next are requested into L2 (lanes 0..15,
@@ -649,11 +681,13 @@ __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
     pf = nxt;
     advance(pf);
     int64_t row_nxt = -1, row_pf = -1;
+    RowReq req_pf = {-1, 0};  // the started lookup of pf
     if (i_beg < i_end) fetch(row_of(cur), cur.kh);
     if (i_beg + 1 < i_end) {
         row_nxt = row_of(nxt);
         request(row_nxt, nxt.kh);
     }
+    if (i_beg + 2 < i_end) row_start(pf, req_pf);
     for (int64_t left = i_end - i_beg; left > 0; --left) {
         const int b = cur.b, kh = cur.kh, j = cur.j;
         if (b != cur_b || kh != cur_kh) {
@@ -697,6 +731,10 @@ __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
         // zero) = K Q^T: rows gid (kn[0]) and gid + 8 (kn[1]) are this lane's
         // tokens, and the query fragments serve as the B operand unchanged
         const uint32_t mask = q_ok ? mask_n : 0u;
+        // the next item's rows, each 16-byte run requested as soon as this
+        // item's MMAs have used the registers it goes into
+        const uint16_t* kp[2] = {a.cache_k, a.cache_k};
+        if (left > 1) mask_n = rows_of(row_nxt, nxt.kh, kp);
         float c[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
         for (int k = 0; k < KS; ++k) {
@@ -706,12 +744,18 @@ __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
             const uint32_t a1 = (k & 1) ? w1.z : w1.x, a3 = (k & 1) ? w1.w : w1.y;
             mma_16816(c, a0, a1, a2, a3, qh[k][0], qh[k][1]);
             mma_16816(c, a0, a1, a2, a3, ql[k][0], ql[k][1]);
+            if ((k & 1) && left > 1) {
+                kn[0][k >> 1] = ld_stream(kp[0] + 8 * (k >> 1));
+                kn[1][k >> 1] = ld_stream(kp[1] + 8 * (k >> 1));
+            }
         }
-        if (left > 1) fetch(row_nxt, nxt.kh);
+        Item pf2 = pf;  // the item after pf: its lookup starts now
+        advance(pf2);
         if (left > 2) {
-            row_pf = row_of(pf);
+            row_pf = row_finish(pf, req_pf);
             request(row_pf, pf.kh);
         }
+        if (left > 3) row_start(pf2, req_pf);
 
         // token gid: heads 2t, 2t + 1 in c[0], c[1]; token gid + 8 in c[2], c[3]
         // (the softmax statistics come from the normaliser kernel, one pass
@@ -736,7 +780,7 @@ __global__ void __launch_bounds__(256, D > 128 ? 1 : 2)
         cur = nxt;
         nxt = pf;
         row_nxt = row_pf;
-        advance(pf);
+        pf = pf2;
     }
     if (err) atomicOr(a.status, err);
 }
