@@ -292,7 +292,6 @@ __device__ __forceinline__ uint32_t word_of(const uint4& v, int i) {
 template <int D, int NW>
 __global__ void __launch_bounds__(NW * 32, 2) ads_logits_mma_kernel(const __grid_constant__ SelectArgs a) {
     pdl_allow();
-    pdl_wait();
     constexpr int P = D / 2, KS = D / 8, NR = KS / 8;  // k-steps; 16-byte runs per half row
     constexpr int T = 16 * NW;                         // tokens per work item
     static_assert(NR == 1 || NR == 2, "head_dim 64 or 128");
@@ -312,13 +311,16 @@ __global__ void __launch_bounds__(NW * 32, 2) ads_logits_mma_kernel(const __grid
         if (pair_axis(i, a.layout, a.sec_t, a.sec_h, a.sec_w) == 2) sincos_coord(8, a.turn_freq[i], &r.y, &r.x);
         r8_s[i] = r;
     }
-    __syncthreads();
     // axis of this lane's pair at each k-step, two bits each
     uint32_t axes = 0u;
 #pragma unroll
     for (int s = 0; s < KS; ++s)
         axes |= uint32_t(pair_axis(32 * (s / 8) + 8 * tq + s % 8, a.layout, a.sec_t, a.sec_h,
                                    a.sec_w)) << (2 * s);
+    // the tables above come from the arguments alone: they are set up while
+    // the grid this one depends on finishes; every global input is read after
+    pdl_wait();
+    __syncthreads();
     // Schedule: q = total / grid whole items per CTA, a contiguous run. The
     // R = total - q * grid items left over would make R CTAs run q + 1 items;
     // when 2 R <= grid they are split instead into halves by KV heads, one
