@@ -675,7 +675,7 @@ def next_rows(args):
 
     out = {}
     for src in ("raw", "cache"):
-        d = run(run_select_path, path="select", layers=1, steps=50, warmup=5, select_source=src)
+        d = run(run_select_path, path="select", layers=1, steps=200, warmup=10, select_source=src)
         out[f"select_{src}"] = dict(workload=d["config"]["workload"], ms=d["ms_per_step"],
                                     gbs=d["value"], frac=d["roofline"]["frac"],
                                     l2=d["config"]["l2"])
