@@ -821,9 +821,10 @@ __global__ void __launch_bounds__(256) ads_norm_kernel(const __grid_constant__ S
 }
 
 // Softmax normaliser of each (sequence, query head) straight from its logits
-// (the tensor-core logits kernel writes no tile statistics): every thread
-// keeps a running (max, sum of exp) over sixteen logits at a time (four
-// 16-byte loads when the row is 16-byte aligned), and the block merges them.
+// (the tensor-core and cached-key logits kernels write no tile statistics):
+// every thread keeps a running (max, sum of exp) over sixteen logits at a
+// time, all of a round's loads requested at once (16-byte loads when the row
+// is 16-byte aligned), and the block merges them.
 __device__ __forceinline__ void merge_max_sum(float& m, float& s, float m2, float s2) {
     const float mn = fmaxf(m, m2);
     if (mn == -INFINITY) return;
@@ -835,8 +836,8 @@ __global__ void __launch_bounds__(256) ads_norm_logits_kernel(const __grid_const
     pdl_allow();
     pdl_wait();
     __shared__ float s_m[8], s_z[8];
-    const int hq = blockIdx.x, b = blockIdx.y, M = a.n_tokens;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int hq = blockIdx.x, b = blockIdx.y, M = a.n_tokens, NT = blockDim.x;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = NT >> 5;
     const float* lg = a.logits + (int64_t(b) * a.n_q_heads + hq) * M;
     float mx = -INFINITY, z = 0.0f;
     // sixteen logits (-inf past the end) into the running (max, sum of exp)
@@ -851,38 +852,33 @@ __global__ void __launch_bounds__(256) ads_norm_logits_kernel(const __grid_const
         z = (mx == -INFINITY ? 0.0f : z * __expf(mx - cm)) + cz;
         mx = cm;
     };
-    int i = 0;  // logits [0, i) done
     if ((M & 3) == 0) {
+        // 16-byte loads, eight per thread requested at once (the launch sizes
+        // the block so that one round covers the row where it can)
         const float4* l4 = reinterpret_cast<const float4*>(lg);
-        for (; i + 8192 <= M; i += 8192) {  // 256 threads x 32 logits, all requested at once
+        const int M4 = M >> 2;
+        for (int i4 = 0; i4 < M4; i4 += 8 * NT) {
             float x[2][16];
 #pragma unroll
             for (int u = 0; u < 8; ++u) {
-                const float4 v = l4[(i >> 2) + u * 256 + threadIdx.x];
+                const int j = i4 + u * NT + threadIdx.x;
+                const float4 v = j < M4 ? l4[j] : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
                 x[u >> 2][4 * (u & 3)] = v.x; x[u >> 2][4 * (u & 3) + 1] = v.y;
                 x[u >> 2][4 * (u & 3) + 2] = v.z; x[u >> 2][4 * (u & 3) + 3] = v.w;
             }
             chunk(x[0]);
             chunk(x[1]);
         }
-        for (; i + 4096 <= M; i += 4096) {  // 256 threads x 16 logits
+    } else {
+        for (int i = 0; i < M; i += 16 * NT) {
             float x[16];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const float4 v = l4[(i >> 2) + u * 256 + threadIdx.x];
-                x[4 * u] = v.x; x[4 * u + 1] = v.y; x[4 * u + 2] = v.z; x[4 * u + 3] = v.w;
+            for (int u = 0; u < 16; ++u) {
+                const int t = i + u * NT + threadIdx.x;
+                x[u] = t < M ? lg[t] : -INFINITY;
             }
             chunk(x);
         }
-    }
-    for (; i < M; i += 4096) {
-        float x[16];
-#pragma unroll
-        for (int u = 0; u < 16; ++u) {
-            const int t = i + u * 256 + threadIdx.x;
-            x[u] = t < M ? lg[t] : -INFINITY;
-        }
-        chunk(x);
     }
 #pragma unroll
     for (int o = 16; o; o >>= 1) {
@@ -895,7 +891,7 @@ __global__ void __launch_bounds__(256) ads_norm_logits_kernel(const __grid_const
     }
     __syncthreads();
     if (threadIdx.x == 0) {
-        for (int w = 1; w < 8; ++w) merge_max_sum(mx, z, s_m[w], s_z[w]);
+        for (int w = 1; w < nw; ++w) merge_max_sum(mx, z, s_m[w], s_z[w]);
         float* nrm = a.norm + (int64_t(b) * a.n_q_heads + hq) * 2;
         nrm[0] = mx == -INFINITY ? 0.0f : mx;
         nrm[1] = mx == -INFINITY ? 0.0f : 1.0f / (z * float(a.n_q_heads));
@@ -935,12 +931,12 @@ __global__ void __launch_bounds__(256) ads_relevance_kernel(const __grid_constan
         for (; h < Hq; ++h) r[0] = fmaf(__expf(lg[int64_t(h) * M] - s_n[2 * h]), s_n[2 * h + 1], r[0]);
     } else if ((M & 3) == 0) {
         int h = 0;
-        for (; h + 8 <= Hq; h += 8) {
-            float4 x[8];
+        for (; h + 16 <= Hq; h += 16) {  // sixteen heads' logits requested together
+            float4 x[16];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) x[u] = *reinterpret_cast<const float4*>(lg + int64_t(h + u) * M);
+            for (int u = 0; u < 16; ++u) x[u] = *reinterpret_cast<const float4*>(lg + int64_t(h + u) * M);
 #pragma unroll
-            for (int u = 0; u < 8; ++u) {
+            for (int u = 0; u < 16; ++u) {
                 const float mh = s_n[2 * (h + u)], wh = s_n[2 * (h + u) + 1];
                 r[0] = fmaf(__expf(x[u].x - mh), wh, r[0]);
                 r[1 % TPT] = fmaf(__expf(x[u].y - mh), wh, r[1 % TPT]);
@@ -1176,8 +1172,14 @@ cudaError_t launch_logits_mma(const SelectArgs& a, int n_seqs, int sms, cudaStre
 // The normalisers, relevances and selection after a logits kernel.
 static cudaError_t launch_select_tail(const SelectArgs& a, int n_seqs, cudaStream_t stream,
                                       bool norm_from_logits = false) {
-    cudaError_t e = launch_pdl(norm_from_logits ? ads_norm_logits_kernel : ads_norm_kernel,
-                               dim3(a.n_q_heads, n_seqs, 1), dim3(256), 0, stream, a);
+    // the normaliser from the logits: about 32 logits per thread, one round
+    // up to 256 threads (wider blocks would take large grids past one wave)
+    int nt = int(((a.n_tokens + 31) / 32 + 31) / 32 * 32);
+    nt = nt < 64 ? 64 : (nt > 256 ? 256 : nt);
+    cudaError_t e = norm_from_logits
+                        ? launch_pdl(ads_norm_logits_kernel, dim3(a.n_q_heads, n_seqs, 1), dim3(nt), 0,
+                                     stream, a)
+                        : launch_pdl(ads_norm_kernel, dim3(a.n_q_heads, n_seqs, 1), dim3(256), 0, stream, a);
     if (e != cudaSuccess) return e;
     // four tokens per thread once the grid fills the GPU a few times over
     if (int64_t(n_seqs) * a.n_tokens >= (int64_t(1) << 19))
