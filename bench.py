@@ -45,9 +45,9 @@ SPEC_HBM_GBS = 8000.0
 # workload, from an ncu capture; valid only for the kernel source it was
 # measured on (its sha256 prefix), reported as null otherwise.
 TRAFFIC = {
-    # captured on the stress shape cut to 2 sequences (8,192 tokens: 1,194,926,336 B
-    # read + 1,150,225,920 B written) and scaled by the 16x more tokens of a full launch
-    ("stress", "a12a4266b6a504aa"): 37522436096,
+    # captured on the stress shape cut to 2 sequences (8,192 tokens: 1,193,440,000 B
+    # read + 1,150,144,256 B written) and scaled by the 16x more tokens of a full launch
+    ("stress", "46dd442ca336fc40"): 37497348096,
 }
 
 # the Table 3 shapes (Qwen3-VL-8B dimensions, a 768-token image, K = 32 and
